@@ -1,0 +1,212 @@
+"""fp64 CPU oracle for forced-weight subset evaluation -- TEST INFRASTRUCTURE.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline and
+reference legs may import this package.  The product path (the CUDA library and
+its binding) never does, and the oracle never imports the product: the two
+share nothing but the seeded generators in ``workloads``.
+
+The arithmetic lives in ``fw_oracle.c`` (plain C, double precision, straight
+from the paper's definitions).  This module compiles it with gcc and marshals
+numpy arrays into it.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "fw_oracle.c")
+_SO = os.path.join(_HERE, "_fw_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle shared library (gcc, OpenMP, -O2)."""
+    if force or not os.path.exists(_SO) or os.path.getmtime(_SO) < os.path.getmtime(_SRC):
+        tmp = _SO + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c11",
+                               "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _SO)
+    return _SO
+
+
+class _Rows(C.Structure):
+    _fields_ = [("num_groups", C.c_int64), ("rows_per_group", C.c_int32), ("d", C.c_int32),
+                ("logits", C.c_void_p), ("logit_off", C.c_void_p), ("n", C.c_void_p),
+                ("v", C.c_void_p), ("v_off", C.c_void_p), ("v_dtype", C.c_int32)]
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            build()
+            L = C.CDLL(_SO)
+            vp = C.c_void_p
+            L.orc_eval_instance.argtypes = [C.c_int, C.c_int, vp, vp, vp, vp, vp, vp]
+            L.orc_dense_and_topk_gap.argtypes = [C.POINTER(_Rows), C.c_int, vp] + [vp] * 9 + [C.c_int, vp]
+            L.orc_swap_refine.argtypes = [C.POINTER(_Rows), C.c_int, vp, C.c_int, C.c_int] + [vp] * 8
+            L.orc_best_subset.argtypes = [C.POINTER(_Rows), vp, vp, vp, vp, C.c_int, vp, vp]
+            L.orc_colex_rank.argtypes = [C.c_int, vp]
+            L.orc_colex_rank.restype = C.c_uint64
+            L.orc_contour_alloc.argtypes = [vp, C.c_int, C.c_int, C.c_int, C.c_int64, C.c_int,
+                                            vp, vp, vp, vp, vp, vp]
+            L.orc_ragged_compact.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, C.c_int, vp, vp, vp, vp]
+            L.orc_num_threads.restype = C.c_int
+            _lib = L
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data_as(C.c_void_p)
+
+
+def _host(a, dtype=None):
+    """numpy view of a host array or a torch tensor (copied to the host)."""
+    if hasattr(a, "detach"):
+        import torch
+
+        t = a.detach()
+        if t.dtype == torch.bfloat16:
+            t = t.view(torch.int16)
+        a = t.cpu().numpy()
+        if a.dtype == np.int16:
+            a = a.view(np.uint16)
+    a = np.ascontiguousarray(a)
+    if dtype is not None:
+        a = np.ascontiguousarray(a, dtype=dtype)
+    return a
+
+
+class HostRows:
+    """A row batch on the host in the oracle's layout (keeps arrays alive)."""
+
+    def __init__(self, batch):
+        self.R = int(batch.rows_per_group)
+        self.d = int(batch.d)
+        self.n = _host(batch.n_host, np.int32)
+        self.logits = _host(batch.logits, np.float32)
+        self.logit_off = _host(batch.logit_off, np.int64)
+        self.v = _host(batch.v)
+        self.v_off = _host(batch.v_off, np.int64)
+        if batch.v_dtype == "bf16":
+            self.v = self.v.view(np.uint16)
+            self.v_dtype = 1
+        elif self.v.dtype == np.float64:
+            self.v_dtype = 2
+        else:
+            self.v = np.ascontiguousarray(self.v, np.float32)
+            self.v_dtype = 0
+        self.k = _host(batch.k, np.int32)
+        self.nb = int(self.k.shape[1])
+        self.num_rows = len(self.n) * self.R
+        self.max_n = int(self.n.max())
+        self.c = _Rows(len(self.n), self.R, self.d, _p(self.logits).value, _p(self.logit_off).value,
+                       _p(self.n).value, _p(self.v).value, _p(self.v_off).value, self.v_dtype)
+
+
+def eval_instance(p, v, in_A):
+    """Definition 2.1 / Lemma 2.1 quantities for one instance given by masses p,
+    points v ([n][d]) and a kept-set mask.  Returns dict."""
+    p = np.ascontiguousarray(p, np.float64)
+    v = np.ascontiguousarray(np.atleast_2d(v).reshape(len(p), -1), np.float64)
+    m = np.ascontiguousarray(in_A, np.uint8)
+    n, d = v.shape
+    mu = np.zeros(d)
+    mA = np.zeros(d)
+    out = np.zeros(6)
+    st = lib().orc_eval_instance(n, d, _p(p), _p(v), _p(m), _p(mu), _p(mA), _p(out))
+    assert st == 0, st
+    return dict(mu=mu, m_A=mA, kept_mass=out[0], dropped=out[1], gap=out[2], phi=out[3],
+                form1=out[4], form2=out[5])
+
+
+def dense_and_topk_gap(batch, words=None):
+    """a1-a4 on every row and budget.  Returns dict of numpy arrays (fp64)."""
+    H = batch if isinstance(batch, HostRows) else HostRows(batch)
+    rows, nb, d = H.num_rows, H.nb, H.d
+    words = words or (H.max_n + 31) // 32
+    out = dict(o=np.zeros((rows, d)), o_kept=np.zeros((rows, nb, d)), gap=np.zeros((rows, nb)),
+               dropped=np.zeros((rows, nb)), kept_mass=np.zeros((rows, nb)), phi=np.zeros((rows, nb)),
+               form1=np.zeros((rows, nb)), form2=np.zeros((rows, nb)),
+               kept_bits=np.zeros((rows, nb, words), np.uint32), status=np.zeros(rows, np.int32))
+    st = lib().orc_dense_and_topk_gap(C.byref(H.c), nb, _p(H.k), _p(out["o"]), _p(out["o_kept"]),
+                                      _p(out["gap"]), _p(out["dropped"]), _p(out["kept_mass"]),
+                                      _p(out["phi"]), _p(out["form1"]), _p(out["form2"]),
+                                      _p(out["kept_bits"]), words, _p(out["status"]))
+    assert st == 0, st
+    return out
+
+
+def swap_refine(batch, E, max_swaps=64):
+    H = batch if isinstance(batch, HostRows) else HostRows(batch)
+    rows, nb = H.num_rows, H.nb
+    out = dict(n_swaps=np.zeros((rows, nb), np.int32),
+               swap_out=np.full((rows, nb, max_swaps), -1, np.int32),
+               swap_in=np.full((rows, nb, max_swaps), -1, np.int32),
+               refined_gap=np.zeros((rows, nb)), topk_gap=np.zeros((rows, nb)),
+               capped=np.zeros((rows, nb), np.int32), margin=np.zeros((rows, nb)),
+               pool_margin=np.zeros((rows, nb)))
+    st = lib().orc_swap_refine(C.byref(H.c), nb, _p(H.k), int(E), int(max_swaps),
+                               _p(out["n_swaps"]), _p(out["swap_out"]), _p(out["swap_in"]),
+                               _p(out["refined_gap"]), _p(out["topk_gap"]), _p(out["capped"]),
+                               _p(out["margin"]), _p(out["pool_margin"]))
+    assert st == 0, st
+    return out
+
+
+def best_subset(batch):
+    H = batch if isinstance(batch, HostRows) else HostRows(batch)
+    rows = H.num_rows
+    kk = np.ascontiguousarray(H.k[:, 0], np.int32)
+    kmax = int(kk.max())
+    out = dict(best_rank=np.zeros(rows, np.uint64), best_gap=np.zeros(rows),
+               best_idx=np.full((rows, kmax), -1, np.int32), second_gap=np.zeros(rows),
+               topk_gap=np.zeros(rows))
+    st = lib().orc_best_subset(C.byref(H.c), _p(kk), _p(out["best_rank"]), _p(out["best_gap"]),
+                               _p(out["best_idx"]), kmax, _p(out["second_gap"]), _p(out["topk_gap"]))
+    assert st == 0, st
+    return out
+
+
+def colex_rank(combo):
+    c = np.ascontiguousarray(sorted(combo), np.int32)
+    return int(lib().orc_colex_rank(len(c), _p(c)))
+
+
+def contour_alloc(scores, floor, total_budget, uniform_s):
+    s = _host(scores, np.float32)
+    cells, T = s.shape
+    out = dict(counts=np.zeros(cells, np.int32), offsets=np.zeros(cells + 1, np.int64),
+               kept_pos=np.zeros(int(total_budget), np.int32), tau=np.zeros(1, np.float32),
+               dropped_uniform=np.zeros(cells), dropped_alloc=np.zeros(cells))
+    st = lib().orc_contour_alloc(_p(s), cells, T, int(floor), int(total_budget), int(uniform_s),
+                                 _p(out["counts"]), _p(out["offsets"]), _p(out["kept_pos"]),
+                                 _p(out["tau"]), _p(out["dropped_uniform"]), _p(out["dropped_alloc"]))
+    out["status"] = st
+    out["tau"] = float(out["tau"][0])
+    return out
+
+
+def ragged_compact(K, V, offsets, kept_pos):
+    K = _host(K)
+    V = _host(V)
+    cells, T, d = K.shape
+    off = np.ascontiguousarray(offsets, np.int64)
+    kp = np.ascontiguousarray(kept_pos, np.int32)
+    tot = int(off[-1])
+    Ko = np.zeros((tot, d), K.dtype)
+    Vo = np.zeros((tot, d), V.dtype)
+    st = lib().orc_ragged_compact(_p(K), _p(V), cells, T, d, K.dtype.itemsize, _p(off), _p(kp),
+                                  _p(Ko), _p(Vo))
+    assert st == 0, st
+    return Ko, Vo
+
+
+def num_threads() -> int:
+    return int(lib().orc_num_threads())
