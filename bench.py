@@ -1,0 +1,395 @@
+"""Benchmark: forced-weight subset evaluation on GB300.
+
+Headline workload: exact enumeration at measurement scale -- 168,192 rows in
+five groups (d = 64,128,128,128,64), n = 24 keys, k = 6 (134,596 subsets per
+row), logits Gumbel*tau + sink, V fp32.  One step runs the whole path on every
+row: softmax, top-k kept set, dense and forced-weight outputs, gap and dropped
+mass (fw_dense_and_topk_gap), the swap rule over all keys (fw_swap_refine) and
+the exact best subset (fw_best_subset).  Metric: subsets/s.
+
+Also timed in the same run (reported under "sections"): the long-row top-k
+gap workload (4,096 rows x 32,768 keys, d=128, three budgets) and ContourKV
+allocation + ragged compaction (256 cells x 32,768 tokens, d=128).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+import workloads  # noqa: E402
+
+N_KEYS, K_SEL = 24, 6
+SUBSETS_PER_ROW = math.comb(N_KEYS, K_SEL)
+ALU_OPS_PER_SUBSET = 3  # inner walk leaf: value add, carry add, running min
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm_gbs=p.get("hbm_gbs", 6800.0), bf16=p.get("bf16_tflops", 1900.0),
+                    sm_max=p.get("sm_max_mhz", 2070.0), source="measured")
+    return dict(hbm_gbs=6800.0, bf16=1900.0, sm_max=2070.0, source="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during a region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.f = None
+
+    def __enter__(self):
+        try:
+            self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.f is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.f.flush()
+        rows = []
+        with open(self.f.name) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.f.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+class L2Flush:
+    """Writes a buffer larger than L2 between timed iterations."""
+
+    def __init__(self, device):
+        self.buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+
+    def __call__(self):
+        self.buf.fill_(1)
+
+
+# ---------------------------------------------------------------- workloads
+
+class EnumWorkload:
+    """168,192 rows, n=24, k=6: the whole a1..a6 path per step."""
+
+    def __init__(self, fw, seed, device, rows_scale=1.0):
+        self.fw = fw
+        self.batches = workloads.exact_enum(seed=seed, rows_scale=rows_scale, backend="torch", device=device)
+        self.rows = [fw.rows_from_batch(b, device) for b in self.batches]
+        self.k2 = [b.k for b in self.batches]
+        self.k1 = [b.k[:, 0].contiguous() for b in self.batches]
+        self.num_rows = sum(r.num_rows for r in self.rows)
+        self.subsets = self.num_rows * SUBSETS_PER_ROW
+        self.ev = []
+
+    def step(self, time_enum=False):
+        fw = self.fw
+        outs = []
+        for rows, k2, k1 in zip(self.rows, self.k2, self.k1):
+            top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
+            sw = fw.swap_refine(rows, k2, top, E=N_KEYS, max_swaps=32)
+            if time_enum:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+            bs = fw.best_subset(rows, k1, k_max=K_SEL)
+            if time_enum:
+                e1.record()
+                self.ev.append((e0, e1, rows.num_rows))
+            outs.append((top, sw, bs))
+        return outs
+
+    def enum_times(self):
+        """(ms, rows) of every timed fw_best_subset launch."""
+        torch.cuda.synchronize()
+        r = [(a.elapsed_time(b), n) for a, b, n in self.ev]
+        self.ev = []
+        return r
+
+
+class EnumE2E:
+    """The same step through the public API from pinned host buffers: inputs are
+    copied to the device, results copied back, inside the timed region."""
+
+    def __init__(self, wl: EnumWorkload):
+        self.wl = wl
+        self.host = []
+        self.h2d = 0
+        self.d2h = 0
+        for rows in wl.rows:
+            hl = rows.logits.cpu().pin_memory()
+            hv = rows.v.cpu().pin_memory()
+            self.host.append((hl, hv))
+            self.h2d += hl.numel() * hl.element_size() + hv.numel() * hv.element_size()
+        for rows in wl.rows:
+            # per row: topk gap, dropped, refined gap, best gap, best rank (8 B), best idx (k * 4 B)
+            self.d2h += rows.num_rows * (4 * 4 + 8 + 4 * K_SEL)
+
+    def step(self):
+        wl = self.wl
+        for (hl, hv), rows in zip(self.host, wl.rows):
+            rows.logits.copy_(hl, non_blocking=True)
+            rows.v.copy_(hv, non_blocking=True)
+        outs = wl.step()
+        res = []
+        for top, sw, bs in outs:
+            res.append([t.to("cpu", non_blocking=True) for t in
+                        (top["gap"], top["dropped"], sw["refined_gap"], bs["best_gap"], bs["best_rank"],
+                         bs["best_idx"][:, :K_SEL])])
+        return res
+
+
+def time_steps(step, K, W, flush, barrier):
+    for _ in range(W):
+        step()
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    times = []
+    start_all = torch.cuda.Event(enable_timing=True)
+    end_all = torch.cuda.Event(enable_timing=True)
+    total = 0.0
+    for _ in range(K):
+        flush()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        step()
+        e1.record()
+        e1.synchronize()
+        t = e0.elapsed_time(e1)
+        times.append(t)
+        total += t
+    torch.cuda.synchronize()
+    barrier()
+    del start_all, end_all
+    return total, times
+
+
+# ------------------------------------------------------------- CPU oracle
+
+def cpu_baseline(seed, rows_per_group=40):
+    """The fp64 oracle on a bounded sample of the headline workload: the first
+    rows_per_group rows of each of the five groups, the whole path."""
+    import oracle
+
+    oracle.build()
+    bs = workloads.exact_enum(seed=seed, rows_scale=rows_per_group / 24192,
+                              groups=tuple((rows_per_group, d) for _, d in workloads.ENUM_GROUPS))
+    Hs = [oracle.HostRows(b) for b in bs]
+    t0 = time.perf_counter()
+    for H in Hs:
+        oracle.dense_and_topk_gap(H)
+        oracle.swap_refine(H, E=N_KEYS, max_swaps=32)
+        oracle.best_subset(H)
+    dt = time.perf_counter() - t0
+    rows = sum(H.num_rows for H in Hs)
+    return dict(value=rows * SUBSETS_PER_ROW / dt, unit="subsets/s", cores=oracle.num_threads(), kind="oracle",
+                sample=f"first {rows_per_group} rows of each of the 5 groups ({rows} rows, "
+                       f"{rows * SUBSETS_PER_ROW:,} subsets), whole path (gap, swap, best subset), fp64",
+                seconds=dt)
+
+
+# ----------------------------------------------------------------- sections
+
+def section_long_rows(fw, device, K, W, flush, peaks):
+    b = workloads.long_rows(seed=0, backend="torch", device=device)
+    rows = fw.rows_from_batch(b, device)
+    del b.logits
+    step = lambda: fw.dense_and_topk_gap(rows, rows_k, kept_bits=True)  # noqa: E731
+    rows_k = torch.tensor([[2048, 4096, 8192]], dtype=torch.int32, device=device).repeat(rows.num_rows, 1)
+    total, times = time_steps(step, K, W, flush, lambda: None)
+    ms = total / K
+    nbytes = (rows.logits.numel() * 4 + rows.v.numel() * 2 + rows.num_rows * (128 * 4 * 4 + 3 * 4 * 4 + 3 * 4096 * 4))
+    ach = nbytes / (ms * 1e-3) / 1e9
+    return dict(workload="long_rows: 8 heads x 512 rows, n=32768, d=128, bf16 V, k in {2048,4096,8192}",
+                path="a1-a4 (fw_dense_and_topk_gap)", metric="rows/s", value=rows.num_rows / (ms * 1e-3),
+                ms_per_step=ms, roofline=dict(bound="hbm", achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s",
+                                              frac=ach / peaks["hbm_gbs"], traffic=None,
+                                              algorithmic_bytes=nbytes))
+
+
+def section_contour(fw, device, K, W, flush, peaks):
+    cb = workloads.contour_cache(seed=0, backend="torch", device=device)
+    Kc, Vc = cb.K.view(torch.int16), cb.V.view(torch.int16)
+    Ko = torch.empty(cb.total_budget, cb.d, dtype=torch.int16, device=device)
+    Vo = torch.empty_like(Ko)
+
+    def step():
+        a = fw.contour_alloc(cb.scores, floor=cb.floor, total_budget=cb.total_budget, uniform_s=cb.uniform_s)
+        fw.ragged_compact(Kc, Vc, a["offsets"], a["kept_pos"], cb.total_budget, out=(Ko, Vo))
+
+    total, times = time_steps(step, K, W, flush, lambda: None)
+    ms = total / K
+    nbytes = cb.cells * cb.T * 4 + 2 * 2 * cb.total_budget * cb.d * 2 + cb.total_budget * 4 + (cb.cells + 1) * 8
+    ach = nbytes / (ms * 1e-3) / 1e9
+    return dict(workload="contour_cache: 256 cells x 32768 tokens, d=128 bf16 K/V, budget 1/8, floor 32",
+                path="a7-a8 (fw_contour_alloc + fw_ragged_compact)", metric="kept KV rows/s",
+                value=cb.total_budget / (ms * 1e-3), ms_per_step=ms,
+                roofline=dict(bound="hbm", achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s",
+                              frac=ach / peaks["hbm_gbs"], traffic=None, algorithmic_bytes=nbytes))
+
+
+# --------------------------------------------------------------------- main
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-sections", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    K, W = args.steps, max(3, args.warmup)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist_mod
+
+        dist = dist_mod
+        dist.init_process_group("nccl" if args.impl == "ours" else "gloo")
+
+    if args.impl == "reference":
+        # the reference arm is the fp64 CPU oracle, on rank 0 only
+        if rank == 0:
+            steps = []
+            for _ in range(W):
+                cpu_baseline(seed=0, rows_per_group=8)
+            for _ in range(K):
+                steps.append(cpu_baseline(seed=0, rows_per_group=8))
+            v = statistics.median(s["value"] for s in steps)
+            sec = sum(s["seconds"] for s in steps) / K
+            line = dict(impl="reference", metric="subsets/s", value=v, unit="subsets/s", n_gpus=args.gpus,
+                        steps=K, warmup=W, ms_per_step=sec * 1e3, higher_is_better=True, scaling="weak",
+                        vs_baseline=None, dtype="f64", data="synthetic",
+                        config=dict(workload="exact_enum: 168,192 rows (5 groups, d=64/128), n=24, k=6",
+                                    sample="first 8 rows of each group per step"),
+                        cpu_baseline=dict(value=v, unit="subsets/s", cores=steps[0]["cores"], kind="oracle",
+                                          sample=steps[0]["sample"]),
+                        e2e=dict(value=v, unit="subsets/s", h2d_bytes_per_step=0, d2h_bytes_per_step=0))
+            print(json.dumps(line), flush=True)
+        if dist:
+            dist.destroy_process_group()
+        return
+
+    device = f"cuda:{local}"
+    torch.cuda.set_device(local)
+    from paper_2608_25230_gb300 import fw
+
+    peaks = read_peaks()
+    flush = L2Flush(device)
+    barrier = (lambda: dist.barrier()) if dist else (lambda: None)
+
+    wl = EnumWorkload(fw, seed=rank, device=device)
+    torch.cuda.synchronize()
+    l0 = fw.launch_count()
+    with ClockSampler(local) as clk:
+        total_ms, times = time_steps(lambda: wl.step(time_enum=True), K, W, flush, barrier)
+    launches = (fw.launch_count() - l0) // (K + W)
+    launches_timed = launches * K
+    enum_ev = wl.enum_times()[-5 * K:]
+    clocks = clk.summary()
+    ms = total_ms / K
+    if dist:
+        t = torch.tensor([ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = wl.subsets * world / (ms * 1e-3)
+
+    # roofline of the dominant kernel (the exact-search walk, fw_best_subset)
+    enum_ms = sum(t for t, _ in enum_ev) / K  # per step, all five groups
+    enum_launch_ms = sum(t for t, _ in enum_ev) / len(enum_ev)
+    sm_mhz = clocks.get("sm_mhz") or peaks["sm_max"]
+    alu_peak = 152 * 128 * sm_mhz * 1e6 / 1e9  # Gop/s, fp32 lanes x clock (issue-limited)
+    alu_ach = wl.subsets * ALU_OPS_PER_SUBSET / (enum_ms * 1e-3) / 1e9
+
+    # end to end through the public API with host buffers
+    e2e = EnumE2E(wl)
+    e2e_total, _ = time_steps(e2e.step, max(3, K // 2), W, flush, barrier)
+    e2e_ms = e2e_total / max(3, K // 2)
+    if dist:
+        t = torch.tensor([e2e_ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    sections = {}
+    if not args.no_sections and rank == 0:
+        sections["long_rows"] = section_long_rows(fw, device, 5, 3, flush, peaks)
+        sections["contour"] = section_contour(fw, device, 5, 3, flush, peaks)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu = cpu_baseline(seed=0)
+        cpu.pop("seconds", None)
+
+    line = dict(metric="subsets/s", value=value, unit="subsets/s", n_gpus=world, steps=K, warmup=W,
+                ms_per_step=ms, higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f32",
+                data="synthetic",
+                config=dict(workload="exact_enum: 168,192 rows in 5 groups (d=64,128,128,128,64), n=24, k=6, "
+                                     "134,596 subsets/row; step = gap + swap (E=all) + exact best subset",
+                            rows_per_gpu=wl.num_rows, subsets_per_step_per_gpu=wl.subsets,
+                            l2="inputs larger than L2 (1.6 GB) and a 256 MiB L2 flush between steps",
+                            parallelism=f"rows sharded, {world} independent replica(s)"),
+                roofline=dict(bound="alu", achieved=alu_ach, peak=alu_peak, unit="Gop/s", frac=alu_ach / alu_peak,
+                              traffic=None, kernel="k_enum (fw_best_subset)", launch_ms=enum_launch_ms,
+                              ops_per_subset=ALU_OPS_PER_SUBSET,
+                              peak_basis=f"152 SMs x 128 fp32 lanes x {sm_mhz:.0f} MHz (median SM clock under load)"),
+                e2e=dict(value=wl.subsets * world / (e2e_ms * 1e-3), unit="subsets/s",
+                         h2d_bytes_per_step=e2e.h2d, d2h_bytes_per_step=e2e.d2h),
+                gpu_launches=int(launches_timed), clocks=clocks, peaks_source=peaks["source"])
+    if cpu:
+        line["cpu_baseline"] = cpu
+    if sections:
+        line["sections"] = sections
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,193 @@
+/*
+ * fw.h -- C ABI of the forced-weight subset evaluation library (libfw.so).
+ *
+ * Implements, for batches of attention rows, the quantities of "Trust the
+ * Mass: Forced Weights in KV-Cache Eviction":
+ *   - Definition 2.1: an instance is a softmax row p over N keys with value
+ *     points v_j; the dense output mu = sum_j p_j v_j; a kept set A with kept
+ *     mass p(A), dropped mass 1 - p(A) and forced-weight output
+ *     m_A = sum_{j in A} (p_j / p(A)) v_j; the top-mass set A*_s.
+ *   - Sec. 2.1: the gap es(A) = ||mu - m_A||, its minimum ES(s) over |A| = s,
+ *     and the balancing selector (greedy one-for-one swaps from A*_s that most
+ *     decrease es, stopping when none does).
+ *   - Lemma 2.1: g_A = sum_{j in A} p_j (v_j - mu) and es(A) = ||g_A|| / p(A);
+ *     Phi = ||g_{A*_s}|| is the one-pass certificate.
+ *   - Definition 2.2: the candidate set (top-mass set plus the keys of largest
+ *     single-key error p_j ||v_j - mu||).
+ *   - Sec. 4: ContourKV (one score, one global threshold, a recency floor of
+ *     the last 32 positions per cell) and ragged per-head storage.
+ *
+ * Conventions for every entry point:
+ *   - All array arguments are DEVICE pointers unless stated otherwise; the
+ *     structs themselves (fw_rows, fw_gap_out, fw_swap_params) live in HOST
+ *     memory and are read during the call only.
+ *   - The caller owns every buffer, including the workspace; the library
+ *     never allocates or frees device memory.  Size workspaces with the
+ *     matching *_workspace() call; a workspace must be 256-byte aligned.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and the call returns without synchronising.  Outputs are valid
+ *     once the stream has reached that point.
+ *   - Arguments are validated on the host before any launch; on any error the
+ *     call returns a status other than FW_OK and enqueues nothing.
+ *   - Conditions only the device can see (non-finite logits) are reported per
+ *     row in `row_status`.  The library never traps, asserts or spins on the
+ *     device.
+ *   - Kept sets are stated by threshold: key j of a row is in the top-k set iff
+ *     key(l_j) > thr_key or (key(l_j) == thr_key and j <= thr_idx), where key()
+ *     maps a float to an unsigned integer of the same order after folding -0
+ *     onto +0 (equal logits: the lower index is kept first).
+ */
+#ifndef FW_H
+#define FW_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    FW_OK = 0,
+    FW_ERR_INVALID_ARG = 1,   /* a size, budget or pointer is out of range     */
+    FW_ERR_UNSUPPORTED = 2,   /* valid but not implemented (e.g. d not in 32k) */
+    FW_ERR_CUDA = 3,          /* a CUDA launch or query failed                */
+    FW_ERR_TIMEOUT = 4,       /* reserved: no entry point waits on the device */
+    FW_ERR_WORKSPACE = 5,     /* workspace missing, too small or misaligned   */
+    FW_ERR_NONFINITE = 6      /* per-row: a logit is NaN or infinite          */
+} fw_status;
+
+typedef enum { FW_F32 = 0, FW_BF16 = 1 } fw_dtype;
+
+/* A batch of attention rows (instances of Definition 2.1).
+ * Rows come in groups of `rows_per_group` consecutive rows that share one
+ * value block and one length: a KV head's query rows, a GQA group, or a single
+ * row (rows_per_group = 1).  Group g has n[g] keys (1 <= n[g] <= max_n); row
+ * r = g * rows_per_group + i has its n[g] fp32 logits at
+ * logits + logit_off[g] + i * n[g]; the group's values are the n[g] x d
+ * row-major block at v + v_off[g] (elements of type v_dtype).  The softmax of
+ * a row's logits is its mass vector p. */
+typedef struct {
+    int64_t num_groups;
+    int32_t rows_per_group;
+    int32_t d;              /* value width: a multiple of 32, at most 256     */
+    int32_t max_n;          /* host-side bound on every n[g]                   */
+    int32_t v_dtype;        /* fw_dtype                                        */
+    const float *logits;    /* device                                          */
+    const int64_t *logit_off; /* device [num_groups], element offsets          */
+    const int32_t *n;       /* device [num_groups]                             */
+    const void *v;          /* device                                          */
+    const int64_t *v_off;   /* device [num_groups], element offsets, multiples of 8 */
+} fw_rows;
+
+/* Outputs of fw_dense_and_topk_gap.  rows = num_groups * rows_per_group.
+ * Every pointer except gap and dropped may be NULL (not written). */
+typedef struct {
+    float *o;            /* [rows][d]      dense output mu                         */
+    float *o_kept;       /* [rows][nb][d]  forced-weight output m_A                */
+    float *gap;          /* [rows][nb]     es(A) = ||m_A - mu||                    */
+    float *dropped;      /* [rows][nb]     dropped mass, summed over keys not in A */
+    float *phi;          /* [rows][nb]     ||g_A|| = p(A) es(A)                    */
+    float *row_max;      /* [rows]         M = max_j l_j                           */
+    float *row_sum;      /* [rows]         Z = sum_j exp(l_j - M)                  */
+    uint32_t *thr_key;   /* [rows][nb]     order key of the k-th kept logit        */
+    int32_t *thr_idx;    /* [rows][nb]     largest kept index carrying thr_key     */
+    uint32_t *kept_bits; /* [rows][nb][kept_words] bit j%32 of word j/32 = (j in A) */
+    int32_t kept_words;  /* words per (row, budget); >= ceil(max_n/32) if kept_bits */
+    int32_t *row_status; /* [rows]         FW_OK or FW_ERR_NONFINITE               */
+} fw_gap_out;
+
+/* Dense output, top-k kept sets, forced-weight outputs, gaps and dropped mass
+ * (Definition 2.1, Sec. 2.1, Lemma 2.1) for every row and each of nb nested or
+ * independent budgets.
+ *   rows : host pointer to the batch description.
+ *   k    : device [rows][nb] int32 budgets, 1 <= k <= n of the row (checked on
+ *          the device: an out-of-range budget sets row_status to
+ *          FW_ERR_INVALID_ARG and leaves that row's outputs unspecified).
+ *   nb   : 1..4.
+ * The kept set of budget b is the k largest logits, equal logits kept in
+ * ascending index order.  The dropped mass is the sum of p_j over the keys
+ * not kept.  Non-finite logits set row_status[r] = FW_ERR_NONFINITE. */
+fw_status fw_dense_and_topk_gap(const fw_rows *rows, const int32_t *k, int32_t nb,
+                                const fw_gap_out *out, void *workspace, size_t workspace_bytes,
+                                void *stream);
+size_t fw_dense_and_topk_gap_workspace(const fw_rows *rows, int32_t nb);
+
+/* Parameters of the balancing selector. */
+typedef struct {
+    int32_t E;          /* extras: the E dropped keys of largest single-key error
+                           p_j ||v_j - mu|| (Definition 2.2) join the candidate
+                           set; 0 <= E.  E >= n - k puts every key in the pool. */
+    int32_t max_swaps;  /* cap on swaps per (row, budget), >= 1                 */
+} fw_swap_params;
+
+/* The balancing selector (Sec. 2.1) inside the candidate set (Definition 2.2).
+ * Starts from the top-k set described by `topk` (a fw_gap_out filled by
+ * fw_dense_and_topk_gap for the same rows, k and nb; its thr_key, thr_idx, o,
+ * row_max and row_sum must be non-NULL).  Each round scores every swap of one
+ * kept key for one pool key outside the set and takes the one with the
+ * smallest es (ties: smallest kept index, then smallest added index) if it is
+ * strictly below the current es; otherwise it stops.
+ * Outputs (device): n_swaps [rows][nb]; swap_out / swap_in
+ * [rows][nb][max_swaps] (removed / added key of each swap in the order taken;
+ * entries past n_swaps are -1); refined_gap [rows][nb]; topk_gap [rows][nb]
+ * (may be NULL); capped [rows][nb] = 1 if max_swaps stopped the search (may be
+ * NULL). */
+fw_status fw_swap_refine(const fw_rows *rows, const int32_t *k, int32_t nb, const fw_gap_out *topk,
+                         const fw_swap_params *prm, int32_t *n_swaps, int32_t *swap_out,
+                         int32_t *swap_in, float *refined_gap, float *topk_gap, int32_t *capped,
+                         void *workspace, size_t workspace_bytes, void *stream);
+size_t fw_swap_refine_workspace(const fw_rows *rows, int32_t nb, const fw_swap_params *prm);
+
+/* Exact ES(k) (Sec. 2.1) by exhaustive search over all C(n, k) subsets, for
+ * rows with n <= 32.  k: device [rows] int32, 1 <= k <= n.
+ * Outputs (device): best_rank [rows] colex rank sum_i C(c_i, i) of the
+ * minimising set c_1 < ... < c_k (0-based; exact ties -> smallest rank);
+ * best_gap [rows] = ES(k); best_idx [rows][k_max] ascending members (entries
+ * past k are -1); topk_gap [rows] = es of the top-k set (may be NULL);
+ * row_status [rows] (may be NULL).  k_max >= every k. */
+fw_status fw_best_subset(const fw_rows *rows, const int32_t *k, uint64_t *best_rank,
+                         float *best_gap, int32_t *best_idx, int32_t k_max, float *topk_gap,
+                         int32_t *row_status, void *workspace, size_t workspace_bytes,
+                         void *stream);
+size_t fw_best_subset_workspace(const fw_rows *rows);
+
+/* ContourKV allocation (Sec. 4).  scores: device [cells][T] fp32, finite and
+ * >= 0.  Every cell keeps its recency floor (the last min(floor, T) positions)
+ * plus the non-floor positions among the K = total_budget - cells*min(floor,T)
+ * best non-floor entries of the whole cache, ranked by (score desc, cell asc,
+ * position asc); *tau is the score of the K-th (+inf if K = 0).
+ * Outputs (device): counts [cells]; offsets [cells+1] exclusive prefix sum
+ * (offsets[cells] = total_budget); kept_pos [total_budget] positions of each
+ * cell in ascending order, cells in order; tau [1]; dropped_uniform [cells] and
+ * dropped_alloc [cells]: the mass of the cell's normalised scores outside the
+ * cell's own top-uniform_s set (ties -> lower position) and outside the
+ * allocated set (either may be NULL).
+ * Requires cells*min(floor,T) <= total_budget <= cells*T. */
+fw_status fw_contour_alloc(const float *scores, int32_t cells, int32_t T, int32_t floor,
+                           int64_t total_budget, int32_t uniform_s, int32_t *counts,
+                           int64_t *offsets, int32_t *kept_pos, float *tau,
+                           float *dropped_uniform, float *dropped_alloc, void *workspace,
+                           size_t workspace_bytes, void *stream);
+size_t fw_contour_alloc_workspace(int32_t cells, int32_t T);
+
+/* Ragged per-head storage (Sec. 4): copy the kept rows of K and V
+ * ([cells][T][row_bytes] each) into packed [offsets[cells]][row_bytes] outputs,
+ * cell by cell, positions in the order of kept_pos.  row_bytes must be a
+ * positive multiple of 16; K, V, K_out, V_out 16-byte aligned.  `total` is
+ * offsets[cells] as known to the host (the size of the packed outputs). */
+fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t T,
+                            int32_t row_bytes, const int64_t *offsets, const int32_t *kept_pos,
+                            int64_t total, void *K_out, void *V_out, void *stream);
+
+/* Human-readable name of a status. */
+const char *fw_status_string(fw_status s);
+
+/* Number of kernels this library has launched since it was loaded. */
+uint64_t fw_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FW_H */

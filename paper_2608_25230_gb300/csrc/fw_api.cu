@@ -1,0 +1,168 @@
+// fw_api.cu -- the C ABI: host-side validation, workspace carving, dispatch.
+#include <cstring>
+
+#include "fw_internal.h"
+
+namespace fw {
+std::atomic<uint64_t> g_launches{0};
+
+static bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+static fw_status check_rows(const fw_rows *r, RowsDev &R)
+{
+    if (!r) return FW_ERR_INVALID_ARG;
+    if (r->num_groups < 0 || r->rows_per_group < 1 || r->max_n < 1) return FW_ERR_INVALID_ARG;
+    if (r->d != 32 && r->d != 64 && r->d != 128 && r->d != 256) return FW_ERR_UNSUPPORTED;
+    if (r->v_dtype != FW_F32 && r->v_dtype != FW_BF16) return FW_ERR_INVALID_ARG;
+    if (r->num_groups > 0 && (!r->logits || !r->logit_off || !r->n || !r->v || !r->v_off))
+        return FW_ERR_INVALID_ARG;
+    R.num_groups = r->num_groups;
+    R.R = r->rows_per_group;
+    R.rows = r->num_groups * (int64_t)r->rows_per_group;
+    R.d = r->d;
+    R.max_n = r->max_n;
+    R.v_dtype = r->v_dtype;
+    R.logits = r->logits;
+    R.logit_off = r->logit_off;
+    R.n = r->n;
+    R.v = r->v;
+    R.v_off = r->v_off;
+    return FW_OK;
+}
+
+}  // namespace fw
+
+using namespace fw;
+
+extern "C" {
+
+const char *fw_status_string(fw_status s)
+{
+    switch (s) {
+    case FW_OK: return "ok";
+    case FW_ERR_INVALID_ARG: return "invalid argument";
+    case FW_ERR_UNSUPPORTED: return "unsupported configuration";
+    case FW_ERR_CUDA: return "CUDA error";
+    case FW_ERR_TIMEOUT: return "timeout";
+    case FW_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case FW_ERR_NONFINITE: return "non-finite logit";
+    default: return "unknown status";
+    }
+}
+
+uint64_t fw_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+size_t fw_dense_and_topk_gap_workspace(const fw_rows *rows, int32_t nb)
+{
+    RowsDev R;
+    if (check_rows(rows, R) != FW_OK || nb < 1 || nb > 4) return 0;
+    if (R.max_n <= 32) return 0;
+    return long_gap_workspace(R, nb);
+}
+
+fw_status fw_dense_and_topk_gap(const fw_rows *rows, const int32_t *k, int32_t nb, const fw_gap_out *out,
+                                void *workspace, size_t workspace_bytes, void *stream)
+{
+    RowsDev R;
+    fw_status st = check_rows(rows, R);
+    if (st != FW_OK) return st;
+    if (nb < 1 || nb > 4 || !k || !out || !out->gap || !out->dropped) return FW_ERR_INVALID_ARG;
+    if (out->kept_bits && out->kept_words < (R.max_n + 31) / 32) return FW_ERR_INVALID_ARG;
+    if (R.rows == 0) return FW_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (R.max_n <= 32) return small_gap(R, k, nb, *out, s);
+    if (workspace_bytes < long_gap_workspace(R, nb) || !workspace || !aligned(workspace, 256))
+        return FW_ERR_WORKSPACE;
+    return long_gap(R, k, nb, *out, workspace, workspace_bytes, s);
+}
+
+size_t fw_swap_refine_workspace(const fw_rows *rows, int32_t nb, const fw_swap_params *prm)
+{
+    RowsDev R;
+    if (check_rows(rows, R) != FW_OK || nb < 1 || nb > 4 || !prm) return 0;
+    if (R.max_n <= 32) return 0;
+    return long_swap_workspace(R, nb, prm->E, prm->max_swaps);
+}
+
+fw_status fw_swap_refine(const fw_rows *rows, const int32_t *k, int32_t nb, const fw_gap_out *topk,
+                         const fw_swap_params *prm, int32_t *n_swaps, int32_t *swap_out, int32_t *swap_in,
+                         float *refined_gap, float *topk_gap, int32_t *capped, void *workspace,
+                         size_t workspace_bytes, void *stream)
+{
+    RowsDev R;
+    fw_status st = check_rows(rows, R);
+    if (st != FW_OK) return st;
+    if (nb < 1 || nb > 4 || !k || !topk || !prm || !n_swaps || !swap_out || !swap_in || !refined_gap)
+        return FW_ERR_INVALID_ARG;
+    if (!topk->thr_key || !topk->thr_idx || !topk->o || !topk->row_max || !topk->row_sum)
+        return FW_ERR_INVALID_ARG;
+    if (prm->E < 0 || prm->max_swaps < 1) return FW_ERR_INVALID_ARG;
+    if (R.rows == 0) return FW_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (R.max_n <= 32)
+        return small_swap(R, k, nb, *topk, prm->E, prm->max_swaps, n_swaps, swap_out, swap_in,
+                          refined_gap, topk_gap, capped, s);
+    if (workspace_bytes < long_swap_workspace(R, nb, prm->E, prm->max_swaps) || !workspace ||
+        !aligned(workspace, 256))
+        return FW_ERR_WORKSPACE;
+    return long_swap(R, k, nb, *topk, prm->E, prm->max_swaps, n_swaps, swap_out, swap_in, refined_gap,
+                     topk_gap, capped, workspace, workspace_bytes, s);
+}
+
+size_t fw_best_subset_workspace(const fw_rows *rows)
+{
+    RowsDev R;
+    if (check_rows(rows, R) != FW_OK) return 0;
+    return enum_workspace(R);
+}
+
+fw_status fw_best_subset(const fw_rows *rows, const int32_t *k, uint64_t *best_rank, float *best_gap,
+                         int32_t *best_idx, int32_t k_max, float *topk_gap, int32_t *row_status,
+                         void *workspace, size_t workspace_bytes, void *stream)
+{
+    RowsDev R;
+    fw_status st = check_rows(rows, R);
+    if (st != FW_OK) return st;
+    if (R.max_n > 32) return FW_ERR_UNSUPPORTED;
+    if (!k || !best_rank || !best_gap || !best_idx || k_max < 1 || k_max > 32) return FW_ERR_INVALID_ARG;
+    if (R.rows == 0) return FW_OK;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < enum_workspace(R)) return FW_ERR_WORKSPACE;
+    return best_subset(R, k, best_rank, best_gap, best_idx, k_max, topk_gap, row_status, workspace,
+                       workspace_bytes, (cudaStream_t)stream);
+}
+
+size_t fw_contour_alloc_workspace(int32_t cells, int32_t T)
+{
+    if (cells < 1 || T < 1) return 0;
+    return contour_workspace(cells, T);
+}
+
+fw_status fw_contour_alloc(const float *scores, int32_t cells, int32_t T, int32_t floor_, int64_t total_budget,
+                           int32_t uniform_s, int32_t *counts, int64_t *offsets, int32_t *kept_pos, float *tau,
+                           float *dropped_uniform, float *dropped_alloc, void *workspace, size_t workspace_bytes,
+                           void *stream)
+{
+    if (!scores || cells < 1 || T < 1 || floor_ < 0 || uniform_s < 0) return FW_ERR_INVALID_ARG;
+    const int F = floor_ < T ? floor_ : T;
+    if (total_budget < (int64_t)cells * F || total_budget > (int64_t)cells * T) return FW_ERR_INVALID_ARG;
+    if (!counts || !offsets || !kept_pos || !tau) return FW_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < contour_workspace(cells, T))
+        return FW_ERR_WORKSPACE;
+    return contour_alloc(scores, cells, T, floor_, total_budget, uniform_s, counts, offsets, kept_pos, tau,
+                         dropped_uniform, dropped_alloc, workspace, workspace_bytes, (cudaStream_t)stream);
+}
+
+fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t T, int32_t row_bytes,
+                            const int64_t *offsets, const int32_t *kept_pos, int64_t total, void *K_out,
+                            void *V_out, void *stream)
+{
+    if (!K || !V || !offsets || !kept_pos || cells < 1 || T < 1 || total < 0) return FW_ERR_INVALID_ARG;
+    if (row_bytes <= 0 || row_bytes % 16 != 0) return FW_ERR_INVALID_ARG;
+    if (total > 0 && (!K_out || !V_out)) return FW_ERR_INVALID_ARG;
+    if (!aligned(K, 16) || !aligned(V, 16) || (total > 0 && (!aligned(K_out, 16) || !aligned(V_out, 16))))
+        return FW_ERR_INVALID_ARG;
+    return ragged_compact(K, V, cells, T, row_bytes, offsets, kept_pos, total, K_out, V_out,
+                          (cudaStream_t)stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,199 @@
+// fw_common.cuh -- device helpers shared by the library's kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <atomic>
+#include <cmath>
+
+#include "fw.h"
+
+#define FW_FULL 0xffffffffu
+
+namespace fw {
+
+// ------------------------------------------------------------ launch accounting
+extern std::atomic<uint64_t> g_launches;
+
+// Launch a kernel, count it, and turn a launch error into FW_ERR_CUDA.
+#define FW_LAUNCH(kernel, grid, block, smem, stream, ...)                                      \
+    do {                                                                                       \
+        kernel<<<(grid), (block), (smem), (cudaStream_t)(stream)>>>(__VA_ARGS__);              \
+        ::fw::g_launches.fetch_add(1, std::memory_order_relaxed);                              \
+        cudaError_t _e = cudaGetLastError();                                                   \
+        if (_e != cudaSuccess) return FW_ERR_CUDA;                                             \
+    } while (0)
+
+#define FW_CUDA_CHECK(expr)                                                                    \
+    do {                                                                                       \
+        if ((expr) != cudaSuccess) return FW_ERR_CUDA;                                         \
+    } while (0)
+
+// ------------------------------------------------------------------- order keys
+// Unsigned key with the order of the float, after folding -0 onto +0, so that
+// equal logits tie (and are then ordered by index).
+__device__ __forceinline__ uint32_t order_key(float x)
+{
+    uint32_t u = __float_as_uint(x == 0.0f ? 0.0f : x);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(((uint32_t)b) << 16); }
+
+template <typename VT> __device__ __forceinline__ float load_v(const VT *p, int64_t i);
+template <> __device__ __forceinline__ float load_v<float>(const float *p, int64_t i) { return __ldg(p + i); }
+template <> __device__ __forceinline__ float load_v<uint16_t>(const uint16_t *p, int64_t i)
+{
+    return bf16_to_f32(__ldg(p + i));
+}
+
+// --------------------------------------------------------- double-float (df)
+// A value hi + lo held in two floats (|lo| <= ulp(hi)/2), about 44 bits of
+// precision on the fp32 pipe.  Built from the classical error-free transforms:
+// Knuth's TwoSum, the Dekker/Fast2Sum renormalisation, and the FMA-based exact
+// product a*b = p + fma(a, b, -p).  GB300 runs fp64 at a small fraction of its
+// fp32 rate, so vector sums that need more than fp32 use this instead.
+struct df {
+    float hi, lo;
+};
+
+__device__ __forceinline__ df df_two_sum(float a, float b)
+{
+    float s = a + b;
+    float bb = s - a;
+    float e = (a - (s - bb)) + (b - bb);
+    return {s, e};
+}
+__device__ __forceinline__ df df_fast_two_sum(float a, float b)
+{
+    float s = a + b;
+    float e = b - (s - a);
+    return {s, e};
+}
+__device__ __forceinline__ df df_add(df x, df y)
+{
+    df s = df_two_sum(x.hi, y.hi);
+    df t = df_two_sum(x.lo, y.lo);
+    float e = s.lo + t.hi;
+    s = df_fast_two_sum(s.hi, e);
+    e = t.lo + s.lo;
+    return df_fast_two_sum(s.hi, e);
+}
+__device__ __forceinline__ df df_neg(df x) { return {-x.hi, -x.lo}; }
+__device__ __forceinline__ df df_sub(df x, df y) { return df_add(x, df_neg(y)); }
+__device__ __forceinline__ df df_mul(df x, df y)
+{
+    float p = x.hi * y.hi;
+    float e = fmaf(x.hi, y.hi, -p);
+    e = fmaf(x.hi, y.lo, e);
+    e = fmaf(x.lo, y.hi, e);
+    return df_fast_two_sum(p, e);
+}
+__device__ __forceinline__ df df_mul_f(df x, float y)
+{
+    float p = x.hi * y;
+    float e = fmaf(x.hi, y, -p);
+    e = fmaf(x.lo, y, e);
+    return df_fast_two_sum(p, e);
+}
+// f - x for a float f and df x
+__device__ __forceinline__ df df_rsub_f(float f, df x)
+{
+    df s = df_two_sum(f, -x.hi);
+    float e = s.lo - x.lo;
+    return df_fast_two_sum(s.hi, e);
+}
+__device__ __forceinline__ df df_from_double(double x)
+{
+    float hi = (float)x;
+    float lo = (float)(x - (double)hi);
+    return {hi, lo};
+}
+__device__ __forceinline__ double df_to_double(df x) { return (double)x.hi + (double)x.lo; }
+__device__ __forceinline__ df df_zero() { return {0.0f, 0.0f}; }
+
+// ----------------------------------------------------------- warp reductions
+__device__ __forceinline__ float warp_max(float v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(FW_FULL, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_min(float v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(FW_FULL, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_sum(float v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FW_FULL, v, o);
+    return v;
+}
+__device__ __forceinline__ double warp_sum_d(double v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FW_FULL, v, o);
+    return v;
+}
+__device__ __forceinline__ df warp_sum_df(df v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        df w = {__shfl_xor_sync(FW_FULL, v.hi, o), __shfl_xor_sync(FW_FULL, v.lo, o)};
+        v = df_add(v, w);
+    }
+    return v;
+}
+__device__ __forceinline__ df shfl_df(df v, int src)
+{
+    return {__shfl_sync(FW_FULL, v.hi, src), __shfl_sync(FW_FULL, v.lo, src)};
+}
+
+// colex rank of the set bits of a 32-bit mask: sum_i C(c_i, i), i = 1.. in ascending order
+__device__ __forceinline__ uint64_t binom64(int a, int b)
+{
+    if (b < 0 || b > a) return 0;
+    uint64_t r = 1;
+    for (int t = 1; t <= b; ++t) r = r * (uint64_t)(a - b + t) / (uint64_t)t;
+    return r;
+}
+__device__ __forceinline__ uint64_t colex_rank_mask(uint32_t m)
+{
+    uint64_t r = 0;
+    int i = 1;
+    while (m) {
+        int c = __ffs(m) - 1;
+        r += binom64(c, i);
+        ++i;
+        m &= m - 1;
+    }
+    return r;
+}
+
+// Dispatch on the value width d (multiples of 32 supported: 32, 64, 128, 256)
+// and the value dtype; binds DPL (dims per lane) and VT (element type).
+#define FW_DISPATCH(d, vdt, ...)                                                              \
+    do {                                                                                       \
+        if ((vdt) == FW_F32) {                                                                 \
+            using VT = float;                                                                  \
+            FW_DISPATCH_D(d, __VA_ARGS__);                                                            \
+        } else if ((vdt) == FW_BF16) {                                                         \
+            using VT = uint16_t;                                                               \
+            FW_DISPATCH_D(d, __VA_ARGS__);                                                            \
+        } else {                                                                               \
+            return FW_ERR_INVALID_ARG;                                                         \
+        }                                                                                      \
+    } while (0)
+#define FW_DISPATCH_D(d, ...)                                                                 \
+    switch (d) {                                                                               \
+    case 32: { constexpr int DPL = 1; __VA_ARGS__; } break;                                           \
+    case 64: { constexpr int DPL = 2; __VA_ARGS__; } break;                                           \
+    case 128: { constexpr int DPL = 4; __VA_ARGS__; } break;                                          \
+    case 256: { constexpr int DPL = 8; __VA_ARGS__; } break;                                          \
+    default: return FW_ERR_UNSUPPORTED;                                                        \
+    }
+
+}  // namespace fw

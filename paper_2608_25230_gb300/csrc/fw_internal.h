@@ -1,0 +1,57 @@
+// fw_internal.h -- launcher interfaces between the C ABI (fw_api.cu) and the
+// kernel translation units.
+#pragma once
+
+#include "fw_common.cuh"
+
+namespace fw {
+
+// Device-side copy of fw_rows plus the derived row count.
+struct RowsDev {
+    int64_t num_groups;
+    int64_t rows;
+    int32_t R;      // rows per group
+    int32_t d;
+    int32_t max_n;
+    int32_t v_dtype;
+    const float *logits;
+    const int64_t *logit_off;
+    const int32_t *n;
+    const void *v;
+    const int64_t *v_off;
+};
+
+// Rows with n <= 32 ("small rows": exact-enumeration workloads).
+fw_status small_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out,
+                    cudaStream_t s);
+fw_status small_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &topk,
+                     int E, int max_swaps, int32_t *n_swaps, int32_t *swap_out, int32_t *swap_in,
+                     float *refined_gap, float *topk_gap, int32_t *capped, cudaStream_t s);
+size_t enum_workspace(const RowsDev &R);
+fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, float *best_gap,
+                      int32_t *best_idx, int k_max, float *topk_gap, int32_t *row_status,
+                      void *ws, size_t ws_bytes, cudaStream_t s);
+
+// Long rows (any n): row statistics + radix top-k, then the P.V products.
+size_t long_gap_workspace(const RowsDev &R, int nb);
+fw_status long_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, void *ws,
+                   size_t ws_bytes, cudaStream_t s);
+size_t long_swap_workspace(const RowsDev &R, int nb, int E, int max_swaps);
+fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &topk, int E,
+                    int max_swaps, int32_t *n_swaps, int32_t *swap_out, int32_t *swap_in,
+                    float *refined_gap, float *topk_gap, int32_t *capped, void *ws,
+                    size_t ws_bytes, cudaStream_t s);
+
+// ContourKV allocation and ragged compaction.
+size_t contour_workspace(int cells, int T);
+fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64_t total_budget,
+                        int uniform_s, int32_t *counts, int64_t *offsets, int32_t *kept_pos,
+                        float *tau, float *dropped_uniform, float *dropped_alloc, void *ws,
+                        size_t ws_bytes, cudaStream_t s);
+fw_status ragged_compact(const void *K, const void *V, int cells, int T, int row_bytes,
+                         const int64_t *offsets, const int32_t *kept_pos, int64_t total,
+                         void *K_out, void *V_out, cudaStream_t s);
+
+inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+}  // namespace fw
