@@ -180,6 +180,34 @@ fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t
                             int32_t row_bytes, const int64_t *offsets, const int32_t *kept_pos,
                             int64_t total, void *K_out, void *V_out, void *stream);
 
+/* Largest cells accepted by fw_contour_alloc_noalloc. */
+#define FW_CONTOUR_NOALLOC_MAX_CELLS 4096
+
+/* fw_contour_alloc for callers that cannot allocate device memory.
+ * The paper has no counterpart: this is a deployment convenience.  Some
+ * callers may not call cudaMalloc at all -- a plugin living inside another
+ * framework's device-memory pool, or a latency-critical path where a
+ * cudaMalloc would synchronise the device -- and cannot provide the
+ * workspace fw_contour_alloc asks for.  This variant takes the same
+ * arguments minus the workspace and uses a scratch area compiled into the
+ * library instead (about 50 KB, held by every GPU that loads the library
+ * until the process exits).
+ *   - cells must be <= FW_CONTOUR_NOALLOC_MAX_CELLS, otherwise the call
+ *     returns FW_ERR_WORKSPACE and launches nothing; the other argument
+ *     rules and all outputs are exactly those of fw_contour_alloc.
+ *   - It never allocates or frees device memory.
+ *   - The first call on each device looks up the scratch area's device
+ *     address (with that device current); make that first call before any
+ *     stream capture on the device.
+ *   - All calls share the one scratch area and every call re-initialises
+ *     what it reads, so consecutive calls are independent; calls that
+ *     overlap on the GPU (concurrent streams, several host threads) race on
+ *     the scratch and must be serialised by the caller. */
+fw_status fw_contour_alloc_noalloc(const float *scores, int32_t cells, int32_t T, int32_t floor,
+                                   int64_t total_budget, int32_t uniform_s, int32_t *counts,
+                                   int64_t *offsets, int32_t *kept_pos, float *tau,
+                                   float *dropped_uniform, float *dropped_alloc, void *stream);
+
 /* Human-readable name of a status. */
 const char *fw_status_string(fw_status s);
 

@@ -12,6 +12,7 @@
 // prefix sum into ragged offsets, and per-cell ordered compaction of the kept
 // positions.  The compaction copy moves 16-byte vectors, a row per 16 lanes.
 #include <algorithm>
+#include <mutex>
 
 #include "fw_internal.h"
 
@@ -447,3 +448,50 @@ fw_status ragged_compact(const void *K, const void *V, int cells, int T, int row
 }
 
 }  // namespace fw
+
+// ------------------------------------------------------------------------
+// Allocation-free variant: the scratch lives in a fixed device array.
+namespace fw {
+namespace {
+
+constexpr size_t kNoallocBytes = 256 * 4 + 256 + 3 * (size_t)FW_CONTOUR_NOALLOC_MAX_CELLS * 4;  // >= contour_workspace
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocBytes + 3 * 256];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array for the current device (looked up once per device).
+fw_status noalloc_scratch(void **ptr)
+{
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FW_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return FW_ERR_CUDA;
+        g_noalloc_ptr[dev] = p;
+    }
+    *ptr = g_noalloc_ptr[dev];
+    return FW_OK;
+}
+
+}  // namespace
+}  // namespace fw
+
+extern "C" fw_status fw_contour_alloc_noalloc(const float *scores, int32_t cells, int32_t T, int32_t floor_,
+                                              int64_t total_budget, int32_t uniform_s, int32_t *counts,
+                                              int64_t *offsets, int32_t *kept_pos, float *tau,
+                                              float *dropped_uniform, float *dropped_alloc, void *stream)
+{
+    if (cells > FW_CONTOUR_NOALLOC_MAX_CELLS) return FW_ERR_WORKSPACE;
+    if (cells >= 1 && T >= 1 && fw::contour_workspace(cells, T) > sizeof(fw::g_noalloc_scratch))
+        return FW_ERR_WORKSPACE;
+    void *ws = nullptr;
+    if (cells >= 1 && T >= 1) {
+        const fw_status st = fw::noalloc_scratch(&ws);
+        if (st != FW_OK) return st;
+    }
+    return fw_contour_alloc(scores, cells, T, floor_, total_budget, uniform_s, counts, offsets, kept_pos, tau,
+                            dropped_uniform, dropped_alloc, ws, sizeof(fw::g_noalloc_scratch), stream);
+}
