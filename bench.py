@@ -214,7 +214,7 @@ def cpu_baseline(seed, rows_per_group=40):
     import oracle
 
     oracle.build()
-    bs = workloads.exact_enum(seed=seed, rows_scale=rows_per_group / 24192,
+    bs = workloads.exact_enum(seed=seed, rows_scale=1.0,
                               groups=tuple((rows_per_group, d) for _, d in workloads.ENUM_GROUPS))
     Hs = [oracle.HostRows(b) for b in bs]
     t0 = time.perf_counter()

@@ -33,8 +33,9 @@
 namespace fw {
 namespace {
 
-constexpr int EM = 10;    // inner key set size
+constexpr int EM = 12;    // inner key set size
 constexpr int ECAP = 32;  // candidate masks per row
+constexpr int FBS = 16;   // chunks (blocks) per row on the exhaustive path
 constexpr int MAXD = 24;  // depth bound of the phase-2 walk
 constexpr int PERM = 48;  // local index space per row: NS <= EM + 32
 
@@ -54,30 +55,44 @@ struct EnumArgs {
     int32_t *cand_count;  // [rows]
     int32_t *fb_list;     // [rows]
     int32_t *fb_count;    // [1]
+    double *fb_e;         // [rows][FBS] best es^2 of each chunk of an exhaustive row
+    unsigned long long *fb_r;  // [rows][FBS] its colex rank
     int stride;           // floats per row slot (odd)
 };
 
-// Per-row slot (floats), local key order [L (EM, padded) | A0 (k) | H' (nHp)], NS = EM + k + nHp:
-//   GP : upper triangle of G'_xy = u_x.u_y - t p_x p_y over the NS local keys
-//   AA : a_x [NS];  LL : l_x [NS] (difference-form linear term, sign included)
-__host__ __device__ constexpr int slot_floats(int NS) { return NS * (NS + 1) / 2 + 2 * NS; }
+// Per-row slot (floats).  Local key order: L (EM inner keys, padded), A0 (k),
+// H' (nHp outer added keys).  Entries "folded" have the error-bound term
+// kappa a_x a_y subtracted; G' = u.u - t p p^T; l = difference-form linear term.
+//   [0, EM)        Gd  : folded direct-form diagonal of L (+inf on padding)
+//   [EM, 2EM)      lS  : extra difference-form diagonal of L (l_j - 4 kappa g0n a_j)
+//   [2EM, 3EM)     aL  : a_j of L
+//   [3EM, 3EM+EM^2) G2 : 2 x folded off-diagonal of L x L (square, zero diagonal)
+//   A0 rows (k x RA, RA = EM + k + nHp + 2): raw G'(x, L) | G'(x, A0) | G'(x, H') | a_x | l_x
+//   H' rows (nHp x RH, RH = EM + nHp + 2): folded G'(y, L) | HH (2 x folded off-diagonal,
+//                                          folded diagonal) | l_y - 4 kappa g0n a_y | a_y
+constexpr int OFF_A = 3 * EM + EM * EM;
+__host__ __device__ constexpr int slot_floats(int k, int nHp)
+{
+    return OFF_A + k * (EM + k + nHp + 2) + nHp * (EM + nHp + 2);
+}
 
 struct Walk {
     const float *slot;
     const uint8_t *perm;  // local index -> original key
-    int k, nL, nHp, NS;
+    int k, nL, nHp;
+    int half;             // which of the row's two lanes: takes every other R of each size class
+    uint32_t sync_mask;   // lanes that walk rows of identical (n, k); 0 when they differ
     float kappa, g0n;
     uint32_t *cand;
     int32_t *ccount;
 };
 
-__device__ __forceinline__ float GPx(const Walk &W, int x, int y) { return W.slot[tri_s(x, y, W.NS)]; }
-__device__ __forceinline__ float AAx(const Walk &W, int x) { return W.slot[W.NS * (W.NS + 1) / 2 + x]; }
-__device__ __forceinline__ float LLx(const Walk &W, int x) { return W.slot[W.NS * (W.NS + 1) / 2 + W.NS + x]; }
-
 // ---- slow path: list every inner set C (size c) of a node whose folded value is <= 0
-__device__ __noinline__ void collect(const Walk W, uint32_t amask_outer, const float *w, float q, int c)
+__device__ __noinline__ void collect(const Walk W, uint32_t keep0, uint32_t hmask, const float *w, float q, int c)
 {
+    const float *G2 = W.slot + 3 * EM;
+    uint32_t amask = keep0;
+    for (uint32_t m = hmask; m; m &= m - 1) amask |= 1u << W.perm[EM + W.k + __ffs(m) - 1];
     uint32_t cm = c == 0 ? 0u : (1u << c) - 1u;
     const uint32_t lim = 1u << W.nL;
     for (;;) {
@@ -85,22 +100,18 @@ __device__ __noinline__ void collect(const Walk W, uint32_t amask_outer, const f
         for (uint32_t a = cm; a; a &= a - 1) {
             const int j = __ffs(a) - 1;
             v += w[j];
-            for (uint32_t b2 = a & (a - 1); b2; b2 &= b2 - 1) {
-                const int j2 = __ffs(b2) - 1;
-                v += 2.f * (GPx(W, j, j2) - W.kappa * AAx(W, j) * AAx(W, j2));
-            }
+            for (uint32_t b2 = a & (a - 1); b2; b2 &= b2 - 1) v += G2[j * EM + __ffs(b2) - 1];
         }
         if (v <= 0.f) {
-            uint32_t m = amask_outer;
+            uint32_t m = amask;
             for (uint32_t a = cm; a; a &= a - 1) m |= 1u << W.perm[__ffs(a) - 1];
-            const int s = *W.ccount;
-            if (s < ECAP) W.cand[s] = m;
-            *W.ccount = s + 1;
+            const int sl = atomicAdd(W.ccount, 1);
+            if (sl < ECAP) W.cand[sl] = m;
         }
         if (c == 0) break;
         const uint32_t lo = cm & (0u - cm);  // next subset of the same size (Gosper's rule)
-        const uint32_t r = cm + lo;
-        cm = (((r ^ cm) >> 2) / lo) | r;
+        const uint32_t rr = cm + lo;
+        cm = (((rr ^ cm) >> 2) / lo) | rr;
         if (cm >= lim) break;
     }
 }
@@ -150,28 +161,10 @@ __device__ __forceinline__ float inner_dispatch(int c, const float (&w)[EM], flo
     case 8: return inner<8>(w, q, G2);
     case 9: return inner<9>(w, q, G2);
     case 10: return inner<10>(w, q, G2);
+    case 11: return inner<11>(w, q, G2);
+    case 12: return inner<12>(w, q, G2);
     default: return INFINITY;
     }
-}
-
-// Push key e of H' onto the phase-2 path: update h, q, the added-key mask.
-__device__ __forceinline__ void push_added(const Walk &W, int e, int depth, bool sform, const float (&aL)[EM],
-                                           float (&h)[EM], float &q, const float *base, const int *path,
-                                           uint32_t &imask)
-{
-    const int ly = EM + W.k + e;
-    const float ay = AAx(W, ly), kay = W.kappa * ay;
-#pragma unroll
-    for (int j = 0; j < EM; ++j)
-        if (j < W.nL) h[j] += GPx(W, ly, j) - kay * aL[j];
-    float dq = GPx(W, ly, ly) - kay * ay + 2.f * base[e];
-    if (sform) dq += LLx(W, ly) - 4.f * kay * W.g0n;
-    for (int t = 0; t < depth; ++t) {
-        const int lz = EM + W.k + path[t];
-        dq += 2.f * (GPx(W, ly, lz) - kay * AAx(W, lz));
-    }
-    q += dq;
-    imask |= 1u << W.perm[ly];
 }
 
 // The whole walk of one row (one lane).  Compiled once; every kernel
@@ -180,80 +173,96 @@ __device__ __noinline__ void walk_row(const Walk W)
 {
     const float kap = W.kappa, g0n = W.g0n;
     const int k = W.k, nL = W.nL, nHp = W.nHp;
-    const int A0b = EM, Hb = EM + k;  // local index bases
-    float aL[EM], Gd[EM], lS[EM], G2[EM][EM];
+    const int RA = EM + k + nHp + 2, RH = EM + nHp + 2;
+    const float *SA = W.slot + OFF_A;
+    const float *SH = SA + k * RA;
+    float Gd[EM], lS[EM], aL[EM], G2[EM][EM];
 #pragma unroll
     for (int x = 0; x < EM; ++x) {
-        const bool real = x < nL;
-        aL[x] = real ? AAx(W, x) : 0.f;
-        Gd[x] = real ? GPx(W, x, x) - kap * aL[x] * aL[x] : INFINITY;
-        lS[x] = real ? LLx(W, x) - 4.f * kap * g0n * aL[x] : 0.f;
+        Gd[x] = W.slot[x];
+        lS[x] = W.slot[EM + x];
+        aL[x] = W.slot[2 * EM + x];
 #pragma unroll
-        for (int y = x + 1; y < EM; ++y)
-            G2[x][y] = (real && y < nL) ? 2.f * (GPx(W, x, y) - kap * aL[x] * AAx(W, y)) : 0.f;
+        for (int y = x + 1; y < EM; ++y) G2[x][y] = W.slot[3 * EM + x * EM + y];
     }
-    float base[MAXD];  // per H' key: sum over the phase-1 outer keys of E(x, y)
+    float base[MAXD];  // per H' key: sum over the phase-1 outer keys of the folded E(x, y)
     float hst[MAXD][EM];
     float qst[MAXD];
     int path[MAXD];
     const uint32_t nR = 1u << k;
-    for (uint32_t R = 0; R < nR; ++R) {
-        const int r = __popc(R);
-        if (r > nL + nHp) continue;  // cannot add back r keys
+    // Removal sets R of A0 by size class; the row's two lanes take alternate
+    // members of the same class at the same time, so they run the same code.
+    for (int r = 0; r <= k; ++r) {
+        if (r > nL + nHp) break;  // cannot add back r keys
+        uint32_t R = r == 0 ? 0u : (1u << r) - 1u;
+        bool valid = true;
+        auto next_same_size = [&](uint32_t x) -> uint32_t {  // Gosper's rule
+            if (x == 0u) return nR;
+            const uint32_t lo = x & (0u - x);
+            const uint32_t ri = x + lo;
+            return (((ri ^ x) >> 2) / lo) | ri;
+        };
+        if (W.half) {
+            R = next_same_size(R);
+            valid = R < nR;
+        }
+        while (valid) {
         // choose the form with the smaller error bound
         float sR = 0.f, sK = 0.f;
         for (int x = 0; x < k; ++x) {
-            const float ax = AAx(W, A0b + x);
+            const float ax = SA[x * RA + RA - 2];
             if ((R >> x) & 1u) sR += ax;
             else sK += ax;
         }
         const bool sform = sR * (4.f * g0n + sR) <= sK * sK;
         const uint32_t O = sform ? R : (~R & (nR - 1u));  // outer keys of A0 in this form
         const float sgn = sform ? -1.f : 1.f;            // their sign
-        // phase 1: h (inner keys), q, base (H' keys) from scratch
+        // phase 1: h (inner keys), q, base (H' keys) from scratch, fixed trip counts
         float h[EM];
 #pragma unroll
         for (int j = 0; j < EM; ++j) h[j] = 0.f;
         float q = 0.f;
         for (int y = 0; y < nHp; ++y) base[y] = 0.f;
-        for (uint32_t m = O; m; m &= m - 1) {
-            const int x = __ffs(m) - 1, lx = A0b + x;
-            const float ax = AAx(W, lx);
-            const float kax = kap * ax;
+        for (int x = 0; x < k; ++x) {
+            const float on = ((O >> x) & 1u) ? 1.f : 0.f;
+            const float *row = SA + x * RA;
+            const float ax = row[RA - 2], kax = kap * ax;
+            const float so = sgn * on, ko = kax * on;
 #pragma unroll
-            for (int j = 0; j < EM; ++j)
-                if (j < nL) h[j] += sgn * GPx(W, lx, j) - kax * aL[j];
-            float dq = GPx(W, lx, lx) - kax * ax;
-            if (sform) dq += LLx(W, lx) - 4.f * kax * g0n;
-            for (uint32_t m2 = O & ((1u << x) - 1u); m2; m2 &= m2 - 1) {
-                const int ly = A0b + __ffs(m2) - 1;
-                dq += 2.f * (GPx(W, lx, ly) - kax * AAx(W, ly));  // sign^2 = +1
+            for (int j = 0; j < EM; ++j) h[j] += fmaf(so, row[j], -ko * aL[j]);
+            float dq = row[EM + x] - kax * ax;
+            if (sform) dq += row[RA - 1] - 4.f * kax * g0n;
+            for (int x2 = 0; x2 < x; ++x2) {
+                const float on2 = ((O >> x2) & 1u) ? 2.f : 0.f;
+                dq += on2 * (row[EM + x2] - kax * SA[x2 * RA + RA - 2]);  // sign^2 = +1
             }
-            q += dq;
-            for (int y = 0; y < nHp; ++y) base[y] += sgn * GPx(W, lx, Hb + y) - kax * AAx(W, Hb + y);
+            q += on * dq;
+            for (int y = 0; y < nHp; ++y) base[y] += fmaf(so, row[EM + k + y], -ko * SH[y * RH + RH - 1]);
         }
         uint32_t keep0 = 0u;  // original-key mask of the kept part of A0
         for (int x = 0; x < k; ++x)
-            if (!((R >> x) & 1u)) keep0 |= 1u << W.perm[A0b + x];
+            if (!((R >> x) & 1u)) keep0 |= 1u << W.perm[EM + x];
+        float GdS[EM];
+#pragma unroll
+        for (int j = 0; j < EM; ++j) GdS[j] = sform ? Gd[j] + lS[j] : Gd[j];
         // phase 2: depth-first over I subset of H' with |I| <= r
         int depth = 0, e = 0;
-        uint32_t imask = 0u;
+        uint32_t imask = 0u;  // local H' bits
         for (;;) {
             const int c = r - depth;  // inner keys still to add
             if (c >= 0 && c <= nL) {
                 float w[EM];
 #pragma unroll
-                for (int j = 0; j < EM; ++j) w[j] = fmaf(2.f, h[j], Gd[j]) + (sform ? lS[j] : 0.f);
+                for (int j = 0; j < EM; ++j) w[j] = fmaf(2.f, h[j], GdS[j]);
                 const float mval = inner_dispatch(c, w, q, G2);
-                if (mval <= 0.f) collect(W, keep0 | imask, w, q, c);
+                if (mval <= 0.f) collect(W, keep0, imask, w, q, c);
             }
             if (!(depth < r && e < nHp && depth < MAXD)) {
-                // back up to the next sibling
-                bool done = true;
+                bool done = true;  // back up to the next sibling
                 while (depth > 0) {
                     --depth;
                     const int pe = path[depth];
-                    imask &= ~(1u << W.perm[Hb + pe]);
+                    imask &= ~(1u << pe);
 #pragma unroll
                     for (int j = 0; j < EM; ++j) h[j] = hst[depth][j];
                     q = qst[depth];
@@ -270,34 +279,100 @@ __device__ __noinline__ void walk_row(const Walk W)
             for (int j = 0; j < EM; ++j) hst[depth][j] = h[j];
             qst[depth] = q;
             path[depth] = e;
-            push_added(W, e, depth, sform, aL, h, q, base, path, imask);
+            const float *hrow = SH + e * RH;
+#pragma unroll
+            for (int j = 0; j < EM; ++j) h[j] += hrow[j];
+            float dq = hrow[EM + e] + 2.f * base[e];
+            if (sform) dq += hrow[RH - 2];
+            for (int t = 0; t < depth; ++t) dq += hrow[EM + path[t]];
+            q += dq;
+            imask |= 1u << e;
             ++depth;
             ++e;
         }
+        R = next_same_size(R);
+        if (R < nR) R = next_same_size(R);
+        valid = R < nR;
+        }
+        // The two halves may differ by one member in this class; meet again
+        // before the next one.  Every lane in sync_mask walks the same (n, k),
+        // hence runs this loop the same number of times.
+        if (W.sync_mask) __syncwarp(W.sync_mask);
     }
 }
 
-// ---- the fast kernel: one warp = 32 rows; prologue and re-scoring are
-// warp-cooperative per row, the walk is one row per lane.
+// Write one Gram entry (or a_x / l_x) into the walk tables of a row slot.
+// Tables are described in the slot layout comment above.
+struct SlotGeom {
+    float *slot;
+    int k, nL, nHp, RA, RH, offH;
+    float kap, g0n;
+};
+__device__ __forceinline__ void put_entry(const SlotGeom &S, int la, int lb, float g, float aa, float ab)
+{
+    // row la, column lb (la != lb), g = G'_ab
+    const int eA = EM, eH = EM + S.k;
+    if (la < eA) {
+        if (lb < eA) S.slot[3 * EM + la * EM + lb] = 2.f * (g - S.kap * aa * ab);
+    } else if (la < eH) {
+        S.slot[OFF_A + (la - eA) * S.RA + lb] = g;
+    } else {
+        float *hr = S.slot + S.offH + (la - eH) * S.RH;
+        if (lb < eA) hr[lb] = g - S.kap * aa * ab;
+        else if (lb >= eH) hr[EM + (lb - eH)] = 2.f * (g - S.kap * aa * ab);
+    }
+}
+__device__ __forceinline__ void put_diag(const SlotGeom &S, int l, float g, float a)
+{
+    const int eA = EM, eH = EM + S.k;
+    if (l < eA) {
+        S.slot[l] = g - S.kap * a * a;
+        S.slot[2 * EM + l] = a;
+    } else if (l < eH) {
+        S.slot[OFF_A + (l - eA) * S.RA + l] = g;
+        S.slot[OFF_A + (l - eA) * S.RA + S.RA - 2] = a;
+    } else {
+        float *hr = S.slot + S.offH + (l - eH) * S.RH;
+        hr[EM + (l - eH)] = g - S.kap * a * a;
+        hr[S.RH - 1] = a;
+    }
+}
+__device__ __forceinline__ void put_linear(const SlotGeom &S, int l, float lin, float a)
+{
+    const int eA = EM, eH = EM + S.k;
+    if (l < eA) S.slot[EM + l] = lin - 4.f * S.kap * S.g0n * a;
+    else if (l < eH) S.slot[OFF_A + (l - eA) * S.RA + S.RA - 1] = lin;
+    else S.slot[S.offH + (l - eH) * S.RH + S.RH - 2] = lin - 4.f * S.kap * S.g0n * a;
+}
+
+constexpr int ERW = 16;  // rows per warp (two lanes per row)
+constexpr int PPL = 18;  // Gram pairs per lane: (33 * 34 / 2) / 32 rounded up
+
+// ---- the fast kernel: one warp = 16 rows; prologue and re-scoring are
+// warp-cooperative per row, the walk gives each row two lanes that split its
+// removal sets.
 template <int DPL, typename VT>
 __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
 {
     extern __shared__ float smem[];
     constexpr int d = DPL * 32;
+    constexpr int DCH = d < 64 ? d : 64;  // dimensions staged at a time
+    constexpr int TCH = DCH / 32;         // per-lane dims in one chunk
     const int lane = threadIdx.x;
-    float *slots = smem;                                                   // [32][stride]
-    float *Ust = smem + 32 * a.stride;                                     // [max_n+1][d+1] staging
-    const int ust_floats = (((a.R.max_n + 1) * (d + 1)) + 1) & ~1;        // even: keeps pscr 8-byte aligned
-    double *pscr = reinterpret_cast<double *>(Ust + ust_floats);           // [32] masses
-    uint8_t *perms = reinterpret_cast<uint8_t *>(pscr + 32);               // [32 rows][PERM]
-    uint8_t *inv = perms + 32 * PERM;                                      // [32]
-    const int64_t row0 = (int64_t)blockIdx.x * 32;
+    float *slots = smem;                                                   // [ERW][stride]
+    float *Ust = smem + ERW * a.stride;                                    // [max_n+1][DCH+1]
+    const int ust_floats = (((a.R.max_n + 1) * (DCH + 1)) + 1) & ~1;
+    float *aX = Ust + ust_floats;                                          // [32]
+    double *pscr = reinterpret_cast<double *>(aX + 32);                    // [32]
+    uint8_t *perms = reinterpret_cast<uint8_t *>(pscr + 32);               // [ERW][PERM]
+    uint8_t *inv = perms + ERW * PERM;                                     // [32]
+    const int64_t row0 = (int64_t)blockIdx.x * ERW;
 
     Walk my;
     bool my_walk = false;
 
     // ------------------------------------------------------------ prologue
-    for (int rr = 0; rr < 32; ++rr) {
+    for (int rr = 0; rr < ERW; ++rr) {
         const int64_t row = row0 + rr;
         if (row >= a.R.rows) break;
         const int64_t g = row / a.R.R;
@@ -325,9 +400,9 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
         double p = lane < n ? exp((double)l - (double)M) : 0.0;
         p = p / warp_sum_d(p);
         int rank = 0;
-        for (int s = 0; s < n; ++s) {
-            const float ls = __shfl_sync(FW_FULL, l, s);
-            rank += (ls > l) || (ls == l && s < lane);
+        for (int s2 = 0; s2 < n; ++s2) {
+            const float ls = __shfl_sync(FW_FULL, l, s2);
+            rank += (ls > l) || (ls == l && s2 < lane);
         }
         const bool inA0 = lane < n && rank < k;
         const uint32_t A0 = __ballot_sync(FW_FULL, inA0);
@@ -341,94 +416,130 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
             for (int t = 0; t < DPL; ++t)
                 mu[t] = df_add(mu[t], df_mul_f(pj, load_v(V, (int64_t)j * d + lane + 32 * t)));
         }
-        // u_j staged in fp32; g0 = sum_{A0} u_j exactly (double-float), staged as row n
-        df g0[DPL];
-#pragma unroll
-        for (int t = 0; t < DPL; ++t) g0[t] = df_zero();
-        for (int j = 0; j < n; ++j) {
-            const df pj = shfl_df(pd, j);
-            const bool in = (A0 >> j) & 1u;
-#pragma unroll
-            for (int t = 0; t < DPL; ++t) {
-                const int c = lane + 32 * t;
-                const df u = df_mul(pj, df_rsub_f(load_v(V, (int64_t)j * d + c), mu[t]));
-                Ust[j * (d + 1) + c] = u.hi;
-                if (in) g0[t] = df_add(g0[t], u);
-            }
-        }
-        df nrm = df_zero();
-#pragma unroll
-        for (int t = 0; t < DPL; ++t) {
-            nrm = df_add(nrm, df_mul(g0[t], g0[t]));
-            Ust[n * (d + 1) + lane + 32 * t] = g0[t].hi;
-        }
-        nrm = warp_sum_df(nrm);
-        const double P0 = warp_sum_d(inA0 ? p : 0.0);
-        const double g0n2 = fmax(df_to_double(nrm), 0.0);
-        const double t = g0n2 / (P0 * P0);  // es(A0)^2
-        const double sqt = sqrt(t);
-        if (lane == 0 && a.topk_gap) a.topk_gap[row] = (float)sqrt(t);
         // local key order: L = first nL keys outside A0, then A0, then H'
         const int nL = min(EM, n - k);
         const int nHp = n - k - nL;
-        const int NS = EM + k + nHp;
         uint8_t *perm = perms + rr * PERM;
         if (lane < n) {
             const uint32_t below = (1u << lane) - 1u;
-            const int bo = __popc(~A0 & below & ((n == 32) ? FW_FULL : ((1u << n) - 1u)));
+            const int bo = __popc(~A0 & below);
             const int bi = __popc(A0 & below);
             const int loc = inA0 ? EM + bi : (bo < nL ? bo : EM + k + (bo - nL));
             perm[loc] = (uint8_t)lane;
             inv[lane] = (uint8_t)loc;
             pscr[lane] = p;
         }
-        float *slot = slots + (size_t)rr * a.stride;
-        for (int i = lane; i < slot_floats(NS); i += 32) slot[i] = 0.f;
-        __syncwarp();
-        // fp32 Gram entries over the n keys plus g0 (index n), four partial sums each
+        SlotGeom S;
+        S.slot = slots + (size_t)rr * a.stride;
+        S.k = k;
+        S.nL = nL;
+        S.nHp = nHp;
+        S.RA = EM + k + nHp + 2;
+        S.RH = EM + nHp + 2;
+        S.offH = OFF_A + k * S.RA;
+        const int tot = slot_floats(k, nHp);
+        for (int i = lane; i < tot; i += 32) S.slot[i] = (i >= nL && i < EM) ? INFINITY : 0.f;
+        // Gram entries over the n keys plus g0 (index n), staged DCH dimensions at a time;
+        // each dot is four interleaved partial sums per chunk
         const int npr = (n + 1) * (n + 2) / 2;
-        const int off_a = NS * (NS + 1) / 2, off_l = off_a + NS;
-        for (int qd = lane; qd < npr; qd += 32) {
-            int x = 0, rem = qd;
+        int px_[PPL], py_[PPL];
+        float acc[PPL];
+#pragma unroll
+        for (int i = 0; i < PPL; ++i) {
+            const int qd = lane + 32 * i;
+            int x = 0, rem = qd < npr ? qd : 0;
             while (rem >= n + 1 - x) {
                 rem -= n + 1 - x;
                 ++x;
             }
-            const int y = x + rem;  // x <= y <= n
-            if (x == n) continue;   // |g0|^2 is known exactly
-            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-            const float *ux = Ust + x * (d + 1), *uy = Ust + y * (d + 1);
-#pragma unroll 4
-            for (int c = 0; c < d; c += 4) {
-                s0 = fmaf(ux[c], uy[c], s0);
-                s1 = fmaf(ux[c + 1], uy[c + 1], s1);
-                s2 = fmaf(ux[c + 2], uy[c + 2], s2);
-                s3 = fmaf(ux[c + 3], uy[c + 3], s3);
+            px_[i] = qd < npr ? x : -1;
+            py_[i] = x + rem;
+            acc[i] = 0.f;
+        }
+        df g0[DPL];
+#pragma unroll
+        for (int t = 0; t < DPL; ++t) g0[t] = df_zero();
+#pragma unroll
+        for (int ch = 0; ch < DPL / TCH; ++ch) {
+            __syncwarp();
+            for (int j = 0; j < n; ++j) {
+                const df pj = shfl_df(pd, j);
+                const bool in = (A0 >> j) & 1u;
+#pragma unroll
+                for (int tt = 0; tt < TCH; ++tt) {
+                    const int t = ch * TCH + tt;
+                    const int c = lane + 32 * t;
+                    const df u = df_mul(pj, df_rsub_f(load_v(V, (int64_t)j * d + c), mu[t]));
+                    Ust[j * (DCH + 1) + lane + 32 * tt] = u.hi;
+                    if (in) g0[t] = df_add(g0[t], u);
+                }
             }
-            const float gxy = (s0 + s1) + (s2 + s3);
-            const double px = pscr[x];
-            const int lx = inv[x];
-            if (y < n) {
-                const double py = pscr[y];
-                slot[tri_s(lx, inv[y], NS)] = (float)((double)gxy - t * px * py);
-                if (x == y) slot[off_a + lx] = sqrtf(fmaxf(gxy, 0.f)) * 1.0001f + (float)(sqt * px) * 1.0001f;
-            } else {
+#pragma unroll
+            for (int tt = 0; tt < TCH; ++tt) Ust[n * (DCH + 1) + lane + 32 * tt] = g0[ch * TCH + tt].hi;
+            __syncwarp();
+#pragma unroll
+            for (int i = 0; i < PPL; ++i) {
+                if (px_[i] < 0 || px_[i] == n) continue;  // |g0|^2 is known exactly
+                const float *ux = Ust + px_[i] * (DCH + 1), *uy = Ust + py_[i] * (DCH + 1);
+                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll 4
+                for (int c = 0; c < DCH; c += 4) {
+                    s0 = fmaf(ux[c], uy[c], s0);
+                    s1 = fmaf(ux[c + 1], uy[c + 1], s1);
+                    s2 = fmaf(ux[c + 2], uy[c + 2], s2);
+                    s3 = fmaf(ux[c + 3], uy[c + 3], s3);
+                }
+                acc[i] += (s0 + s1) + (s2 + s3);
+            }
+        }
+        df nrm = df_zero();
+#pragma unroll
+        for (int t = 0; t < DPL; ++t) nrm = df_add(nrm, df_mul(g0[t], g0[t]));
+        nrm = warp_sum_df(nrm);
+        const double P0 = warp_sum_d(inA0 ? p : 0.0);
+        const double g0n2 = fmax(df_to_double(nrm), 0.0);
+        const double t = g0n2 / (P0 * P0);  // es(A0)^2
+        const double sqt = sqrt(t);
+        if (lane == 0 && a.topk_gap) a.topk_gap[row] = (float)sqt;
+        // kappa: 2.2x the per-subset error bound of an fp32 evaluation of either form
+        const int Lc = k * (k + 1) / 2 + 2 * n + 16;
+        S.kap = (float)(2.2 * ((double)d * 0.25 + Lc + 16) * 5.9604644775390625e-8);
+        S.g0n = (float)sqrt(g0n2) * 1.0001f;
+        // a_x = |u_x| + sqrt(t) p_x (rounded up) from the diagonal entries
+#pragma unroll
+        for (int i = 0; i < PPL; ++i)
+            if (px_[i] >= 0 && px_[i] == py_[i] && px_[i] < n)
+                aX[px_[i]] = sqrtf(fmaxf(acc[i], 0.f)) * 1.0001f + (float)(sqt * pscr[px_[i]]) * 1.0001f;
+        __syncwarp();
+        // scatter the folded entries into the walk tables
+#pragma unroll
+        for (int i = 0; i < PPL; ++i) {
+            const int x = px_[i], y = py_[i];
+            if (x < 0 || x == n) continue;
+            const double pxd = pscr[x];
+            if (y == n) {
                 const double sx = ((A0 >> x) & 1u) ? -1.0 : 1.0;
-                slot[off_l + lx] = (float)(2.0 * sx * ((double)gxy - t * P0 * px));
+                put_linear(S, inv[x], (float)(2.0 * sx * ((double)acc[i] - t * P0 * pxd)), aX[x]);
+            } else {
+                const float gp = (float)((double)acc[i] - t * pxd * pscr[y]);
+                if (x == y) {
+                    put_diag(S, inv[x], gp, aX[x]);
+                } else {
+                    put_entry(S, inv[x], inv[y], gp, aX[x], aX[y]);
+                    put_entry(S, inv[y], inv[x], gp, aX[y], aX[x]);
+                }
             }
         }
         __syncwarp();
-        if (lane == rr && k <= 31) {
-            // kappa: 2x the per-subset error bound of an fp32 evaluation of either form
-            const int Lc = k * (k + 1) / 2 + 2 * n + 16;
-            my.slot = slot;
+        if ((lane & (ERW - 1)) == rr && k <= 31) {
+            my.slot = S.slot;
             my.perm = perm;
             my.k = k;
             my.nL = nL;
             my.nHp = nHp;
-            my.NS = NS;
-            my.kappa = (float)(2.2 * ((double)d * 0.25 + Lc + 12) * 5.9604644775390625e-8);
-            my.g0n = (float)sqrt(g0n2) * 1.0001f;
+            my.half = lane / ERW;
+            my.kappa = S.kap;
+            my.g0n = S.g0n;
             my.cand = a.cand + row * ECAP;
             my.ccount = a.cand_count + row;
             my_walk = true;
@@ -442,11 +553,18 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
     __syncwarp();
 
     // ------------------------------------------------------------------ walk
+    {
+        const uint32_t wmask = __ballot_sync(FW_FULL, my_walk);
+        const int key = my_walk ? (my.k << 8) | (my.nL << 16) | my.nHp : -1;
+        const int key0 = __shfl_sync(FW_FULL, key, wmask ? __ffs(wmask) - 1 : 0);
+        const bool same = __all_sync(FW_FULL, !my_walk || key == key0);
+        my.sync_mask = same ? wmask : 0u;
+    }
     if (my_walk) walk_row(my);
     __syncwarp();
 
     // ----------------------------------------------------- exact re-scoring
-    for (int rr = 0; rr < 32; ++rr) {
+    for (int rr = 0; rr < ERW; ++rr) {
         const int64_t row = row0 + rr;
         if (row >= a.R.rows) break;
         const int cc = a.cand_count[row];
@@ -490,12 +608,12 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
                 for (int t = 0; t < DPL; ++t)
                     gv[t] = df_add(gv[t], df_mul(pj, df_rsub_f(load_v(V, (int64_t)j * d + lane + 32 * t), mu[t])));
             }
-            df s = df_zero();
+            df s3 = df_zero();
 #pragma unroll
-            for (int t = 0; t < DPL; ++t) s = df_add(s, df_mul(gv[t], gv[t]));
-            s = warp_sum_df(s);
+            for (int t = 0; t < DPL; ++t) s3 = df_add(s3, df_mul(gv[t], gv[t]));
+            s3 = warp_sum_df(s3);
             const double P = warp_sum_d(((m >> lane) & 1u) ? p : 0.0);
-            const double e = fmax(df_to_double(s), 0.0) / (P * P);
+            const double e = fmax(df_to_double(s3), 0.0) / (P * P);
             const uint64_t rk = colex_rank_mask(m);
             if (e < best || (e == best && rk < brank)) {
                 best = e;
@@ -533,7 +651,8 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
     float *Usl = dyn + 33 * (d + 1);  // [33][d]
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int cnt = *a.fb_count;
-    for (int li = blockIdx.x; li < cnt; li += gridDim.x) {
+    for (int item = blockIdx.x; item < cnt * FBS; item += gridDim.x) {
+        const int li = item / FBS, chunk = item % FBS;
         const int64_t row = a.fb_list[li];
         const int64_t g = row / a.R.R;
         const int64_t ri = row - g * a.R.R;
@@ -613,9 +732,13 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
         }
         __syncthreads();
         const uint64_t total = binom64(n, k);
-        const uint64_t per = (total + blockDim.x - 1) / blockDim.x;
-        const uint64_t lo = per * tid;
-        const uint64_t hi = lo + per < total ? lo + per : total;
+        const uint64_t cper = (total + FBS - 1) / FBS;  // this block's share of the colex ranks
+        const uint64_t clo = cper * chunk;
+        const uint64_t chi = clo + cper < total ? clo + cper : total;
+        const uint64_t span = chi > clo ? chi - clo : 0;
+        const uint64_t per = (span + blockDim.x - 1) / blockDim.x;
+        const uint64_t lo = clo + per * tid;
+        const uint64_t hi = lo + per < chi ? lo + per : chi;
         double best = INFINITY;
         unsigned long long brank = ~0ull;
         if (lo < hi) {
@@ -666,38 +789,67 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
             __syncthreads();
         }
         if (tid == 0) {
-            const unsigned long long rk = ured_r[0];
-            a.best_rank[row] = rk;
-            a.best_gap[row] = (float)sqrt(ured_e[0]);
-            uint64_t r = rk;
-            int top = n - 1;
-            for (int i = k; i >= 1; --i) {
-                int c = i - 1;
-                while (c + 1 <= top && binom64(c + 1, i) <= r) ++c;
-                r -= binom64(c, i);
-                a.best_idx[row * a.k_max + (i - 1)] = c;
-                top = c - 1;
-            }
-            for (int q2 = k; q2 < a.k_max; ++q2) a.best_idx[row * a.k_max + q2] = -1;
+            a.fb_e[(int64_t)li * FBS + chunk] = ured_e[0];
+            a.fb_r[(int64_t)li * FBS + chunk] = ured_r[0];
         }
         __syncthreads();
     }
 }
 
+// merge the chunks of every exhaustive row: smallest es^2, then smallest rank
+__global__ void k_enum_exhaustive_merge(const EnumArgs a)
+{
+    const int cnt = *a.fb_count;
+    for (int li = blockIdx.x * blockDim.x + threadIdx.x; li < cnt; li += gridDim.x * blockDim.x) {
+        const int64_t row = a.fb_list[li];
+        double be = INFINITY;
+        unsigned long long br = ~0ull;
+        for (int c = 0; c < FBS; ++c) {
+            const double e = a.fb_e[(int64_t)li * FBS + c];
+            const unsigned long long r = a.fb_r[(int64_t)li * FBS + c];
+            if (e < be || (e == be && r < br)) {
+                be = e;
+                br = r;
+            }
+        }
+        const int64_t g = row / a.R.R;
+        const int n = a.R.n[g];
+        const int k = a.k[row];
+        a.best_rank[row] = br;
+        a.best_gap[row] = (float)sqrt(be);
+        uint64_t r = br;
+        int top = n - 1;
+        for (int i = k; i >= 1; --i) {
+            int c = i - 1;
+            while (c + 1 <= top && binom64(c + 1, i) <= r) ++c;
+            r -= binom64(c, i);
+            a.best_idx[row * a.k_max + (i - 1)] = c;
+            top = c - 1;
+        }
+        for (int q2 = k; q2 < a.k_max; ++q2) a.best_idx[row * a.k_max + q2] = -1;
+    }
+}
+
 }  // namespace
 
-// NS = EM + k + nHp <= max(n, EM + k): sized from the largest n and k
+// floats per row slot: the largest table set over every n <= max_n, k <= k_max (odd stride)
 static int enum_stride(int max_n, int k_max)
 {
-    const int kk = k_max < max_n ? k_max : max_n;
-    const int NS = max_n > EM + kk ? max_n : EM + kk;
-    return slot_floats(NS) | 1;
+    int best = 1;
+    for (int n = 1; n <= max_n && n <= 32; ++n)
+        for (int k = 1; k <= n && k <= k_max; ++k) {
+            const int nL = n - k < EM ? n - k : EM;
+            const int v = slot_floats(k, n - k - nL);
+            best = v > best ? v : best;
+        }
+    return best | 1;
 }
 
 size_t enum_workspace(const RowsDev &R)
 {
     const size_t rows = (size_t)R.rows;
-    return align256(rows * ECAP * 4) + align256(rows * 4) + align256(rows * 4) + 256;
+    return align256(rows * ECAP * 4) + align256(rows * 4) + align256(rows * 4) + 256 +
+           2 * align256(rows * FBS * 8);
 }
 
 fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, float *best_gap, int32_t *best_idx,
@@ -722,18 +874,25 @@ fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, f
     a.fb_list = (int32_t *)w;
     w += align256((size_t)R.rows * 4);
     a.fb_count = (int32_t *)w;
+    w += 256;
+    a.fb_e = (double *)w;
+    w += align256((size_t)R.rows * FBS * 8);
+    a.fb_r = (unsigned long long *)w;
     a.stride = enum_stride(R.max_n, k_max);
     FW_CUDA_CHECK(cudaMemsetAsync(a.fb_count, 0, sizeof(int32_t), s));
     FW_DISPATCH(R.d, R.v_dtype, {
-        const size_t smem = ((size_t)32 * a.stride + (size_t)(R.max_n + 1) * (DPL * 32 + 1) + 2) * sizeof(float) +
-                            32 * sizeof(double) + 32 * PERM + 32;
+        constexpr int DCH = DPL * 32 < 64 ? DPL * 32 : 64;
+        const size_t ust = (((size_t)(R.max_n + 1) * (DCH + 1)) + 1) & ~(size_t)1;
+        const size_t smem = ((size_t)ERW * a.stride + ust + 32) * sizeof(float) + 32 * sizeof(double) +
+                            ERW * PERM + 32;
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        const unsigned grid = (unsigned)((R.rows + 31) / 32);
+        const unsigned grid = (unsigned)((R.rows + ERW - 1) / ERW);
         FW_LAUNCH((k_enum<DPL, VT>), grid, 32, smem, s, a);
         const size_t smem2 = (size_t)33 * (2 * DPL * 32 + 1) * sizeof(float);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum_exhaustive<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)smem2));
-        FW_LAUNCH((k_enum_exhaustive<DPL, VT>), 152, 256, smem2, s, a);
+        FW_LAUNCH((k_enum_exhaustive<DPL, VT>), 152 * 4, 256, smem2, s, a);
+        FW_LAUNCH(k_enum_exhaustive_merge, 8, 128, 0, s, a);
     });
     return FW_OK;
 }
