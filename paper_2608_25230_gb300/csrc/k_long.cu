@@ -401,22 +401,4 @@ fw_status long_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out 
     return FW_OK;
 }
 
-size_t long_swap_workspace(const RowsDev &R, int nb, int E, int max_swaps)
-{
-    (void)R;
-    (void)nb;
-    (void)E;
-    (void)max_swaps;
-    return 256;
-}
-
-fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &topk, int E, int max_swaps,
-                    int32_t *n_swaps, int32_t *swap_out, int32_t *swap_in, float *refined_gap, float *topk_gap,
-                    int32_t *capped, void *ws, size_t ws_bytes, cudaStream_t s)
-{
-    (void)R, (void)k, (void)nb, (void)topk, (void)E, (void)max_swaps, (void)n_swaps, (void)swap_out;
-    (void)swap_in, (void)refined_gap, (void)topk_gap, (void)capped, (void)ws, (void)ws_bytes, (void)s;
-    return FW_ERR_UNSUPPORTED;
-}
-
 }  // namespace fw

@@ -113,3 +113,50 @@ def test_long_rows_full_scale_sampled(fw):
     assert np.all(np_(g["row_status"]) == 0)
     assert np.all(np.diff(dr, axis=1) <= 1e-7)  # nested budgets drop less mass
     assert np.all(np.isfinite(gap))
+
+
+# ------------------------------------------------------------ swap rule, long rows
+
+def check_swap_long(fw, batch, E=32, max_swaps=16):
+    from tests.parity import NEAR_TIE
+
+    rows = fw.rows_from_batch(batch)
+    k = torch.as_tensor(np.asarray(batch.k)).cuda()
+    top = fw.dense_and_topk_gap(rows, k)
+    sw = fw.swap_refine(rows, k, top, E=E, max_swaps=max_swaps)
+    torch.cuda.synchronize()
+    o = oracle.swap_refine(batch, E=E, max_swaps=max_swaps)
+    on = row_onorm(oracle.dense_and_topk_gap(batch)["o"])
+    assert_close(np_(sw["topk_gap"]), o["topk_gap"], on, "swap topk_gap")
+    exempt = (o["margin"] < NEAR_TIE) | (o["pool_margin"] < NEAR_TIE)
+    strict = ~exempt
+    assert strict.mean() > 0.5  # most decisions are not near-ties
+    np.testing.assert_array_equal(np_(sw["n_swaps"])[strict], o["n_swaps"][strict])
+    np.testing.assert_array_equal(np_(sw["swap_out"])[strict], o["swap_out"][strict])
+    np.testing.assert_array_equal(np_(sw["swap_in"])[strict], o["swap_in"][strict])
+    np.testing.assert_array_equal(np_(sw["capped"])[strict], o["capped"][strict])
+    assert_close(np_(sw["refined_gap"]), o["refined_gap"], on, "refined_gap")
+    assert np.all(np_(sw["refined_gap"]) <= np_(sw["topk_gap"]) * (1 + 1e-6))
+    return sw, o
+
+
+def test_swap_long_rows_reduced(fw):
+    b = workloads.long_rows(seed=1, heads=2, rows_per_head=6, n=2048)
+    check_swap_long(fw, b)
+
+
+@pytest.mark.parametrize("n,E", [(40, 32), (300, 8), (1000, 32)])
+def test_swap_long_shapes(fw, n, E):
+    rng = np.random.default_rng(n + E)
+    rows, d = 8, 64
+    L = (rng.normal(size=(rows, n)) * rng.uniform(0.3, 3, size=(rows, 1))).astype(np.float32)
+    L[:, 0] += 6
+    V = rng.normal(size=(rows, n, d)).astype(np.float32)
+    k = np.tile(np.array([1, max(1, n // 8), n // 2], np.int32), (rows, 1))
+    check_swap_long(fw, rows_batch(L, V, k), E=E, max_swaps=8)
+
+
+def test_swap_mixed_profiles_reduced(fw):
+    for b in workloads.mixed_profiles(seed=2, rows_scale=6e-4,
+                                      profiles=(("A", 36864, 64, 1024), ("B", 24192, 128, 4096))):
+        check_swap_long(fw, b)
