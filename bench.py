@@ -180,6 +180,22 @@ class EnumE2E:
         return res
 
 
+def combine_ranks(ms, units_per_rank, dist=None, device=None):
+    """Whole-job throughput of weak-scaling replicas: every rank processed
+    units_per_rank in its own ms; the job took the slowest rank's time.
+    Returns (units per second over all ranks, max ms)."""
+    world = 1
+    if dist is not None and dist.is_initialized():
+        import torch as _t
+
+        world = dist.get_world_size()
+        dev = device if dist.get_backend() == "nccl" else "cpu"
+        t = _t.tensor([float(ms)], dtype=_t.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return units_per_rank * world / (ms * 1e-3), ms
+
+
 def time_steps(step, K, W, flush, barrier):
     for _ in range(W):
         step()
@@ -233,20 +249,29 @@ def cpu_baseline(seed, rows_per_group=40):
 # ----------------------------------------------------------------- sections
 
 def section_long_rows(fw, device, K, W, flush, peaks):
+    """a1-a4 (top-k gap) and a5 (swap rule, E=32) on 4,096 rows x 32,768 keys."""
     b = workloads.long_rows(seed=0, backend="torch", device=device)
     rows = fw.rows_from_batch(b, device)
-    del b.logits
-    step = lambda: fw.dense_and_topk_gap(rows, rows_k, kept_bits=True)  # noqa: E731
-    rows_k = torch.tensor([[2048, 4096, 8192]], dtype=torch.int32, device=device).repeat(rows.num_rows, 1)
-    total, times = time_steps(step, K, W, flush, lambda: None)
-    ms = total / K
+    rows_k = b.k
+    holder = {}
+
+    def gap_step():
+        holder["top"] = fw.dense_and_topk_gap(rows, rows_k, kept_bits=True)
+
+    total, _ = time_steps(gap_step, K, W, flush, lambda: None)
+    ms_gap = total / K
+    top = holder["top"]
+    total, _ = time_steps(lambda: fw.swap_refine(rows, rows_k, top, E=32, max_swaps=64), max(2, K // 2), 2,
+                          flush, lambda: None)
+    ms_swap = total / max(2, K // 2)
     nbytes = (rows.logits.numel() * 4 + rows.v.numel() * 2 + rows.num_rows * (128 * 4 * 4 + 3 * 4 * 4 + 3 * 4096 * 4))
-    ach = nbytes / (ms * 1e-3) / 1e9
+    ach = nbytes / (ms_gap * 1e-3) / 1e9
     return dict(workload="long_rows: 8 heads x 512 rows, n=32768, d=128, bf16 V, k in {2048,4096,8192}",
-                path="a1-a4 (fw_dense_and_topk_gap)", metric="rows/s", value=rows.num_rows / (ms * 1e-3),
-                ms_per_step=ms, roofline=dict(bound="hbm", achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s",
-                                              frac=ach / peaks["hbm_gbs"], traffic=None,
-                                              algorithmic_bytes=nbytes))
+                path="a1-a4 (fw_dense_and_topk_gap) then a5 (fw_swap_refine, E=32)", metric="rows/s",
+                value=rows.num_rows / ((ms_gap + ms_swap) * 1e-3), gap_rows_per_s=rows.num_rows / (ms_gap * 1e-3),
+                swap_rows_per_s=rows.num_rows / (ms_swap * 1e-3), ms_gap=ms_gap, ms_swap=ms_swap,
+                roofline=dict(bound="hbm", kernel="k_long_select + k_long_pv", achieved=ach, peak=peaks["hbm_gbs"],
+                              unit="GB/s", frac=ach / peaks["hbm_gbs"], traffic=None, algorithmic_bytes=nbytes))
 
 
 def section_contour(fw, device, K, W, flush, peaks):
@@ -280,6 +305,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-sections", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--rows-scale", type=float, default=1.0,
+                    help="fraction of the headline rows (profiling captures of a smaller case)")
     args = ap.parse_args()
     K, W = args.steps, max(3, args.warmup)
 
@@ -324,7 +351,7 @@ def main():
     flush = L2Flush(device)
     barrier = (lambda: dist.barrier()) if dist else (lambda: None)
 
-    wl = EnumWorkload(fw, seed=rank, device=device)
+    wl = EnumWorkload(fw, seed=rank, device=device, rows_scale=args.rows_scale)
     torch.cuda.synchronize()
     l0 = fw.launch_count()
     with ClockSampler(local) as clk:
@@ -333,12 +360,7 @@ def main():
     launches_timed = launches * K
     enum_ev = wl.enum_times()[-5 * K:]
     clocks = clk.summary()
-    ms = total_ms / K
-    if dist:
-        t = torch.tensor([ms], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = wl.subsets * world / (ms * 1e-3)
+    value, ms = combine_ranks(total_ms / K, wl.subsets, dist, device)
 
     # roofline of the dominant kernel (the exact-search walk, fw_best_subset)
     enum_ms = sum(t for t, _ in enum_ev) / K  # per step, all five groups
@@ -350,11 +372,7 @@ def main():
     # end to end through the public API with host buffers
     e2e = EnumE2E(wl)
     e2e_total, _ = time_steps(e2e.step, max(3, K // 2), W, flush, barrier)
-    e2e_ms = e2e_total / max(3, K // 2)
-    if dist:
-        t = torch.tensor([e2e_ms], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_value, e2e_ms = combine_ranks(e2e_total / max(3, K // 2), wl.subsets, dist, device)
 
     sections = {}
     if not args.no_sections and rank == 0:
@@ -378,7 +396,7 @@ def main():
                               traffic=None, kernel="k_enum (fw_best_subset)", launch_ms=enum_launch_ms,
                               ops_per_subset=ALU_OPS_PER_SUBSET,
                               peak_basis=f"152 SMs x 128 fp32 lanes x {sm_mhz:.0f} MHz (median SM clock under load)"),
-                e2e=dict(value=wl.subsets * world / (e2e_ms * 1e-3), unit="subsets/s",
+                e2e=dict(value=e2e_value, unit="subsets/s",
                          h2d_bytes_per_step=e2e.h2d, d2h_bytes_per_step=e2e.d2h),
                 gpu_launches=int(launches_timed), clocks=clocks, peaks_source=peaks["source"])
     if cpu:
