@@ -76,7 +76,7 @@ typedef struct {
     const float *logits;    /* device                                          */
     const int64_t *logit_off; /* device [num_groups], element offsets          */
     const int32_t *n;       /* device [num_groups]                             */
-    const void *v;          /* device                                          */
+    const void *v;          /* device, 16-byte aligned                         */
     const int64_t *v_off;   /* device [num_groups], element offsets, multiples of 8 */
 } fw_rows;
 
@@ -132,7 +132,7 @@ typedef struct {
  * [rows][nb][max_swaps] (removed / added key of each swap in the order taken;
  * entries past n_swaps are -1); refined_gap [rows][nb]; topk_gap [rows][nb]
  * (may be NULL); capped [rows][nb] = 1 if max_swaps stopped the search (may be
- * NULL). */
+ * NULL).  Rows with max_n > 32 accept E <= 96 (FW_ERR_UNSUPPORTED above). */
 fw_status fw_swap_refine(const fw_rows *rows, const int32_t *k, int32_t nb, const fw_gap_out *topk,
                          const fw_swap_params *prm, int32_t *n_swaps, int32_t *swap_out,
                          int32_t *swap_in, float *refined_gap, float *topk_gap, int32_t *capped,

@@ -16,6 +16,7 @@ static fw_status check_rows(const fw_rows *r, RowsDev &R)
     if (r->v_dtype != FW_F32 && r->v_dtype != FW_BF16) return FW_ERR_INVALID_ARG;
     if (r->num_groups > 0 && (!r->logits || !r->logit_off || !r->n || !r->v || !r->v_off))
         return FW_ERR_INVALID_ARG;
+    if (((uintptr_t)r->v & 15u) != 0) return FW_ERR_INVALID_ARG;  // rows are read in 16-byte vectors
     R.num_groups = r->num_groups;
     R.R = r->rows_per_group;
     R.rows = r->num_groups * (int64_t)r->rows_per_group;
@@ -102,6 +103,7 @@ fw_status fw_swap_refine(const fw_rows *rows, const int32_t *k, int32_t nb, cons
     if (R.max_n <= 32)
         return small_swap(R, k, nb, *topk, prm->E, prm->max_swaps, n_swaps, swap_out, swap_in,
                           refined_gap, topk_gap, capped, s);
+    if (prm->E > kLongSwapMaxE) return FW_ERR_UNSUPPORTED;
     if (workspace_bytes < long_swap_workspace(R, nb, prm->E, prm->max_swaps) || !workspace ||
         !aligned(workspace, 256))
         return FW_ERR_WORKSPACE;

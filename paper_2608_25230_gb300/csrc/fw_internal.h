@@ -33,9 +33,20 @@ fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, f
                       void *ws, size_t ws_bytes, cudaStream_t s);
 
 // Long rows (any n): row statistics + radix top-k, then the P.V products.
+// Per-row results of the select kernel that the P.V kernels read.
+struct LongWs {
+    float *M, *Z;          // [rows]
+    uint32_t *tk;          // [rows][nb]
+    int32_t *ti;           // [rows][nb]
+    int32_t *status;       // [rows]
+};
+bool long_pv_tc_supported(const RowsDev &R, int nb);
+fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, const LongWs &L,
+                     cudaStream_t s);
 size_t long_gap_workspace(const RowsDev &R, int nb);
 fw_status long_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, void *ws,
                    size_t ws_bytes, cudaStream_t s);
+constexpr int kLongSwapMaxE = 96;  // largest pool the long-row selector stages in shared memory
 size_t long_swap_workspace(const RowsDev &R, int nb, int E, int max_swaps);
 fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &topk, int E,
                     int max_swaps, int32_t *n_swaps, int32_t *swap_out, int32_t *swap_in,

@@ -18,15 +18,9 @@ namespace fw {
 namespace {
 
 constexpr int LT = 256;  // threads of the select kernel
+constexpr int kSelStageMax = 32768;  // longest row whose keys the select kernel stages (128 KB)
 constexpr int RT = 8;    // rows per P.V tile
 constexpr int JT = 64;   // keys per staged chunk
-
-struct LongWs {
-    float *M, *Z;          // [rows]
-    uint32_t *tk;          // [rows][nb]
-    int32_t *ti;           // [rows][nb]
-    int32_t *status;       // [rows]
-};
 
 struct SelArgs {
     RowsDev R;
@@ -73,8 +67,13 @@ __device__ __forceinline__ void block_max_sum(float &m, float &s, float *red_m, 
     __syncthreads();
 }
 
+// STAGED: the row's order keys are kept in shared memory (rows of at most
+// kSelStageMax keys), so the logits are read from HBM once; otherwise every
+// pass re-reads them.
+template <bool STAGED>
 __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
 {
+    extern __shared__ uint32_t skeys[];  // [n] order keys when STAGED
     __shared__ uint32_t hist[4][256];
     __shared__ float red_m[32], red_s[32];
     __shared__ uint32_t s_prefix[4], s_rem[4];
@@ -88,13 +87,15 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
     const int n = a.R.n[g];
     const int nb = a.nb;
     const float *lg = a.R.logits + a.R.logit_off[g] + ri * n;
+    auto key_at = [&](int j) -> uint32_t { return STAGED ? skeys[j] : order_key(lg[j]); };
     if (tid == 0) s_bad = 0;
     __syncthreads();
-    // online max / sum of exp
+    // online max / sum of exp (and the staged keys)
     float m = -INFINITY, s = 0.f;
     bool bad = n < 1;
     for (int j = tid; j < n; j += LT) {
         const float x = lg[j];
+        if (STAGED) skeys[j] = order_key(x);
         if (!isfinite(x)) {
             bad = true;
             continue;
@@ -138,7 +139,7 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
 #pragma unroll
         for (int b = 0; b < 4; ++b) pre[b] = b < nb ? s_prefix[b] : 0u;
         for (int j = tid; j < n; j += LT) {
-            const uint32_t key = order_key(lg[j]);
+            const uint32_t key = key_at(j);
 #pragma unroll
             for (int b = 0; b < 4; ++b)
                 if (b < nb && (key & pmask) == pre[b]) atomicAdd(&hist[b][(key >> shift) & 255u], 1u);
@@ -168,7 +169,7 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
         __syncthreads();
         for (int j0 = 0; j0 < n; j0 += LT) {
             const int j = j0 + tid;
-            const bool match = j < n && order_key(lg[j]) == T;
+            const bool match = j < n && key_at(j) == T;
             const uint32_t bal = __ballot_sync(FW_FULL, match);
             if (lane == 0) wcnt[wid] = __popc(bal);
             __syncthreads();
@@ -201,7 +202,7 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
                 const int j = w0 + tid;
                 bool kept = false;
                 if (j < n) {
-                    const uint32_t key = order_key(lg[j]);
+                    const uint32_t key = key_at(j);
                     kept = key > T || (key == T && j <= ti);
                 }
                 const uint32_t bal = __ballot_sync(FW_FULL, kept);
@@ -394,7 +395,14 @@ fw_status long_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out 
     (void)ws_bytes;
     const LongWs L = carve(R, nb, ws);
     const SelArgs sa{R, k, nb, out, L};
-    FW_LAUNCH(k_long_select, (unsigned)R.rows, LT, 0, s, sa);
+    if (R.max_n <= kSelStageMax) {
+        const size_t smem = (size_t)R.max_n * 4;
+        FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_select<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        FW_LAUNCH(k_long_select<true>, (unsigned)R.rows, LT, smem, s, sa);
+    } else {
+        FW_LAUNCH(k_long_select<false>, (unsigned)R.rows, LT, 0, s, sa);
+    }
+    if (long_pv_tc_supported(R, nb)) return long_pv_tc(R, k, nb, out, L, s);
     PvArgs pa{R, k, nb, out, L, (R.R + RT - 1) / RT};
     const unsigned grid = (unsigned)(R.num_groups * pa.tiles_per_group);
     FW_DISPATCH(R.d, R.v_dtype, FW_LAUNCH((k_long_pv<DPL, VT>), grid, DPL * 32, 0, s, pa));

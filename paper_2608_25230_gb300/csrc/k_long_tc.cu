@@ -1,0 +1,417 @@
+// k_long_tc.cu -- the P.V products of the long-row path (dense output mu,
+// forced-weight outputs m_A, gaps and dropped mass; Definition 2.1, Sec. 2.1,
+// Lemma 2.1) on the 5th-generation tensor cores, for bf16 values.
+//
+// For a tile of RT rows of one group (rows sharing V) the kernel forms
+//   S[b][r][:] = sum_j [band(r, j) = b] p_rj v_j,   b = 0..nb,
+// where band(r, j) = number of budgets of row r that drop key j, as one GEMM:
+// A = (band, row) x keys, 128 x 64 per stage, B = keys x d (V itself), the
+// fp32 accumulator D = 128 x d in tensor memory.  Each probability is split
+// into three bf16 terms (hi + mid + lo reproduce the fp32 value to ~2^-24), so
+// with bf16 V every product is exact and only the fp32 accumulation rounds,
+// as on the CUDA cores.  The A tiles are written by the producer warps
+// (exp, band, split) in the 128-byte-swizzled K-major layout; V tiles arrive
+// by cp.async in the 128-byte-swizzled MN-major layout; one thread issues
+// tcgen05.mma and tcgen05.commit frees each stage.  The tensor core rounds its
+// fp32 accumulation toward zero, which over thousands of additions into one
+// accumulator biases the sums by ~1e-3; so every stage accumulates into a fresh
+// TMEM buffer (two, alternating) and the producers add it into fp32 registers
+// with round-to-nearest once the stage's MMAs complete.  The epilogue combines
+// the bands exactly as the CUDA-core kernel does:
+//   N_A = sum of the bands inside A, N_{A^c} = the rest,
+//   p(A) (m_A - mu) = pbar(A) N_A - p(A) N_{A^c}.
+#include <cuda_bf16.h>
+
+#include "fw_internal.h"
+#include "tc_sm100.cuh"
+
+namespace fw {
+namespace {
+
+constexpr int TM = 128;       // rows of the MMA tile: (band, row) pairs, band-major
+constexpr int KS = 64;        // keys per stage: one 128-byte swizzle atom of bf16
+constexpr int PW = 8;         // producer warps
+constexpr int NT = (PW + 1) * 32;
+constexpr int NPROD = PW * 32;
+constexpr int NSPLIT = 3;     // bf16 terms per probability
+constexpr int ASLOTS = 2;     // A tiles in flight
+constexpr int BSLOTS = 3;     // V / logit tiles in flight (prefetch distance 2)
+constexpr int MAXRT = 64;     // rows per tile for two bands
+constexpr uint32_t WAIT_POLLS = 1u << 20;  // polls before a wait gives up (well over a second)
+constexpr int A_SPLIT_BYTES = TM * 128;            // 16 KB
+constexpr int A_SLOT_BYTES = NSPLIT * A_SPLIT_BYTES;  // 48 KB
+
+struct TcArgs {
+    RowsDev R;
+    const int32_t *k;
+    int nb;
+    fw_gap_out out;
+    LongWs ws;
+    int tiles_per_group;
+    int RT;
+};
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void *src, uint32_t src_bytes)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait2() { asm volatile("cp.async.wait_group 2;" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t bf16_bits_rn(float x)
+{
+    return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(x));
+}
+
+template <int D>
+__global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
+{
+    constexpr int B_SLOT_BYTES = D * 128;  // KS keys x D bf16
+    constexpr int NC = D / 8;              // 16-byte chunks per V row
+    extern __shared__ uint8_t smraw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~(uintptr_t)1023);
+    uint8_t *sA = sm;                                  // [ASLOTS][NSPLIT][TM x 128 B]
+    uint8_t *sB = sA + ASLOTS * A_SLOT_BYTES;          // [BSLOTS][D/64][KS x 128 B]
+    float *sL = reinterpret_cast<float *>(sB + BSLOTS * B_SLOT_BYTES);  // [BSLOTS][RT][KS] raw logits
+    float *acc = reinterpret_cast<float *>(sA);       // epilogue: [TM][D + 1]
+    __shared__ __align__(8) uint64_t full[BSLOTS], empty[BSLOTS], accfree[2];
+    __shared__ uint32_t s_taddr;
+    __shared__ int s_err;
+    __shared__ float rowM[MAXRT], rowZi[MAXRT];
+    __shared__ uint32_t rtk[MAXRT][4];
+    __shared__ int32_t rti[MAXRT][4];
+    __shared__ int rok[MAXRT];
+    __shared__ float bmass[MAXRT][5];
+
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int nb = a.nb, nbb = nb + 1, RT = a.RT;
+    const int64_t g = blockIdx.x / a.tiles_per_group;
+    const int tile = (int)(blockIdx.x - g * a.tiles_per_group);
+    const int r0 = tile * RT;
+    const int nr = min(RT, a.R.R - r0);
+    const int n = a.R.n[g];
+    const uint16_t *V = reinterpret_cast<const uint16_t *>(a.R.v) + a.R.v_off[g];
+    const float *LG = a.R.logits + a.R.logit_off[g];
+    const int nst = (n + KS - 1) / KS;
+
+    if (tid < MAXRT) {
+        const int r = tid;
+        rok[r] = 0;
+        if (r < nr) {
+            const int64_t row = g * a.R.R + r0 + r;
+            rok[r] = a.ws.status[row] == FW_OK;
+            rowM[r] = a.ws.M[row];
+            rowZi[r] = 1.f / a.ws.Z[row];
+            for (int b = 0; b < 4; ++b) {
+                rtk[r][b] = b < nb ? a.ws.tk[row * nb + b] : 0u;
+                rti[r][b] = b < nb ? a.ws.ti[row * nb + b] : -1;
+            }
+        }
+    }
+    if (tid == 0) {
+        s_err = 0;
+        for (int s = 0; s < BSLOTS; ++s) {
+            tc::mbar_init(&full[s], NPROD);
+            tc::mbar_init(&empty[s], 1);
+        }
+        for (int x = 0; x < 2; ++x) tc::mbar_init(&accfree[x], NPROD);
+        tc::mbar_init_fence();
+    }
+    // rows of A past nbb * RT stay zero in every slot
+    for (int e = tid; e < ASLOTS * NSPLIT * TM * 8; e += NT) {
+        const int m = (e / 8) % TM;
+        if (m >= nbb * RT) reinterpret_cast<uint4 *>(sA)[e] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    tc::fence_async_smem();
+    if (wid == PW) tc::tmem_alloc(&s_taddr, 2 * D);  // two stage accumulators
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t taddr = s_taddr;
+
+    if (wid == PW) {
+        // ---------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(TM, D, false, true);
+            const uint32_t a0 = tc::smem_u32(sA), b0 = tc::smem_u32(sB);
+            bool ok = true;
+            for (int it = 0; it < nst && ok; ++it) {
+                const int bs = it % BSLOTS, as = it % ASLOTS;
+                ok = tc::mbar_wait(&full[bs], (uint32_t)(it / BSLOTS) & 1u, WAIT_POLLS);
+                // accumulator it % 2 was last read by the producers after stage it - 2
+                if (ok && it >= 2) ok = tc::mbar_wait(&accfree[it & 1], (uint32_t)((it - 2) >> 1) & 1u, WAIT_POLLS);
+                if (!ok) break;
+                tc::fence_after_sync();
+                const uint32_t dacc = taddr + (uint32_t)((it & 1) * D);
+#pragma unroll
+                for (int ks = 0; ks < KS / 16; ++ks) {
+                    const uint64_t bd = tc::sdesc_sw128(b0 + bs * B_SLOT_BYTES + ks * 2048, KS * 128, 1024);
+#pragma unroll
+                    for (int sp = 0; sp < NSPLIT; ++sp) {
+                        const uint64_t ad =
+                            tc::sdesc_sw128(a0 + as * A_SLOT_BYTES + sp * A_SPLIT_BYTES + ks * 32, 16, 1024);
+                        tc::mma_bf16(dacc, ad, bd, idesc, ks > 0 || sp > 0);
+                    }
+                }
+                tc::commit(&empty[bs]);
+            }
+            if (!ok) atomicOr(&s_err, 1);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ producers
+        const int ptid = tid;                 // 0..NPROD-1
+        const int kc = ptid & 7;              // 8-key chunk of the stage
+        const int rr0 = ptid >> 3;            // first row handled (rows rr0, rr0 + 32)
+        float bm[2][5];
+#pragma unroll
+        for (int q = 0; q < 2; ++q)
+#pragma unroll
+            for (int b = 0; b < 5; ++b) bm[q][b] = 0.f;
+        bool ok = true;
+        const uint32_t bbase = tc::smem_u32(sB), lbase = tc::smem_u32(sL);
+        // this thread's accumulator entries: TMEM lane 32 (wid % 4) + lane, columns of half wid / 4
+        const int quarter = wid & 3, half = wid >> 2;
+        float racc[D / 2];
+#pragma unroll
+        for (int i = 0; i < D / 2; ++i) racc[i] = 0.f;
+        auto flush = [&](int st) {  // add the accumulator of stage st once its MMAs completed
+            if (ok) ok = tc::mbar_wait(&empty[st % BSLOTS], (uint32_t)(st / BSLOTS) & 1u, WAIT_POLLS);
+            tc::fence_after_sync();
+            const uint32_t base = taddr + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((st & 1) * D + half * (D / 2));
+#pragma unroll
+            for (int c0 = 0; c0 < D / 2; c0 += 32) {
+                float v[32];
+                tc::ld32(base + c0, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) racc[c0 + i] += v[i];
+            }
+            tc::fence_before_sync();
+            tc::mbar_arrive(&accfree[st & 1]);
+        };
+        auto issue = [&](int st) {  // cp.async of stage st's V tile and this thread's logits
+            if (st < nst) {
+                const int bs = st % BSLOTS, j0 = st * KS;
+                for (int e = ptid; e < KS * NC; e += NPROD) {
+                    const int kk = e / NC, nc = e % NC;
+                    const int j = j0 + kk;
+                    const int n2 = nc >> 3, c = nc & 7;
+                    const uint32_t dst = bbase + bs * B_SLOT_BYTES + n2 * (KS * 128) + (kk >> 3) * 1024 +
+                                         (kk & 7) * 128 + ((c ^ (kk & 7)) << 4);
+                    const bool in = j < n;
+                    cp_async16(dst, V + (int64_t)(in ? j : 0) * D + nc * 8, in ? 16u : 0u);
+                }
+                for (int r = rr0; r < RT; r += 32) {
+                    const bool live = r < nr && rok[r];
+                    const float *lrow = LG + (int64_t)(r0 + (live ? r : 0)) * n;
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const int j = j0 + kc * 8 + u;
+                        const bool in = live && j < n;
+                        cp_async4(lbase + ((bs * RT + r) * KS + kc * 8 + u) * 4, lrow + (in ? j : 0), in ? 4u : 0u);
+                    }
+                }
+            }
+            cp_async_commit();
+        };
+        issue(0);
+        issue(1);
+        for (int it = 0; it < nst; ++it) {
+            const int bs = it % BSLOTS, as = it % ASLOTS;
+            // the V / logit slot of stage it + 2 was last read by the MMAs of stage it - 1
+            if (ok && it >= 1 && it + 2 < nst) {
+                const int pst = it - 1;
+                ok = tc::mbar_wait(&empty[pst % BSLOTS], (uint32_t)(pst / BSLOTS) & 1u, WAIT_POLLS);
+            }
+            issue(it + 2);
+            cp_async_wait2();  // this thread's copies of stage it are in shared memory
+            // the A slot of stage it was last read by the MMAs of stage it - 2
+            if (ok && it >= ASLOTS) {
+                const int pst = it - ASLOTS;
+                ok = tc::mbar_wait(&empty[pst % BSLOTS], (uint32_t)(pst / BSLOTS) & 1u, WAIT_POLLS);
+            }
+            uint8_t *aslot = sA + as * A_SLOT_BYTES;
+            const int j0 = it * KS;
+            for (int q = 0, r = rr0; r < RT; ++q, r += 32) {
+                const float *lr = sL + (bs * RT + r) * KS + kc * 8;
+                const bool live = r < nr && rok[r];
+                const float Mr = live ? rowM[r] : 0.f, Zr = live ? rowZi[r] : 0.f;
+                uint32_t h16[8], m16[8], l16[8];
+                int band[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int j = j0 + kc * 8 + u;
+                    float p = 0.f;
+                    int bd = 0;
+                    if (live && j < n) {
+                        const float x = lr[u];
+                        p = expf(x - Mr) * Zr;
+                        const uint32_t key = order_key(x);
+                        for (int b = 0; b < nb; ++b)
+                            bd += !(key > rtk[r][b] || (key == rtk[r][b] && j <= rti[r][b]));
+                    }
+                    band[u] = bd;
+#pragma unroll
+                    for (int b = 0; b < 5; ++b) bm[q & 1][b] += bd == b ? p : 0.f;
+                    h16[u] = bf16_bits_rn(p);
+                    const float r1 = p - __uint_as_float(h16[u] << 16);
+                    m16[u] = bf16_bits_rn(r1);
+                    l16[u] = bf16_bits_rn(r1 - __uint_as_float(m16[u] << 16));
+                }
+                for (int b = 0; b < nbb; ++b) {
+                    const int m = b * RT + r;
+                    const uint32_t off = (m >> 3) * 1024 + (m & 7) * 128 + ((kc ^ (m & 7)) << 4);
+                    uint32_t w[NSPLIT][4];
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const bool e0 = band[2 * h] == b, e1 = band[2 * h + 1] == b;
+                        w[0][h] = (e0 ? h16[2 * h] : 0u) | ((e1 ? h16[2 * h + 1] : 0u) << 16);
+                        w[1][h] = (e0 ? m16[2 * h] : 0u) | ((e1 ? m16[2 * h + 1] : 0u) << 16);
+                        w[2][h] = (e0 ? l16[2 * h] : 0u) | ((e1 ? l16[2 * h + 1] : 0u) << 16);
+                    }
+#pragma unroll
+                    for (int sp = 0; sp < NSPLIT; ++sp)
+                        *reinterpret_cast<uint4 *>(aslot + sp * A_SPLIT_BYTES + off) =
+                            make_uint4(w[sp][0], w[sp][1], w[sp][2], w[sp][3]);
+                }
+            }
+            tc::fence_async_smem();
+            tc::mbar_arrive(&full[bs]);
+            if (it >= 1) flush(it - 1);
+        }
+        flush(nst - 1);
+        // band masses: the 8 threads of a row sit in consecutive lanes
+#pragma unroll
+        for (int q = 0; q < 2; ++q)
+#pragma unroll
+            for (int b = 0; b < 5; ++b) {
+                float v = bm[q][b];
+                v += __shfl_xor_sync(FW_FULL, v, 1);
+                v += __shfl_xor_sync(FW_FULL, v, 2);
+                v += __shfl_xor_sync(FW_FULL, v, 4);
+                bm[q][b] = v;
+            }
+        for (int q = 0, r = rr0; r < RT; ++q, r += 32)
+            if (kc == 0)
+                for (int b = 0; b < 5; ++b) bmass[r][b] = bm[q & 1][b];
+        // accumulators -> shared for the per-row epilogue (the stage buffers are idle now)
+        if (!ok) atomicOr(&s_err, 1);
+        {
+            const int m = quarter * 32 + lane;
+#pragma unroll
+            for (int i = 0; i < D / 2; ++i) acc[m * (D + 1) + half * (D / 2) + i] = racc[i];
+        }
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    if (wid == PW) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(taddr, 2 * D);
+        return;
+    }
+    // --------------------------------------------------------------- epilogue
+    const bool failed = s_err != 0;
+    constexpr int CPT = D / 32;
+    for (int r = wid; r < nr; r += PW) {
+        const int64_t row = g * a.R.R + r0 + r;
+        if (failed) {
+            if (lane == 0 && a.out.row_status) a.out.row_status[row] = FW_ERR_TIMEOUT;
+            continue;
+        }
+        if (!rok[r]) continue;
+        float S[5][CPT];
+#pragma unroll
+        for (int b = 0; b < 5; ++b)
+#pragma unroll
+            for (int t = 0; t < CPT; ++t)
+                S[b][t] = b < nbb ? acc[(b * RT + r) * (D + 1) + lane + 32 * t] : 0.f;
+        if (a.out.o) {
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) {
+                float o = 0.f;
+#pragma unroll
+                for (int b = 0; b < 5; ++b) o += S[b][t];
+                a.out.o[row * D + lane + 32 * t] = o;
+            }
+        }
+        for (int b = 0; b < nb; ++b) {
+            const int kb = a.k[row * nb + b];
+            int sb = 0;
+            for (int b2 = 0; b2 < nb; ++b2) {
+                const int k2 = a.k[row * nb + b2];
+                sb += (k2 < kb) || (k2 == kb && b2 < b);
+            }
+            float PA = 0.f, PC = 0.f;
+            for (int q = 0; q < 5; ++q) {
+                if (q <= sb) PA += bmass[r][q];
+                else PC += bmass[r][q];
+            }
+            float s2 = 0.f;
+            float NAv[CPT];
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) {
+                float NA = 0.f, NC = 0.f;
+#pragma unroll
+                for (int q = 0; q < 5; ++q) {
+                    if (q <= sb) NA += S[q][t];
+                    else NC += S[q][t];
+                }
+                NAv[t] = NA;
+                const float diff = PC * NA - PA * NC;  // p(A) (m_A - mu)
+                s2 = fmaf(diff, diff, s2);
+            }
+            s2 = warp_sum(s2);
+            if (lane == 0) {
+                const float phi = sqrtf(s2);
+                a.out.gap[row * nb + b] = phi / PA;
+                a.out.dropped[row * nb + b] = PC;
+                if (a.out.phi) a.out.phi[row * nb + b] = phi;
+            }
+            if (a.out.o_kept)
+#pragma unroll
+                for (int t = 0; t < CPT; ++t) a.out.o_kept[(row * nb + b) * D + lane + 32 * t] = NAv[t] / PA;
+        }
+    }
+}
+
+template <int D> size_t tc_smem(int RT)
+{
+    return 1024 + (size_t)ASLOTS * A_SLOT_BYTES + (size_t)BSLOTS * D * 128 + (size_t)BSLOTS * RT * KS * 4;
+}
+
+}  // namespace
+
+bool long_pv_tc_supported(const RowsDev &R, int nb)
+{
+    return R.v_dtype == FW_BF16 && (R.d == 64 || R.d == 128) && nb >= 1 && nb <= 4;
+}
+
+fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, const LongWs &L,
+                     cudaStream_t s)
+{
+    TcArgs a;
+    a.R = R;
+    a.k = k;
+    a.nb = nb;
+    a.out = out;
+    a.ws = L;
+    a.RT = TM / (nb + 1);
+    a.tiles_per_group = (R.R + a.RT - 1) / a.RT;
+    const unsigned grid = (unsigned)(R.num_groups * a.tiles_per_group);
+    if (R.d == 128) {
+        const size_t smem = tc_smem<128>(a.RT);
+        FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_pv_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        FW_LAUNCH(k_long_pv_tc<128>, grid, NT, smem, s, a);
+    } else {
+        const size_t smem = tc_smem<64>(a.RT);
+        FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_pv_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        FW_LAUNCH(k_long_pv_tc<64>, grid, NT, smem, s, a);
+    }
+    return FW_OK;
+}
+
+}  // namespace fw

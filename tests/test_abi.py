@@ -61,4 +61,15 @@ def test_host_validation_rejects_bad_arguments(lib):
     rows = fw.FwRows(1, 1, 64, 33, 0, *([C.c_void_p(256)] * 5))
     assert fw._lib.fw_best_subset(C.byref(rows), C.c_void_p(256), *([C.c_void_p(256)] * 3), 8, None, None,
                                   C.c_void_p(256), 1 << 20, None) == fw.FW_ERR_UNSUPPORTED
+    # value rows must be 16-byte aligned; the long-row selector stages at most 96 pool keys
+    rows = fw.FwRows(1, 1, 64, 64, 1, C.c_void_p(256), C.c_void_p(256), C.c_void_p(256), C.c_void_p(264),
+                     C.c_void_p(256))
+    assert fw._lib.fw_dense_and_topk_gap(C.byref(rows), C.c_void_p(256), 1, C.byref(out), C.c_void_p(256), 1 << 30,
+                                         None) == fw.FW_ERR_INVALID_ARG
+    rows = fw.FwRows(1, 1, 64, 64, 1, *([C.c_void_p(256)] * 5))
+    top = fw.FwGapOut()
+    top.o = top.row_max = top.row_sum = top.thr_key = top.thr_idx = 256
+    prm = fw.FwSwapParams(97, 4)
+    assert fw._lib.fw_swap_refine(C.byref(rows), C.c_void_p(256), 1, C.byref(top), C.byref(prm),
+                                  *([C.c_void_p(256)] * 6), C.c_void_p(256), 1 << 40, None) == fw.FW_ERR_UNSUPPORTED
     assert fw.launch_count() == before  # nothing was launched
