@@ -70,6 +70,12 @@ __device__ __forceinline__ void block_max_sum(float &m, float &s, float *red_m, 
 // STAGED: the row's order keys are kept in shared memory (rows of at most
 // kSelStageMax keys), so the logits are read from HBM once; otherwise every
 // pass re-reads them.
+// The float of an order key (inverse of order_key; -0 comes back as +0).
+__device__ __forceinline__ float key_float(uint32_t k)
+{
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
 template <bool STAGED>
 __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
 {
@@ -90,25 +96,47 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
     auto key_at = [&](int j) -> uint32_t { return STAGED ? skeys[j] : order_key(lg[j]); };
     if (tid == 0) s_bad = 0;
     __syncthreads();
-    // online max / sum of exp (and the staged keys)
     float m = -INFINITY, s = 0.f;
     bool bad = n < 1;
-    for (int j = tid; j < n; j += LT) {
-        const float x = lg[j];
-        if (STAGED) skeys[j] = order_key(x);
-        if (!isfinite(x)) {
-            bad = true;
-            continue;
+    if (STAGED) {
+        // max and staged keys (independent loads, no branch), then sum of exp from shared memory
+#pragma unroll 8
+        for (int j = tid; j < n; j += LT) {
+            const float x = lg[j];
+            skeys[j] = order_key(x);
+            bad |= !isfinite(x);
+            m = fmaxf(m, x);
         }
-        if (x > m) {
-            s = s * expf(m - x) + 1.f;
-            m = x;
-        } else {
-            s += expf(x - m);
+        if (bad) atomicOr(&s_bad, 1);
+        m = warp_max(m);
+        if (lane == 0) red_m[wid] = m;
+        __syncthreads();
+        m = red_m[0];
+        for (int w = 1; w < LT / 32; ++w) m = fmaxf(m, red_m[w]);
+        for (int j = tid; j < n; j += LT) s += expf(key_float(skeys[j]) - m);
+        s = warp_sum(s);
+        if (lane == 0) red_s[wid] = s;
+        __syncthreads();
+        s = 0.f;
+        for (int w = 0; w < LT / 32; ++w) s += red_s[w];
+    } else {
+        // online max / sum of exp
+        for (int j = tid; j < n; j += LT) {
+            const float x = lg[j];
+            if (!isfinite(x)) {
+                bad = true;
+                continue;
+            }
+            if (x > m) {
+                s = s * expf(m - x) + 1.f;
+                m = x;
+            } else {
+                s += expf(x - m);
+            }
         }
+        if (bad) atomicOr(&s_bad, 1);
+        block_max_sum(m, s, red_m, red_s);
     }
-    if (bad) atomicOr(&s_bad, 1);
-    block_max_sum(m, s, red_m, red_s);
     int status = s_bad ? FW_ERR_NONFINITE : FW_OK;
     if (status == FW_OK) {
         for (int b = 0; b < nb; ++b) {

@@ -113,38 +113,36 @@ __device__ __forceinline__ void ld8(const float *p, float (&x)[8])
     x[4] = b.x, x[5] = b.y, x[6] = b.z, x[7] = b.w;
 }
 
-// D_ij / P'^2 for one pair (the fast form of the file comment), and the scale
-// of the terms it cancels: its rounding error is a few ulps of *terms / P'^2.
-// The form loses everything when P' << P or |g'| << |g| (a swap that removes
-// most of the kept mass); such pairs are scored by vector_score instead.
+// D_ij / P'^2 for one pair (the fast form of the file comment).
 __device__ __forceinline__ float pair_score(float alpha, float p_i, float p_j, float beta, float cij, float P,
-                                           float P2, float N, float s_i, float r_j, float sqN, float *terms)
+                                           float P2, float N)
 {
     const float cross = p_i * p_j * cij;
     const float delta = alpha + beta - 2.f * cross;
     const float dp = p_j - p_i;
     const float Pp = P + dp;
     const float D = delta * P2 - N * dp * (2.f * P + dp);
-    const float sr = s_i + r_j;
-    *terms = (sr * sr + 2.f * sqN * sr) * P2 + N * fabsf(dp) * (2.f * P + fabsf(dp));
     return D / (Pp * Pp);
 }
 
-// The fast form is trusted when its terms stay below 4 N P'^2 (rounding error
-// about 1e-6 N at most, inside the decision margins that matter); otherwise the pair is
-// rescored from g' = g - u_i + u_j, which keeps the cancellation in d-vectors.
-__device__ __forceinline__ bool needs_vector(float terms, float P, float p_i, float p_j, float N)
+// The fast form divides D (a difference of terms of size ~N P^2) by P'^2, so
+// its rounding grows like P^2 / P'^2; it is trusted while P'^2 >= P^2 / 16
+// (error ~1e-6 N, inside the decision margins that matter).  A swap that
+// removes more of the kept mass is rescored from g' = g - u_i + u_j, which keeps
+// the cancellation in d-vectors.
+__device__ __forceinline__ bool needs_vector(float P, float p_i, float p_j)
 {
     const float Pp = P + p_j - p_i;
-    return !(terms <= 4.f * N * Pp * Pp);
+    return !(16.f * Pp * Pp >= P * P);
 }
 
 // Rounding allowances of the lower bound.  alpha_i and beta_j are computed once
 // and shared by the bound and the exact scores, so the bound only has to cover
-// the few operations that combine them (kRoundRel of their magnitude), the
+// the few operations that combine them (kRoundRel, about 16 ulps, of their
+// magnitude), the
 // rounding of the computed cross product C_ij against |w_i||w_j| (d ulps at
 // most) and, where a pair may take the vector form, that form's rounding.
-constexpr float kRoundRel = 2e-6f;
+constexpr float kRoundRel = 1e-6f;
 constexpr float kUlp = 1.2e-7f;
 
 // The score from |g'|^2, g' = g - u_i + u_j summed by the caller.
@@ -227,10 +225,8 @@ __device__ __forceinline__ void score_positions(const int *list, int cnt, const 
                 for (int m = 0; m < 4; ++m) {
                     const int q = q0 + 4 * sub + m;
                     if (q < nadd) {
-                        float terms;
-                        const float sc = pair_score(al, p_i, pj[q], betaj[q], h4[m], P, P2, N, s_i,
-                                                    rj[q], sqN, &terms);
-                        if (needs_vector(terms, P, p_i, pj[q], N)) {
+                        const float sc = pair_score(al, p_i, pj[q], betaj[q], h4[m], P, P2, N);
+                        if (needs_vector(P, p_i, pj[q])) {
                             fl |= 1u << m;
                             continue;
                         }
@@ -626,7 +622,7 @@ __global__ void __launch_bounds__(SWT, 2) k_long_swap(const LSArgs a)
                         const float dlo = P + dmin;
                         const float mag = (fabsf(alpha) + gab[gi] + 2.f * sr) * P2 + N * dabs * (twoP + dabs);
                         float allow = kRoundRel * mag + (float)d * kUlp * 2.f * sr * P2;
-                        if (!(mag <= 4.f * N * dlo * dlo)) {  // some pair may take the vector form
+                        if (!(16.f * dlo * dlo >= P2)) {  // some pair may take the vector form
                             const float tv = sqN + s_i + G.y;
                             allow += kRoundRel * tv * tv * P2;
                         }
