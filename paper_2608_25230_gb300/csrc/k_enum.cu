@@ -70,11 +70,41 @@ struct EnumArgs {
 //   A0 rows (k x RA, RA = EM + k + nHp + 2): raw G'(x, L) | G'(x, A0) | G'(x, H') | a_x | l_x
 //   H' rows (nHp x RH, RH = EM + nHp + 2): folded G'(y, L) | HH (2 x folded off-diagonal,
 //                                          folded diagonal) | l_y - 4 kappa g0n a_y | a_y
+//   inner bound (npref(k) + 1): prefix sums of the ascending G2 entries x < y of L
+//                               (pref[m] = sum of the m smallest), then sum |G2|
 constexpr int OFF_A = 3 * EM + EM * EM;
-__host__ __device__ constexpr int slot_floats(int k, int nHp)
+__host__ __device__ constexpr int cmax_inner(int k) { return k < EM ? k : EM; }
+__host__ __device__ constexpr int npref(int k) { return cmax_inner(k) * (cmax_inner(k) - 1) / 2 + 1; }
+__host__ __device__ constexpr int off_pref(int k, int nHp)
 {
     return OFF_A + k * (EM + k + nHp + 2) + nHp * (EM + nHp + 2);
 }
+__host__ __device__ constexpr int slot_floats(int k, int nHp) { return off_pref(k, nHp) + npref(k) + 1; }
+
+// Ascending sort of 16 registers: Batcher's odd-even merge network (63
+// compare-exchanges, indices fixed at compile time).
+__device__ __forceinline__ void sort16(float (&x)[16])
+{
+#pragma unroll
+    for (int p = 1; p < 16; p <<= 1)
+#pragma unroll
+        for (int kk = p; kk >= 1; kk >>= 1)
+#pragma unroll
+            for (int j = kk % p; j + kk < 16; j += 2 * kk)
+#pragma unroll
+                for (int i = 0; i < kk; ++i) {
+                    if (i + j + kk >= 16) break;
+                    if ((i + j) / (2 * p) == (i + j + kk) / (2 * p)) {
+                        const float a = x[i + j], b = x[i + j + kk];
+                        x[i + j] = fminf(a, b);
+                        x[i + j + kk] = fmaxf(a, b);
+                    }
+                }
+}
+
+// Relative slack of the inner bound: covers the rounding of the bound and of
+// the inner walk's chains (at most 1 + 12 + 66 additions) twice over.
+constexpr float kInnerSlack = 1.52587890625e-5f;  // 2^-16
 
 struct Walk {
     const float *slot;
@@ -176,6 +206,8 @@ __device__ __noinline__ void walk_row(const Walk W)
     const int RA = EM + k + nHp + 2, RH = EM + nHp + 2;
     const float *SA = W.slot + OFF_A;
     const float *SH = SA + k * RA;
+    const float *PF = W.slot + off_pref(k, nHp);  // inner-bound prefix sums, then sum |G2|
+    const float g2abs = PF[npref(k)];
     float Gd[EM], lS[EM], aL[EM], G2[EM][EM];
 #pragma unroll
     for (int x = 0; x < EM; ++x) {
@@ -254,8 +286,31 @@ __device__ __noinline__ void walk_row(const Walk W)
                 float w[EM];
 #pragma unroll
                 for (int j = 0; j < EM; ++j) w[j] = fmaf(2.f, h[j], GdS[j]);
-                const float mval = inner_dispatch(c, w, q, G2);
-                if (mval <= 0.f) collect(W, keep0, imask, w, q, c);
+                // Every size-c set C of L has value q + sum_C w + sum_{pairs of C} G2
+                // >= q + (c smallest w) + (c(c-1)/2 smallest G2): when that bound is
+                // positive beyond rounding, no set of this node can pass the test.
+                bool skip = false;
+                if (c >= 3) {
+                    float ws[16];
+                    float aw = 0.f;
+#pragma unroll
+                    for (int j = 0; j < EM; ++j) {
+                        ws[j] = w[j];
+                        aw += w[j] < INFINITY ? fabsf(w[j]) : 0.f;
+                    }
+#pragma unroll
+                    for (int j = EM; j < 16; ++j) ws[j] = INFINITY;
+                    sort16(ws);
+                    float sw = 0.f;
+#pragma unroll
+                    for (int j = 0; j < EM; ++j) sw += j < c ? ws[j] : 0.f;
+                    const float lb = q + sw + PF[c * (c - 1) / 2];
+                    skip = lb > kInnerSlack * (fabsf(q) + aw + g2abs);
+                }
+                if (!skip) {
+                    const float mval = inner_dispatch(c, w, q, G2);
+                    if (mval <= 0.f) collect(W, keep0, imask, w, q, c);
+                }
             }
             if (!(depth < r && e < nHp && depth < MAXD)) {
                 bool done = true;  // back up to the next sibling
@@ -531,6 +586,44 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
             }
         }
         __syncwarp();
+        // inner bound: the G2 entries x < y of L in ascending order (rank by value,
+        // then position), prefix sums of the smallest npref(k) - 1, and sum |G2|
+        {
+            const float *G2s = S.slot + 3 * EM;
+            float *srt = Ust;  // staging buffer, free again
+            for (int e = lane; e < EM * (EM - 1) / 2; e += 32) {
+                int x = 0, rem = e;
+                while (rem >= EM - 1 - x) {
+                    rem -= EM - 1 - x;
+                    ++x;
+                }
+                const float v = G2s[x * EM + x + 1 + rem];
+                int rk = 0;
+                for (int e2 = 0; e2 < EM * (EM - 1) / 2; ++e2) {
+                    int x2 = 0, r2 = e2;
+                    while (r2 >= EM - 1 - x2) {
+                        r2 -= EM - 1 - x2;
+                        ++x2;
+                    }
+                    const float v2 = G2s[x2 * EM + x2 + 1 + r2];
+                    rk += (v2 < v) || (v2 == v && e2 < e);
+                }
+                srt[rk] = v;
+            }
+            __syncwarp();
+            if (lane == 0) {
+                float *PF = S.slot + off_pref(k, nHp);
+                float acc2 = 0.f, ab = 0.f;
+                PF[0] = 0.f;
+                for (int m = 1; m < npref(k); ++m) {
+                    acc2 += srt[m - 1];
+                    PF[m] = acc2;
+                }
+                for (int e = 0; e < EM * (EM - 1) / 2; ++e) ab += fabsf(srt[e]);
+                PF[npref(k)] = ab;
+            }
+            __syncwarp();
+        }
         if ((lane & (ERW - 1)) == rr && k <= 31) {
             my.slot = S.slot;
             my.perm = perm;

@@ -81,6 +81,7 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
 {
     extern __shared__ uint32_t skeys[];  // [n] order keys when STAGED
     __shared__ uint32_t hist[4][256];
+    __shared__ uint32_t whist[LT / 32][4][256];  // per-warp histograms (32 KB)
     __shared__ float red_m[32], red_s[32];
     __shared__ uint32_t s_prefix[4], s_rem[4];
     __shared__ int s_bad;
@@ -153,7 +154,10 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
         if (a.out.row_status) a.out.row_status[row] = status;
     }
     if (status != FW_OK) return;
-    // radix select of the kb-th largest key, 8 bits at a time from the top
+    // radix select of the kb-th largest key, 8 bits at a time from the top.
+    // Per-warp histograms.  Pass 0 (the top byte, where a row's keys share a
+    // handful of values) has one histogram for every budget and counts each
+    // warp's equal bins once; later passes use shared atomics.
     if (tid < nb) {
         s_prefix[tid] = 0u;
         s_rem[tid] = (uint32_t)a.k[row * nb + tid];
@@ -161,22 +165,38 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
     uint32_t pmask = 0u;
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
-        for (int i = tid; i < 4 * 256; i += LT) (&hist[0][0])[i] = 0u;
+        const int nh = pass == 0 ? 1 : nb;  // histograms this pass
+        for (int i = tid; i < (LT / 32) * 4 * 256; i += LT) (&whist[0][0][0])[i] = 0u;
         __syncthreads();
         uint32_t pre[4];
 #pragma unroll
         for (int b = 0; b < 4; ++b) pre[b] = b < nb ? s_prefix[b] : 0u;
-        for (int j = tid; j < n; j += LT) {
-            const uint32_t key = key_at(j);
+        for (int j0 = 0; j0 < n; j0 += LT) {
+            const int j = j0 + tid;
+            const uint32_t key = j < n ? key_at(j) : 0u;
+            if (pass == 0) {  // top bytes: few distinct values, aggregate them in the warp first
+                const uint32_t bin = j < n ? key >> 24 : 256u + lane;  // lone lanes skip
+                const uint32_t grp = __match_any_sync(FW_FULL, bin);
+                if (j < n && lane == __ffs(grp) - 1) whist[wid][0][bin] += __popc(grp);
+            } else {
 #pragma unroll
-            for (int b = 0; b < 4; ++b)
-                if (b < nb && (key & pmask) == pre[b]) atomicAdd(&hist[b][(key >> shift) & 255u], 1u);
+                for (int b = 0; b < 4; ++b)
+                    if (b < nb && j < n && (key & pmask) == pre[b]) atomicAdd(&whist[wid][b][(key >> shift) & 255u], 1u);
+            }
+        }
+        __syncthreads();
+        // merge the warps' histograms (bins split over the threads)
+        for (int e = tid; e < nh * 256; e += LT) {
+            uint32_t c = 0;
+            for (int w = 0; w < LT / 32; ++w) c += whist[w][e >> 8][e & 255];
+            hist[e >> 8][e & 255] = c;
         }
         __syncthreads();
         if (tid < nb) {
+            const int hb = pass == 0 ? 0 : tid;
             uint32_t cum = 0, rem = s_rem[tid];
             for (int v = 255; v >= 0; --v) {
-                const uint32_t c = hist[tid][v];
+                const uint32_t c = hist[hb][v];
                 if (cum + c >= rem) {
                     s_prefix[tid] |= (uint32_t)v << shift;
                     s_rem[tid] = rem - cum;

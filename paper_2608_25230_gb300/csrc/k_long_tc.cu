@@ -15,8 +15,9 @@
 // tcgen05.mma and tcgen05.commit frees each stage.  The tensor core rounds its
 // fp32 accumulation toward zero, which over thousands of additions into one
 // accumulator biases the sums by ~1e-3; so every stage accumulates into a fresh
-// TMEM buffer (two, alternating) and the producers add it into fp32 registers
-// with round-to-nearest once the stage's MMAs complete.  The epilogue combines
+// TMEM buffer (three in rotation) and the producers add it into fp32 registers
+// with round-to-nearest two stages later, when its MMAs have long completed,
+// so that no producer ever waits on the MMAs it has just enabled.  The epilogue combines
 // the bands exactly as the CUDA-core kernel does:
 //   N_A = sum of the bands inside A, N_{A^c} = the rest,
 //   p(A) (m_A - mu) = pbar(A) N_A - p(A) N_{A^c}.
@@ -35,8 +36,9 @@ constexpr int NT = (PW + 1) * 32;
 constexpr int NPROD = PW * 32;
 constexpr int NSPLIT = 3;     // bf16 terms per probability
 constexpr int ASLOTS = 2;     // A tiles in flight
-constexpr int BSLOTS = 3;     // V / logit tiles in flight (prefetch distance 2)
-constexpr int MAXRT = 64;     // rows per tile for two bands
+constexpr int BSLOTS = 4;     // V / logit tiles in flight (prefetch distance 2)
+constexpr int NACC = 3;       // stage accumulators in TMEM (added two stages late)
+constexpr int MAXRT = 32;     // rows per tile
 constexpr uint32_t WAIT_POLLS = 1u << 20;  // polls before a wait gives up (well over a second)
 constexpr int A_SPLIT_BYTES = TM * 128;            // 16 KB
 constexpr int A_SLOT_BYTES = NSPLIT * A_SPLIT_BYTES;  // 48 KB
@@ -71,6 +73,7 @@ template <int D>
 __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
 {
     constexpr int B_SLOT_BYTES = D * 128;  // KS keys x D bf16
+    constexpr uint32_t TCOLS = NACC * D <= 256 ? 256u : 512u;  // TMEM columns (a power of two)
     constexpr int NC = D / 8;              // 16-byte chunks per V row
     extern __shared__ uint8_t smraw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~(uintptr_t)1023);
@@ -78,7 +81,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
     uint8_t *sB = sA + ASLOTS * A_SLOT_BYTES;          // [BSLOTS][D/64][KS x 128 B]
     float *sL = reinterpret_cast<float *>(sB + BSLOTS * B_SLOT_BYTES);  // [BSLOTS][RT][KS] raw logits
     float *acc = reinterpret_cast<float *>(sA);       // epilogue: [TM][D + 1]
-    __shared__ __align__(8) uint64_t full[BSLOTS], empty[BSLOTS], accfree[2];
+    __shared__ __align__(8) uint64_t full[BSLOTS], empty[BSLOTS], accfree[NACC];
     __shared__ uint32_t s_taddr;
     __shared__ int s_err;
     __shared__ float rowM[MAXRT], rowZi[MAXRT];
@@ -118,7 +121,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
             tc::mbar_init(&full[s], NPROD);
             tc::mbar_init(&empty[s], 1);
         }
-        for (int x = 0; x < 2; ++x) tc::mbar_init(&accfree[x], NPROD);
+        for (int x = 0; x < NACC; ++x) tc::mbar_init(&accfree[x], NPROD);
         tc::mbar_init_fence();
     }
     // rows of A past nbb * RT stay zero in every slot
@@ -127,7 +130,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
         if (m >= nbb * RT) reinterpret_cast<uint4 *>(sA)[e] = make_uint4(0u, 0u, 0u, 0u);
     }
     tc::fence_async_smem();
-    if (wid == PW) tc::tmem_alloc(&s_taddr, 2 * D);  // two stage accumulators
+    if (wid == PW) tc::tmem_alloc(&s_taddr, TCOLS);  // NACC stage accumulators
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
@@ -142,11 +145,12 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
             for (int it = 0; it < nst && ok; ++it) {
                 const int bs = it % BSLOTS, as = it % ASLOTS;
                 ok = tc::mbar_wait(&full[bs], (uint32_t)(it / BSLOTS) & 1u, WAIT_POLLS);
-                // accumulator it % 2 was last read by the producers after stage it - 2
-                if (ok && it >= 2) ok = tc::mbar_wait(&accfree[it & 1], (uint32_t)((it - 2) >> 1) & 1u, WAIT_POLLS);
+                // accumulator it % NACC was last read by the producers after stage it - NACC
+                if (ok && it >= NACC)
+                    ok = tc::mbar_wait(&accfree[it % NACC], (uint32_t)((it - NACC) / NACC) & 1u, WAIT_POLLS);
                 if (!ok) break;
                 tc::fence_after_sync();
-                const uint32_t dacc = taddr + (uint32_t)((it & 1) * D);
+                const uint32_t dacc = taddr + (uint32_t)((it % NACC) * D);
 #pragma unroll
                 for (int ks = 0; ks < KS / 16; ++ks) {
                     const uint64_t bd = tc::sdesc_sw128(b0 + bs * B_SLOT_BYTES + ks * 2048, KS * 128, 1024);
@@ -182,7 +186,8 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
         auto flush = [&](int st) {  // add the accumulator of stage st once its MMAs completed
             if (ok) ok = tc::mbar_wait(&empty[st % BSLOTS], (uint32_t)(st / BSLOTS) & 1u, WAIT_POLLS);
             tc::fence_after_sync();
-            const uint32_t base = taddr + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((st & 1) * D + half * (D / 2));
+            const uint32_t base =
+                taddr + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((st % NACC) * D + half * (D / 2));
 #pragma unroll
             for (int c0 = 0; c0 < D / 2; c0 += 32) {
                 float v[32];
@@ -191,7 +196,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
                 for (int i = 0; i < 32; ++i) racc[c0 + i] += v[i];
             }
             tc::fence_before_sync();
-            tc::mbar_arrive(&accfree[st & 1]);
+            tc::mbar_arrive(&accfree[st % NACC]);
         };
         auto issue = [&](int st) {  // cp.async of stage st's V tile and this thread's logits
             if (st < nst) {
@@ -222,18 +227,14 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
         issue(1);
         for (int it = 0; it < nst; ++it) {
             const int bs = it % BSLOTS, as = it % ASLOTS;
-            // the V / logit slot of stage it + 2 was last read by the MMAs of stage it - 1
-            if (ok && it >= 1 && it + 2 < nst) {
-                const int pst = it - 1;
+            // the V / logit slot of stage it + 2 and the A slot of stage it were
+            // last read by the MMAs of stage it - 2
+            if (ok && it >= 2) {
+                const int pst = it - 2;
                 ok = tc::mbar_wait(&empty[pst % BSLOTS], (uint32_t)(pst / BSLOTS) & 1u, WAIT_POLLS);
             }
             issue(it + 2);
             cp_async_wait2();  // this thread's copies of stage it are in shared memory
-            // the A slot of stage it was last read by the MMAs of stage it - 2
-            if (ok && it >= ASLOTS) {
-                const int pst = it - ASLOTS;
-                ok = tc::mbar_wait(&empty[pst % BSLOTS], (uint32_t)(pst / BSLOTS) & 1u, WAIT_POLLS);
-            }
             uint8_t *aslot = sA + as * A_SLOT_BYTES;
             const int j0 = it * KS;
             for (int q = 0, r = rr0; r < RT; ++q, r += 32) {
@@ -281,9 +282,9 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
             }
             tc::fence_async_smem();
             tc::mbar_arrive(&full[bs]);
-            if (it >= 1) flush(it - 1);
+            if (it >= 2) flush(it - 2);
         }
-        flush(nst - 1);
+        for (int st = nst - 2 < 0 ? 0 : nst - 2; st < nst; ++st) flush(st);
         // band masses: the 8 threads of a row sit in consecutive lanes
 #pragma unroll
         for (int q = 0; q < 2; ++q)
@@ -310,7 +311,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
     __syncthreads();
     if (wid == PW) {
         tc::fence_after_sync();
-        tc::tmem_dealloc(taddr, 2 * D);
+        tc::tmem_dealloc(taddr, TCOLS);
         return;
     }
     // --------------------------------------------------------------- epilogue
@@ -399,7 +400,7 @@ fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_ou
     a.nb = nb;
     a.out = out;
     a.ws = L;
-    a.RT = TM / (nb + 1);
+    a.RT = TM / (nb + 1) < MAXRT ? TM / (nb + 1) : MAXRT;
     a.tiles_per_group = (R.R + a.RT - 1) / a.RT;
     const unsigned grid = (unsigned)(R.num_groups * a.tiles_per_group);
     if (R.d == 128) {
