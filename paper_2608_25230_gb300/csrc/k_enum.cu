@@ -72,14 +72,18 @@ struct EnumArgs {
 //                                          folded diagonal) | l_y - 4 kappa g0n a_y | a_y
 //   inner bound (npref(k) + 1): prefix sums of the ascending G2 entries x < y of L
 //                               (pref[m] = sum of the m smallest), then sum |G2|
+//   root bound (nprefr(k) + 1): the same over every pair of keys that can be
+//                               added back (L and H'), then the sum of their |pair terms|
 constexpr int OFF_A = 3 * EM + EM * EM;
 __host__ __device__ constexpr int cmax_inner(int k) { return k < EM ? k : EM; }
 __host__ __device__ constexpr int npref(int k) { return cmax_inner(k) * (cmax_inner(k) - 1) / 2 + 1; }
+__host__ __device__ constexpr int nprefr(int k) { return k * (k - 1) / 2 + 1; }
 __host__ __device__ constexpr int off_pref(int k, int nHp)
 {
     return OFF_A + k * (EM + k + nHp + 2) + nHp * (EM + nHp + 2);
 }
-__host__ __device__ constexpr int slot_floats(int k, int nHp) { return off_pref(k, nHp) + npref(k) + 1; }
+__host__ __device__ constexpr int off_prefr(int k, int nHp) { return off_pref(k, nHp) + npref(k) + 1; }
+__host__ __device__ constexpr int slot_floats(int k, int nHp) { return off_prefr(k, nHp) + nprefr(k) + 1; }
 
 // Ascending sort of 16 registers: Batcher's odd-even merge network (63
 // compare-exchanges, indices fixed at compile time).
@@ -105,6 +109,11 @@ __device__ __forceinline__ void sort16(float (&x)[16])
 // Relative slack of the inner bound: covers the rounding of the bound and of
 // the inner walk's chains (at most 1 + 12 + 66 additions) twice over.
 constexpr float kInnerSlack = 1.52587890625e-5f;  // 2^-16
+
+// Relative slack of the bound over every set that adds back r keys: twice the
+// longest chain such a set's value goes through (q, r linear terms, r(r-1)/2
+// pair terms and the walk's own adds), in units of 2^-24.
+__device__ __forceinline__ float root_slack(int r) { return (float)(2 * (r * (r + 1) / 2 + r + 32)) * 5.9604645e-8f; }
 
 struct Walk {
     const float *slot;
@@ -208,6 +217,8 @@ __device__ __noinline__ void walk_row(const Walk W)
     const float *SH = SA + k * RA;
     const float *PF = W.slot + off_pref(k, nHp);  // inner-bound prefix sums, then sum |G2|
     const float g2abs = PF[npref(k)];
+    const float *PR = W.slot + off_prefr(k, nHp);  // root-bound prefix sums, then sum |pair terms|
+    const float pabs = PR[nprefr(k)];
     float Gd[EM], lS[EM], aL[EM], G2[EM][EM];
 #pragma unroll
     for (int x = 0; x < EM; ++x) {
@@ -277,6 +288,44 @@ __device__ __noinline__ void walk_row(const Walk W)
         float GdS[EM];
 #pragma unroll
         for (int j = 0; j < EM; ++j) GdS[j] = sform ? Gd[j] + lS[j] : Gd[j];
+        // Every set that adds back r keys from L and H' has value q + (its r
+        // linear terms) + (its r(r-1)/2 pair terms).  The m-th smallest linear
+        // term of L u H' is at least min(m-th smallest over L, least over H'),
+        // and the pair terms are at least the smallest ones of the row; when
+        // that bound is positive beyond rounding, no subset of this R passes.
+        bool skip_r = false;
+        if (r >= 2) {
+            float ws[16];
+            float aw = 0.f;
+#pragma unroll
+            for (int j = 0; j < EM; ++j) {
+                ws[j] = fmaf(2.f, h[j], GdS[j]);
+                aw += ws[j] < INFINITY ? fabsf(ws[j]) : 0.f;
+            }
+#pragma unroll
+            for (int j = EM; j < 16; ++j) ws[j] = INFINITY;
+            sort16(ws);
+            float hmin = INFINITY;
+            for (int y = 0; y < nHp; ++y) {
+                const float *hr = SH + y * RH;
+                float lin = hr[EM + y] + 2.f * base[y];
+                if (sform) lin += hr[RH - 2];
+                hmin = fminf(hmin, lin);
+                aw += fabsf(lin);
+            }
+            float sl = 0.f;
+#pragma unroll
+            for (int m = 0; m < 16; ++m) sl += m < r ? fminf(ws[m], hmin) : 0.f;
+            for (int m = 16; m < r; ++m) sl += hmin;
+            const float lb = q + sl + PR[r * (r - 1) / 2];
+            skip_r = lb > root_slack(r) * (fabsf(q) + aw + pabs);
+        }
+        if (skip_r) {
+            R = next_same_size(R);
+            if (R < nR) R = next_same_size(R);
+            valid = R < nR;
+            continue;
+        }
         // phase 2: depth-first over I subset of H' with |I| <= r
         int depth = 0, e = 0;
         uint32_t imask = 0u;  // local H' bits
@@ -621,6 +670,63 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
                 }
                 for (int e = 0; e < EM * (EM - 1) / 2; ++e) ab += fabsf(srt[e]);
                 PF[npref(k)] = ab;
+            }
+            __syncwarp();
+        }
+        // root bound: the pair terms of every two keys that can be added back
+        // (L x L from G2, H' x H' from HH, H' x L as twice the folded G'(y, L)),
+        // ascending, prefix sums of the smallest nprefr(k) - 1, and sum |terms|
+        {
+            const int nLL = EM * (EM - 1) / 2, nHH = nHp * (nHp - 1) / 2, E = nLL + nHH + EM * nHp;
+            float *vals = Ust, *srt = Ust + E;
+            float *PR = S.slot + off_prefr(k, nHp);
+            if (2 * E <= ust_floats) {
+                for (int e = lane; e < E; e += 32) {
+                    float v;
+                    if (e < nLL) {
+                        int x = 0, rem = e;
+                        while (rem >= EM - 1 - x) {
+                            rem -= EM - 1 - x;
+                            ++x;
+                        }
+                        v = S.slot[3 * EM + x * EM + x + 1 + rem];
+                    } else if (e < nLL + nHH) {
+                        int x = 0, rem = e - nLL;
+                        while (rem >= nHp - 1 - x) {
+                            rem -= nHp - 1 - x;
+                            ++x;
+                        }
+                        v = S.slot[S.offH + x * S.RH + EM + x + 1 + rem];
+                    } else {
+                        const int f = e - nLL - nHH, y = f / EM, j = f - y * EM;
+                        v = 2.f * S.slot[S.offH + y * S.RH + j];
+                    }
+                    vals[e] = v;
+                }
+                __syncwarp();
+                for (int e = lane; e < E; e += 32) {
+                    const float v = vals[e];
+                    int rk = 0;
+                    for (int e2 = 0; e2 < E; ++e2) {
+                        const float v2 = vals[e2];
+                        rk += (v2 < v) || (v2 == v && e2 < e);
+                    }
+                    srt[rk] = v;
+                }
+                __syncwarp();
+                if (lane == 0) {
+                    float acc2 = 0.f, ab = 0.f;
+                    PR[0] = 0.f;
+                    for (int m = 1; m < nprefr(k); ++m) {
+                        acc2 += m - 1 < E ? srt[m - 1] : 0.f;
+                        PR[m] = acc2;
+                    }
+                    for (int e = 0; e < E; ++e) ab += fabsf(srt[e]);
+                    PR[nprefr(k)] = ab;
+                }
+            } else if (lane == 0) {  // (cannot happen for n <= 32; the bound then never prunes)
+                for (int m = 0; m < nprefr(k); ++m) PR[m] = -INFINITY;
+                PR[nprefr(k)] = 0.f;
             }
             __syncwarp();
         }

@@ -170,7 +170,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
         // ------------------------------------------------------------ producers
         const int ptid = tid;                 // 0..NPROD-1
         const int kc = ptid & 7;              // 8-key chunk of the stage
-        const int rr0 = ptid >> 3;            // first row handled (rows rr0, rr0 + 32)
+        const int rr0 = ptid >> 3;            // the row handled (tiles have at most 32 rows)
         float bm[2][5];
 #pragma unroll
         for (int q = 0; q < 2; ++q)
@@ -223,6 +223,22 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
             }
             cp_async_commit();
         };
+        // this thread's row: thresholds, softmax statistics and the band rows of its chunk
+        const bool live = rr0 < nr && rok[rr0];
+        const float Mr = live ? rowM[rr0] : 0.f, Zr = live ? rowZi[rr0] : 0.f;
+        uint32_t mtk[4];
+        int mti[4];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            mtk[b] = live ? rtk[rr0][b] : 0u;
+            mti[b] = live ? rti[rr0][b] : -1;
+        }
+        uint32_t boff[5];
+#pragma unroll
+        for (int b = 0; b < 5; ++b) {
+            const int m = b * RT + rr0;
+            boff[b] = (uint32_t)((m >> 3) * 1024 + (m & 7) * 128 + ((kc ^ (m & 7)) << 4));
+        }
         issue(0);
         issue(1);
         for (int it = 0; it < nst; ++it) {
@@ -237,47 +253,38 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
             cp_async_wait2();  // this thread's copies of stage it are in shared memory
             uint8_t *aslot = sA + as * A_SLOT_BYTES;
             const int j0 = it * KS;
-            for (int q = 0, r = rr0; r < RT; ++q, r += 32) {
-                const float *lr = sL + (bs * RT + r) * KS + kc * 8;
-                const bool live = r < nr && rok[r];
-                const float Mr = live ? rowM[r] : 0.f, Zr = live ? rowZi[r] : 0.f;
-                uint32_t h16[8], m16[8], l16[8];
-                int band[8];
+            if (rr0 < RT) {  // (threads past the tile's rows have no band rows)
+                const float *lr = sL + (bs * RT + rr0) * KS + kc * 8;
+                // zero this thread's chunk of every band row, then put each key's three
+                // bf16 terms into the row of its own band (same thread: ordered)
+#pragma unroll
+                for (int b = 0; b < 5; ++b)
+                    if (b < nbb)
+#pragma unroll
+                        for (int sp = 0; sp < NSPLIT; ++sp)
+                            *reinterpret_cast<uint4 *>(aslot + sp * A_SPLIT_BYTES + boff[b]) = make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
                     const int j = j0 + kc * 8 + u;
-                    float p = 0.f;
+                    if (!(live && j < n)) continue;
+                    const float x = lr[u];
+                    const float p = expf(x - Mr) * Zr;
+                    const uint32_t key = order_key(x);
                     int bd = 0;
-                    if (live && j < n) {
-                        const float x = lr[u];
-                        p = expf(x - Mr) * Zr;
-                        const uint32_t key = order_key(x);
-                        for (int b = 0; b < nb; ++b)
-                            bd += !(key > rtk[r][b] || (key == rtk[r][b] && j <= rti[r][b]));
-                    }
-                    band[u] = bd;
 #pragma unroll
-                    for (int b = 0; b < 5; ++b) bm[q & 1][b] += bd == b ? p : 0.f;
-                    h16[u] = bf16_bits_rn(p);
-                    const float r1 = p - __uint_as_float(h16[u] << 16);
-                    m16[u] = bf16_bits_rn(r1);
-                    l16[u] = bf16_bits_rn(r1 - __uint_as_float(m16[u] << 16));
-                }
-                for (int b = 0; b < nbb; ++b) {
-                    const int m = b * RT + r;
-                    const uint32_t off = (m >> 3) * 1024 + (m & 7) * 128 + ((kc ^ (m & 7)) << 4);
-                    uint32_t w[NSPLIT][4];
+                    for (int b = 0; b < 4; ++b)
+                        if (b < nb) bd += !(key > mtk[b] || (key == mtk[b] && j <= mti[b]));
 #pragma unroll
-                    for (int h = 0; h < 4; ++h) {
-                        const bool e0 = band[2 * h] == b, e1 = band[2 * h + 1] == b;
-                        w[0][h] = (e0 ? h16[2 * h] : 0u) | ((e1 ? h16[2 * h + 1] : 0u) << 16);
-                        w[1][h] = (e0 ? m16[2 * h] : 0u) | ((e1 ? m16[2 * h + 1] : 0u) << 16);
-                        w[2][h] = (e0 ? l16[2 * h] : 0u) | ((e1 ? l16[2 * h + 1] : 0u) << 16);
-                    }
-#pragma unroll
-                    for (int sp = 0; sp < NSPLIT; ++sp)
-                        *reinterpret_cast<uint4 *>(aslot + sp * A_SPLIT_BYTES + off) =
-                            make_uint4(w[sp][0], w[sp][1], w[sp][2], w[sp][3]);
+                    for (int b = 0; b < 5; ++b) bm[0][b] += bd == b ? p : 0.f;
+                    const uint32_t h16 = bf16_bits_rn(p);
+                    const float r1 = p - __uint_as_float(h16 << 16);
+                    const uint32_t m16 = bf16_bits_rn(r1);
+                    const uint32_t l16 = bf16_bits_rn(r1 - __uint_as_float(m16 << 16));
+                    const uint32_t off = (bd == 0 ? boff[0] : bd == 1 ? boff[1] : bd == 2 ? boff[2]
+                                          : bd == 3 ? boff[3] : boff[4]) + 2u * u;
+                    *reinterpret_cast<uint16_t *>(aslot + off) = (uint16_t)h16;
+                    *reinterpret_cast<uint16_t *>(aslot + A_SPLIT_BYTES + off) = (uint16_t)m16;
+                    *reinterpret_cast<uint16_t *>(aslot + 2 * A_SPLIT_BYTES + off) = (uint16_t)l16;
                 }
             }
             tc::fence_async_smem();
@@ -296,9 +303,8 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
                 v += __shfl_xor_sync(FW_FULL, v, 4);
                 bm[q][b] = v;
             }
-        for (int q = 0, r = rr0; r < RT; ++q, r += 32)
-            if (kc == 0)
-                for (int b = 0; b < 5; ++b) bmass[r][b] = bm[q & 1][b];
+        if (kc == 0 && rr0 < RT)
+            for (int b = 0; b < 5; ++b) bmass[rr0][b] = bm[0][b];
         // accumulators -> shared for the per-row epilogue (the stage buffers are idle now)
         if (!ok) atomicOr(&s_err, 1);
         {

@@ -72,6 +72,21 @@ def test_long_ties_and_groups(fw):
     compare(fw, rows_batch(L, V, k, v_dtype="bf16", R=R))
 
 
+@pytest.mark.parametrize("nb,d", [(1, 64), (2, 128), (3, 64), (4, 128)])
+def test_long_bf16_band_counts(fw, nb, d):
+    # bf16 values take the tensor-core P.V; nb + 1 bands per row set the tile
+    # height (32 rows, or 25 for five bands) and 70 rows per group leave a
+    # partial tile; n = 1000 leaves a partial 64-key stage
+    rng = np.random.default_rng(10 * nb + d)
+    R, G, n = 70, 2, 1000
+    L = (rng.normal(size=(G * R, n)) * rng.uniform(0.5, 3.0, size=(G * R, 1))).astype(np.float32)
+    L[:, 0] += 5.0
+    V = rng.normal(size=(G, n, d)).astype(np.float32)
+    ks = [7, 100, 333, 999][:nb]
+    k = np.tile(np.array(ks, np.int32), (G * R, 1))
+    compare(fw, rows_batch(L, V, k, v_dtype="bf16", R=R))
+
+
 def test_mixed_profiles_reduced(fw):
     for b in workloads.mixed_profiles(seed=0, rows_scale=2e-3):
         compare(fw, b)
