@@ -616,16 +616,18 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
                 aX[px_[i]] = sqrtf(fmaxf(acc[i], 0.f)) * 1.0001f + (float)(sqt * pscr[px_[i]]) * 1.0001f;
         __syncwarp();
         // scatter the folded entries into the walk tables
+        const float tf = (float)t, P0f = (float)P0;
 #pragma unroll
         for (int i = 0; i < PPL; ++i) {
             const int x = px_[i], y = py_[i];
             if (x < 0 || x == n) continue;
-            const double pxd = pscr[x];
+            // G' = u.u - t p p^T in fp32 (a few ulps of a_x a_y, inside kappa's slack)
+            const float tpx = tf * (float)pscr[x];
             if (y == n) {
-                const double sx = ((A0 >> x) & 1u) ? -1.0 : 1.0;
-                put_linear(S, inv[x], (float)(2.0 * sx * ((double)acc[i] - t * P0 * pxd)), aX[x]);
+                const float sx = ((A0 >> x) & 1u) ? -2.f : 2.f;
+                put_linear(S, inv[x], sx * fmaf(-tpx, P0f, acc[i]), aX[x]);
             } else {
-                const float gp = (float)((double)acc[i] - t * pxd * pscr[y]);
+                const float gp = fmaf(-tpx, (float)pscr[y], acc[i]);
                 if (x == y) {
                     put_diag(S, inv[x], gp, aX[x]);
                 } else {
@@ -635,51 +637,16 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
             }
         }
         __syncwarp();
-        // inner bound: the G2 entries x < y of L in ascending order (rank by value,
-        // then position), prefix sums of the smallest npref(k) - 1, and sum |G2|
-        {
-            const float *G2s = S.slot + 3 * EM;
-            float *srt = Ust;  // staging buffer, free again
-            for (int e = lane; e < EM * (EM - 1) / 2; e += 32) {
-                int x = 0, rem = e;
-                while (rem >= EM - 1 - x) {
-                    rem -= EM - 1 - x;
-                    ++x;
-                }
-                const float v = G2s[x * EM + x + 1 + rem];
-                int rk = 0;
-                for (int e2 = 0; e2 < EM * (EM - 1) / 2; ++e2) {
-                    int x2 = 0, r2 = e2;
-                    while (r2 >= EM - 1 - x2) {
-                        r2 -= EM - 1 - x2;
-                        ++x2;
-                    }
-                    const float v2 = G2s[x2 * EM + x2 + 1 + r2];
-                    rk += (v2 < v) || (v2 == v && e2 < e);
-                }
-                srt[rk] = v;
-            }
-            __syncwarp();
-            if (lane == 0) {
-                float *PF = S.slot + off_pref(k, nHp);
-                float acc2 = 0.f, ab = 0.f;
-                PF[0] = 0.f;
-                for (int m = 1; m < npref(k); ++m) {
-                    acc2 += srt[m - 1];
-                    PF[m] = acc2;
-                }
-                for (int e = 0; e < EM * (EM - 1) / 2; ++e) ab += fabsf(srt[e]);
-                PF[npref(k)] = ab;
-            }
-            __syncwarp();
-        }
-        // root bound: the pair terms of every two keys that can be added back
-        // (L x L from G2, H' x H' from HH, H' x L as twice the folded G'(y, L)),
-        // ascending, prefix sums of the smallest nprefr(k) - 1, and sum |terms|
+        // Bounds of the walk: the pair terms of the inner set L (G2, x < y) and of
+        // every two keys that can be added back (L x L, H' x H' from HH, H' x L as
+        // twice the folded G'(y, L)); for each list the prefix sums of its
+        // smallest terms (pref[m] = sum of the m smallest) and the sum of |terms|.
+        // Ranks by (value, position); an entry stops counting once it is past the
+        // prefix that is needed.
         {
             const int nLL = EM * (EM - 1) / 2, nHH = nHp * (nHp - 1) / 2, E = nLL + nHH + EM * nHp;
             float *vals = Ust, *srt = Ust + E;
-            float *PR = S.slot + off_prefr(k, nHp);
+            float *PF = S.slot + off_pref(k, nHp), *PR = S.slot + off_prefr(k, nHp);
             if (2 * E <= ust_floats) {
                 for (int e = lane; e < E; e += 32) {
                     float v;
@@ -704,27 +671,36 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
                     vals[e] = v;
                 }
                 __syncwarp();
-                for (int e = lane; e < E; e += 32) {
-                    const float v = vals[e];
-                    int rk = 0;
-                    for (int e2 = 0; e2 < E; ++e2) {
-                        const float v2 = vals[e2];
-                        rk += (v2 < v) || (v2 == v && e2 < e);
+                // pass 0: the first nLL entries (L x L) for the inner bound; pass 1: all E
+                for (int pass = 0; pass < 2; ++pass) {
+                    const int En = pass == 0 ? nLL : E;
+                    const int need = (pass == 0 ? npref(k) : nprefr(k)) - 1;
+                    for (int e = lane; e < En; e += 32) {
+                        const float v = vals[e];
+                        int rk = 0;
+                        for (int e2 = 0; e2 < En && rk < need; ++e2) {
+                            const float v2 = vals[e2];
+                            rk += (v2 < v) || (v2 == v && e2 < e);
+                        }
+                        if (rk < need) srt[rk] = v;
                     }
-                    srt[rk] = v;
-                }
-                __syncwarp();
-                if (lane == 0) {
-                    float acc2 = 0.f, ab = 0.f;
-                    PR[0] = 0.f;
-                    for (int m = 1; m < nprefr(k); ++m) {
-                        acc2 += m - 1 < E ? srt[m - 1] : 0.f;
-                        PR[m] = acc2;
+                    __syncwarp();
+                    if (lane == 0) {
+                        float *P = pass == 0 ? PF : PR;
+                        float acc2 = 0.f, ab = 0.f;
+                        P[0] = 0.f;
+                        for (int m = 1; m <= need; ++m) {
+                            acc2 += m - 1 < En ? srt[m - 1] : 0.f;
+                            P[m] = acc2;
+                        }
+                        for (int e = 0; e < En; ++e) ab += fabsf(vals[e]);
+                        P[need + 1] = ab;
                     }
-                    for (int e = 0; e < E; ++e) ab += fabsf(srt[e]);
-                    PR[nprefr(k)] = ab;
+                    __syncwarp();
                 }
-            } else if (lane == 0) {  // (cannot happen for n <= 32; the bound then never prunes)
+            } else if (lane == 0) {  // (cannot happen for n <= 32; the bounds then never prune)
+                for (int m = 0; m < npref(k); ++m) PF[m] = -INFINITY;
+                PF[npref(k)] = 0.f;
                 for (int m = 0; m < nprefr(k); ++m) PR[m] = -INFINITY;
                 PR[nprefr(k)] = 0.f;
             }
