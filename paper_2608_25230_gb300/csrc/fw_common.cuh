@@ -173,6 +173,27 @@ __device__ __forceinline__ uint64_t colex_rank_mask(uint32_t m)
     return r;
 }
 
+// Columns [c0, c0 + DC) of the n value rows into st[j][DC + 1], fp32; the warp
+// issues all its loads before it stores any (8 elements per lane per step).
+template <int DC, typename VT>
+__device__ __forceinline__ void stage_value_cols(const VT *V, int n, int d, int c0, float *st, int lane)
+{
+    const int tot = n * DC;
+    for (int e0 = 0; e0 < tot; e0 += 32 * 8) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int e = e0 + lane + 32 * u;
+            v[u] = e < tot ? load_v(V, (int64_t)(e / DC) * d + c0 + e % DC) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int e = e0 + lane + 32 * u;
+            if (e < tot) st[(e / DC) * (DC + 1) + e % DC] = v[u];
+        }
+    }
+}
+
 // Dispatch on the value width d (multiples of 32 supported: 32, 64, 128, 256)
 // and the value dtype; binds DPL (dims per lane) and VT (element type).
 #define FW_DISPATCH(d, vdt, ...)                                                              \

@@ -40,7 +40,6 @@ constexpr int MAXD = 24;  // depth bound of the phase-2 walk
 constexpr int PERM = 48;  // local index space per row: NS <= EM + 32
 
 __host__ __device__ constexpr int tri(int a, int b, int n) { return a * n - a * (a - 1) / 2 + (b - a); }
-__device__ __forceinline__ int tri_s(int a, int b, int n) { return a <= b ? tri(a, b, n) : tri(b, a, n); }
 
 struct EnumArgs {
     RowsDev R;
@@ -449,6 +448,53 @@ __device__ __forceinline__ void put_linear(const SlotGeom &S, int l, float lin, 
     else S.slot[S.offH + (l - eH) * S.RH + S.RH - 2] = lin - 4.f * S.kap * S.g0n * a;
 }
 
+// pref[m] = sum of the m smallest of vals[0, E) for m <= need, then
+// pref[need + 1] = sum |vals| (E <= 512).  Each lane holds its entries
+// lane + 32 u in registers; every round the warp takes the smallest unused one
+// (equal values: any of them, the sums do not depend on it).
+__device__ __forceinline__ void smallest_prefix(const float *vals, int E, int need, float *pref, int lane)
+{
+    float x[16];
+    float ab = 0.f;
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+        const int e = lane + 32 * u;
+        x[u] = e < E ? vals[e] : INFINITY;
+        ab += e < E ? fabsf(x[u]) : 0.f;
+    }
+    ab = warp_sum(ab);
+    float run = 0.f;
+    if (lane == 0) pref[0] = 0.f;
+    for (int m = 0; m < need; ++m) {
+        float bv = INFINITY;
+        int bu = 0;
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+            if (x[u] < bv) {
+                bv = x[u];
+                bu = u;
+            }
+        float wv = bv;
+        int wl = lane;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ov = __shfl_xor_sync(FW_FULL, wv, o);
+            const int ol = __shfl_xor_sync(FW_FULL, wl, o);
+            if (ov < wv || (ov == wv && ol < wl)) {
+                wv = ov;
+                wl = ol;
+            }
+        }
+        if (lane == wl)
+#pragma unroll
+            for (int u = 0; u < 16; ++u)
+                if (u == bu) x[u] = INFINITY;
+        run += wv < INFINITY ? wv : 0.f;
+        if (lane == 0) pref[m + 1] = run;
+    }
+    if (lane == 0) pref[need + 1] = ab;
+}
+
 constexpr int ERW = 16;  // rows per warp (two lanes per row)
 constexpr int PPL = 18;  // Gram pairs per lane: (33 * 34 / 2) / 32 rounded up
 
@@ -511,15 +557,6 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
         const bool inA0 = lane < n && rank < k;
         const uint32_t A0 = __ballot_sync(FW_FULL, inA0);
         const df pd = df_from_double(p);
-        df mu[DPL];
-#pragma unroll
-        for (int t = 0; t < DPL; ++t) mu[t] = df_zero();
-        for (int j = 0; j < n; ++j) {
-            const df pj = shfl_df(pd, j);
-#pragma unroll
-            for (int t = 0; t < DPL; ++t)
-                mu[t] = df_add(mu[t], df_mul_f(pj, load_v(V, (int64_t)j * d + lane + 32 * t)));
-        }
         // local key order: L = first nL keys outside A0, then A0, then H'
         const int nL = min(EM, n - k);
         const int nHp = n - k - nL;
@@ -566,15 +603,29 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
 #pragma unroll
         for (int ch = 0; ch < DPL / TCH; ++ch) {
             __syncwarp();
+            // the chunk's values of all n keys into Ust (loads issued back to back)
+            stage_value_cols<DCH>(V, n, d, ch * DCH, Ust, lane);
+            __syncwarp();
+            // mu over the chunk's columns (j ascending, double-float), then
+            // u_j = p_j (v_j - mu) in place
+            df mu[TCH];
+#pragma unroll
+            for (int tt = 0; tt < TCH; ++tt) mu[tt] = df_zero();
+            for (int j = 0; j < n; ++j) {
+                const df pj = shfl_df(pd, j);
+#pragma unroll
+                for (int tt = 0; tt < TCH; ++tt)
+                    mu[tt] = df_add(mu[tt], df_mul_f(pj, Ust[j * (DCH + 1) + lane + 32 * tt]));
+            }
             for (int j = 0; j < n; ++j) {
                 const df pj = shfl_df(pd, j);
                 const bool in = (A0 >> j) & 1u;
 #pragma unroll
                 for (int tt = 0; tt < TCH; ++tt) {
                     const int t = ch * TCH + tt;
-                    const int c = lane + 32 * t;
-                    const df u = df_mul(pj, df_rsub_f(load_v(V, (int64_t)j * d + c), mu[t]));
-                    Ust[j * (DCH + 1) + lane + 32 * tt] = u.hi;
+                    float *cell = Ust + j * (DCH + 1) + lane + 32 * tt;
+                    const df u = df_mul(pj, df_rsub_f(*cell, mu[tt]));
+                    *cell = u.hi;
                     if (in) g0[t] = df_add(g0[t], u);
                 }
             }
@@ -641,13 +692,12 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
         // every two keys that can be added back (L x L, H' x H' from HH, H' x L as
         // twice the folded G'(y, L)); for each list the prefix sums of its
         // smallest terms (pref[m] = sum of the m smallest) and the sum of |terms|.
-        // Ranks by (value, position); an entry stops counting once it is past the
-        // prefix that is needed.
+        // The warp takes the smallest remaining term round by round.
         {
             const int nLL = EM * (EM - 1) / 2, nHH = nHp * (nHp - 1) / 2, E = nLL + nHH + EM * nHp;
-            float *vals = Ust, *srt = Ust + E;
+            float *vals = Ust;
             float *PF = S.slot + off_pref(k, nHp), *PR = S.slot + off_prefr(k, nHp);
-            if (2 * E <= ust_floats) {
+            if (E <= ust_floats && E <= 512) {
                 for (int e = lane; e < E; e += 32) {
                     float v;
                     if (e < nLL) {
@@ -675,28 +725,7 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
                 for (int pass = 0; pass < 2; ++pass) {
                     const int En = pass == 0 ? nLL : E;
                     const int need = (pass == 0 ? npref(k) : nprefr(k)) - 1;
-                    for (int e = lane; e < En; e += 32) {
-                        const float v = vals[e];
-                        int rk = 0;
-                        for (int e2 = 0; e2 < En && rk < need; ++e2) {
-                            const float v2 = vals[e2];
-                            rk += (v2 < v) || (v2 == v && e2 < e);
-                        }
-                        if (rk < need) srt[rk] = v;
-                    }
-                    __syncwarp();
-                    if (lane == 0) {
-                        float *P = pass == 0 ? PF : PR;
-                        float acc2 = 0.f, ab = 0.f;
-                        P[0] = 0.f;
-                        for (int m = 1; m <= need; ++m) {
-                            acc2 += m - 1 < En ? srt[m - 1] : 0.f;
-                            P[m] = acc2;
-                        }
-                        for (int e = 0; e < En; ++e) ab += fabsf(vals[e]);
-                        P[need + 1] = ab;
-                    }
-                    __syncwarp();
+                    smallest_prefix(vals, En, need, pass == 0 ? PF : PR, lane);
                 }
             } else if (lane == 0) {  // (cannot happen for n <= 32; the bounds then never prune)
                 for (int m = 0; m < npref(k); ++m) PF[m] = -INFINITY;
@@ -759,34 +788,49 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
         double p = lane < n ? exp((double)l - (double)M) : 0.0;
         p = p / warp_sum_d(p);
         const df pd = df_from_double(p);
-        df mu[DPL];
+        // per 64-column chunk: stage the values, mu over the chunk, and each
+        // candidate's g over the chunk, whose squares add into a per-lane partial
+        // (kept in the slots, free after the walk); same order of operations as
+        // one pass over all columns
+        df *cacc = reinterpret_cast<df *>(slots);  // [ECAP][32]
+        for (int ci = 0; ci < cc; ++ci) cacc[ci * 32 + lane] = df_zero();
+        for (int ch = 0; ch < DPL / TCH; ++ch) {
+            __syncwarp();
+            stage_value_cols<DCH>(V, n, d, ch * DCH, Ust, lane);
+            __syncwarp();
+            df mu[TCH];
 #pragma unroll
-        for (int t = 0; t < DPL; ++t) mu[t] = df_zero();
-        for (int j = 0; j < n; ++j) {
-            const df pj = shfl_df(pd, j);
+            for (int tt = 0; tt < TCH; ++tt) mu[tt] = df_zero();
+            for (int j = 0; j < n; ++j) {
+                const df pj = shfl_df(pd, j);
 #pragma unroll
-            for (int t = 0; t < DPL; ++t)
-                mu[t] = df_add(mu[t], df_mul_f(pj, load_v(V, (int64_t)j * d + lane + 32 * t)));
+                for (int tt = 0; tt < TCH; ++tt)
+                    mu[tt] = df_add(mu[tt], df_mul_f(pj, Ust[j * (DCH + 1) + lane + 32 * tt]));
+            }
+            for (int ci = 0; ci < cc; ++ci) {
+                const uint32_t m = a.cand[row * ECAP + ci];
+                df gv[TCH];
+#pragma unroll
+                for (int tt = 0; tt < TCH; ++tt) gv[tt] = df_zero();
+                for (uint32_t mm = m; mm; mm &= mm - 1) {
+                    const int j = __ffs(mm) - 1;
+                    const df pj = shfl_df(pd, j);
+#pragma unroll
+                    for (int tt = 0; tt < TCH; ++tt)
+                        gv[tt] = df_add(gv[tt], df_mul(pj, df_rsub_f(Ust[j * (DCH + 1) + lane + 32 * tt], mu[tt])));
+                }
+                df sq = cacc[ci * 32 + lane];
+#pragma unroll
+                for (int tt = 0; tt < TCH; ++tt) sq = df_add(sq, df_mul(gv[tt], gv[tt]));
+                cacc[ci * 32 + lane] = sq;
+            }
         }
         double best = INFINITY;
         uint64_t brank = ~0ull;
         uint32_t bmask = 0u;
         for (int ci = 0; ci < cc; ++ci) {
             const uint32_t m = a.cand[row * ECAP + ci];
-            df gv[DPL];
-#pragma unroll
-            for (int t = 0; t < DPL; ++t) gv[t] = df_zero();
-            for (uint32_t mm = m; mm; mm &= mm - 1) {
-                const int j = __ffs(mm) - 1;
-                const df pj = shfl_df(pd, j);
-#pragma unroll
-                for (int t = 0; t < DPL; ++t)
-                    gv[t] = df_add(gv[t], df_mul(pj, df_rsub_f(load_v(V, (int64_t)j * d + lane + 32 * t), mu[t])));
-            }
-            df s3 = df_zero();
-#pragma unroll
-            for (int t = 0; t < DPL; ++t) s3 = df_add(s3, df_mul(gv[t], gv[t]));
-            s3 = warp_sum_df(s3);
+            const df s3 = warp_sum_df(cacc[ci * 32 + lane]);
             const double P = warp_sum_d(((m >> lane) & 1u) ? p : 0.0);
             const double e = fmax(df_to_double(s3), 0.0) / (P * P);
             const uint64_t rk = colex_rank_mask(m);

@@ -201,16 +201,18 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
     double p = lane < n ? exp((double)l - (double)M) : 0.0;
     p = p / warp_sum_d(p);
     const df pd = df_from_double(p);
+    // the row's values into Uhi (loads issued back to back), then mu from there
+    stage_value_cols<d>(V, n, d, 0, Uhi, lane);
+    __syncwarp();
     df mu[DPL];
 #pragma unroll
     for (int t = 0; t < DPL; ++t) mu[t] = df_zero();
     for (int j = 0; j < n; ++j) {
         const df pj = shfl_df(pd, j);
 #pragma unroll
-        for (int t = 0; t < DPL; ++t)
-            mu[t] = df_add(mu[t], df_mul_f(pj, load_v(V, (int64_t)j * d + lane + 32 * t)));
+        for (int t = 0; t < DPL; ++t) mu[t] = df_add(mu[t], df_mul_f(pj, Uhi[j * (d + 1) + lane + 32 * t]));
     }
-    // u_j = p_j (v_j - mu) into shared memory, and ||u_j||^2 held by lane j
+    // u_j = p_j (v_j - mu) in place (hi in Uhi, lo in Ulo), ||u_j||^2 held by lane j
     double e2 = 0.0;
     for (int j = 0; j < n; ++j) {
         const df pj = shfl_df(pd, j);
@@ -218,7 +220,7 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
 #pragma unroll
         for (int t = 0; t < DPL; ++t) {
             const int c = lane + 32 * t;
-            const df u = df_mul(pj, df_rsub_f(load_v(V, (int64_t)j * d + c), mu[t]));
+            const df u = df_mul(pj, df_rsub_f(Uhi[j * (d + 1) + c], mu[t]));
             Uhi[j * (d + 1) + c] = u.hi;
             Ulo[j * d + c] = u.lo;
             s = df_add(s, df_mul(u, u));
