@@ -496,7 +496,8 @@ __device__ __forceinline__ void smallest_prefix(const float *vals, int E, int ne
 }
 
 constexpr int ERW = 16;  // rows per warp (two lanes per row)
-constexpr int PPL = 18;  // Gram pairs per lane: (33 * 34 / 2) / 32 rounded up
+constexpr int MAXT = 3;         // Gram tiles (2 x 4 products) per lane: 33 rows need at most 96
+constexpr int PPL = 8 * MAXT;   // Gram product slots per lane
 
 // ---- the fast kernel: one warp = 16 rows; prologue and re-scoring are
 // warp-cooperative per row, the walk gives each row two lanes that split its
@@ -580,22 +581,40 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
         S.offH = OFF_A + k * S.RA;
         const int tot = slot_floats(k, nHp);
         for (int i = lane; i < tot; i += 32) S.slot[i] = (i >= nL && i < EM) ? INFINITY : 0.f;
-        // Gram entries over the n keys plus g0 (index n), staged DCH dimensions at a time;
-        // each dot is four interleaved partial sums per chunk
-        const int npr = (n + 1) * (n + 2) / 2;
+        // Gram entries over the n keys plus g0 (index n), staged DCH dimensions at a
+        // time.  The upper triangle is cut into tiles of 2 rows x 4 columns (lane
+        // takes tiles lane, lane + 32, ...); a tile reads 6 staged values per
+        // dimension for its 8 products, and each product is four interleaved
+        // partial sums per chunk.  Slot i = 8 * tile + 4 * (x - x0) + (y - y0);
+        // px_ = -1 marks slots outside the triangle (and |g0|^2, known exactly).
+        const int R1 = n + 1, nby = (R1 + 3) / 4;
+        int tx0[MAXT], ty0[MAXT];
         int px_[PPL], py_[PPL];
         float acc[PPL];
 #pragma unroll
-        for (int i = 0; i < PPL; ++i) {
-            const int qd = lane + 32 * i;
-            int x = 0, rem = qd < npr ? qd : 0;
-            while (rem >= n + 1 - x) {
-                rem -= n + 1 - x;
-                ++x;
+        for (int tl = 0; tl < MAXT; ++tl) {
+            int tid_ = lane + 32 * tl, bx = 0;
+            bool ok = true;
+            for (;;) {  // rows 2bx, 2bx+1 hold tiles by = bx/2 .. nby-1
+                if (2 * bx >= R1) {
+                    ok = false;
+                    break;
+                }
+                const int cnt = nby - bx / 2;
+                if (tid_ < cnt) break;
+                tid_ -= cnt;
+                ++bx;
             }
-            px_[i] = qd < npr ? x : -1;
-            py_[i] = x + rem;
-            acc[i] = 0.f;
+            tx0[tl] = ok ? 2 * bx : -1;
+            ty0[tl] = ok ? 4 * (bx / 2 + tid_) : -1;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int x = tx0[tl] + (e >> 2), y = ty0[tl] + (e & 3);
+                const bool in = ok && x <= y && y < R1 && x < n;
+                px_[8 * tl + e] = in ? x : -1;
+                py_[8 * tl + e] = y;
+                acc[8 * tl + e] = 0.f;
+            }
         }
         df g0[DPL];
 #pragma unroll
@@ -633,18 +652,32 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
             for (int tt = 0; tt < TCH; ++tt) Ust[n * (DCH + 1) + lane + 32 * tt] = g0[ch * TCH + tt].hi;
             __syncwarp();
 #pragma unroll
-            for (int i = 0; i < PPL; ++i) {
-                if (px_[i] < 0 || px_[i] == n) continue;  // |g0|^2 is known exactly
-                const float *ux = Ust + px_[i] * (DCH + 1), *uy = Ust + py_[i] * (DCH + 1);
-                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll 4
+            for (int tl = 0; tl < MAXT; ++tl) {
+                if (tx0[tl] < 0) continue;
+                const float *ux[2], *uy[4];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) ux[e] = Ust + min(tx0[tl] + e, n) * (DCH + 1);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) uy[e] = Ust + min(ty0[tl] + e, n) * (DCH + 1);
+                float sp[8][4];
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) sp[e][c4] = 0.f;
                 for (int c = 0; c < DCH; c += 4) {
-                    s0 = fmaf(ux[c], uy[c], s0);
-                    s1 = fmaf(ux[c + 1], uy[c + 1], s1);
-                    s2 = fmaf(ux[c + 2], uy[c + 2], s2);
-                    s3 = fmaf(ux[c + 3], uy[c + 3], s3);
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        const float a0 = ux[0][c + c4], a1 = ux[1][c + c4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float b = uy[e][c + c4];
+                            sp[e][c4] = fmaf(a0, b, sp[e][c4]);
+                            sp[4 + e][c4] = fmaf(a1, b, sp[4 + e][c4]);
+                        }
+                    }
                 }
-                acc[i] += (s0 + s1) + (s2 + s3);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[8 * tl + e] += (sp[e][0] + sp[e][1]) + (sp[e][2] + sp[e][3]);
             }
         }
         df nrm = df_zero();
