@@ -5,6 +5,8 @@
 // (one exp per key), vector sums are double-float on the fp32 pipe, so every
 // output carries ~1e-13 relative error against an fp64 evaluation of the
 // definitions.
+#include <algorithm>
+
 #include "fw_internal.h"
 
 namespace fw {
@@ -146,10 +148,12 @@ struct SmallSwapArgs {
     int E, max_swaps;
     int32_t *n_swaps, *swap_out, *swap_in, *capped;
     float *refined_gap, *topk_gap;
+    int nr;  // rows of the per-warp tables
 };
 
-// shared memory per warp (floats): Uhi [32][d+1], Ulo [32][d], G [32][33]
-template <int DPL> __host__ __device__ constexpr int swap_smem_floats() { return 32 * (DPL * 32 + 1) + 32 * DPL * 32 + 32 * 33; }
+// shared memory per warp (floats): U [nr][d+1] (the values, then the high
+// parts of u), G [nr][33]; nr = max_n rounded up to a multiple of 4
+__host__ __device__ constexpr int swap_smem_floats(int nr, int d) { return nr * (d + 1) + nr * 33; }
 
 // The balancing selector (Sec. 2.1) inside the candidate set (Definition 2.2).
 // Pair scores are screened in fp32 from the Gram matrix G = U U^T of the
@@ -164,9 +168,8 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
     constexpr int d = DPL * 32;
     const int lane = threadIdx.x & 31;
     const int wib = threadIdx.x >> 5;
-    float *Uhi = smem + (size_t)wib * swap_smem_floats<DPL>();
-    float *Ulo = Uhi + 32 * (d + 1);
-    float *G = Ulo + 32 * d;
+    float *Uhi = smem + (size_t)wib * swap_smem_floats(a.nr, d);
+    float *G = Uhi + a.nr * (d + 1);
     const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
     if (row >= a.R.rows) return;
     const int64_t g = row / a.R.R;
@@ -212,7 +215,8 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
 #pragma unroll
         for (int t = 0; t < DPL; ++t) mu[t] = df_add(mu[t], df_mul_f(pj, Uhi[j * (d + 1) + lane + 32 * t]));
     }
-    // u_j = p_j (v_j - mu) in place (hi in Uhi, lo in Ulo), ||u_j||^2 held by lane j
+    // u_j = p_j (v_j - mu): high parts in place in Uhi (the exact re-scoring
+    // recomputes the double-float value from V), ||u_j||^2 held by lane j
     double e2 = 0.0;
     for (int j = 0; j < n; ++j) {
         const df pj = shfl_df(pd, j);
@@ -222,7 +226,6 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
             const int c = lane + 32 * t;
             const df u = df_mul(pj, df_rsub_f(Uhi[j * (d + 1) + c], mu[t]));
             Uhi[j * (d + 1) + c] = u.hi;
-            Ulo[j * d + c] = u.lo;
             s = df_add(s, df_mul(u, u));
         }
         s = warp_sum_df(s);
@@ -297,6 +300,10 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
             S = warp_sum(inp && cnt <= kb ? unorm : 0.f) * 1.0001f;
         }
         const float CB = 2.0f * ((float)d * 0.25f + 2.0f * (float)kb + 12.0f) * 5.9604645e-8f;
+        // u_j in double-float, recomputed from V (the expression of the pass above)
+        auto u_df = [&](int j, int t) {
+            return df_mul(shfl_df(pd, j), df_rsub_f(load_v(V, (int64_t)j * d + lane + 32 * t), mu[t]));
+        };
         // exact state: g_A (double-float, lanes over dims), p(A), es^2
         df gA[DPL];
 #pragma unroll
@@ -305,8 +312,7 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
             const int j = __ffs(m) - 1;
 #pragma unroll
             for (int t = 0; t < DPL; ++t) {
-                const int c = lane + 32 * t;
-                gA[t] = df_add(gA[t], df{Uhi[j * (d + 1) + c], Ulo[j * d + c]});
+                gA[t] = df_add(gA[t], u_df(j, t));
             }
         }
         double PA = warp_sum_d(((A >> lane) & 1u) ? p : 0.0);
@@ -371,9 +377,7 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
                     df gn[DPL];
 #pragma unroll
                     for (int t = 0; t < DPL; ++t) {
-                        const int c = lane + 32 * t;
-                        gn[t] = df_add(df_sub(gA[t], df{Uhi[i * (d + 1) + c], Ulo[i * d + c]}),
-                                       df{Uhi[j * (d + 1) + c], Ulo[j * d + c]});
+                        gn[t] = df_add(df_sub(gA[t], u_df(i, t)), u_df(j, t));
                     }
                     const double P2 = PA - __shfl_sync(FW_FULL, p, i) + __shfl_sync(FW_FULL, p, j);
                     const double e = exact_es2(gn, P2);
@@ -391,9 +395,7 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
             }
 #pragma unroll
             for (int t = 0; t < DPL; ++t) {
-                const int c = lane + 32 * t;
-                gA[t] = df_add(df_sub(gA[t], df{Uhi[bi * (d + 1) + c], Ulo[bi * d + c]}),
-                               df{Uhi[bj * (d + 1) + c], Ulo[bj * d + c]});
+                gA[t] = df_add(df_sub(gA[t], u_df(bi, t)), u_df(bj, t));
             }
             PA = PA - __shfl_sync(FW_FULL, p, bi) + __shfl_sync(FW_FULL, p, bj);
             A = (A & ~(1u << bi)) | (1u << bj);
@@ -431,11 +433,12 @@ fw_status small_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_ou
                      float *refined_gap, float *topk_gap, int32_t *capped, cudaStream_t s)
 {
     if (R.rows == 0) return FW_OK;
+    const int nr = (std::min(R.max_n, 32) + 3) / 4 * 4;
     const SmallSwapArgs a{R, k, nb, topk.thr_key, topk.thr_idx, E, max_swaps, n_swaps, swap_out,
-                          swap_in, capped, refined_gap, topk_gap};
+                          swap_in, capped, refined_gap, topk_gap, nr};
     FW_DISPATCH(R.d, R.v_dtype, {
         const int warps = DPL >= 8 ? 1 : 2;
-        const size_t smem = (size_t)warps * swap_smem_floats<DPL>() * sizeof(float);
+        const size_t smem = (size_t)warps * swap_smem_floats(nr, DPL * 32) * sizeof(float);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_small_swap<DPL, VT>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
         const unsigned grid = (unsigned)((R.rows + warps - 1) / warps);
