@@ -152,21 +152,38 @@ __device__ __forceinline__ df shfl_df(df v, int src)
     return {__shfl_sync(FW_FULL, v.hi, src), __shfl_sync(FW_FULL, v.lo, src)};
 }
 
-// colex rank of the set bits of a 32-bit mask: sum_i C(c_i, i), i = 1.. in ascending order
+// Binomial coefficients C(a, b) for a <= 32 (all below 2^32), built by
+// Pascal's rule at compile time; per translation unit in constant memory.
+struct BinomTable {
+    uint32_t v[33][33];
+};
+constexpr BinomTable make_binom_table()
+{
+    BinomTable t{};
+    for (int a = 0; a <= 32; ++a) {
+        t.v[a][0] = 1u;
+        for (int b = 1; b <= a; ++b) t.v[a][b] = t.v[a - 1][b - 1] + (b <= a - 1 ? t.v[a - 1][b] : 0u);
+    }
+    return t;
+}
+static __constant__ BinomTable c_binom = make_binom_table();
+
 __device__ __forceinline__ uint64_t binom64(int a, int b)
 {
     if (b < 0 || b > a) return 0;
+    if (a <= 32) return c_binom.v[a][b];
     uint64_t r = 1;
     for (int t = 1; t <= b; ++t) r = r * (uint64_t)(a - b + t) / (uint64_t)t;
     return r;
 }
+// colex rank of the set bits of a 32-bit mask: sum_i C(c_i, i), i = 1.. in ascending order
 __device__ __forceinline__ uint64_t colex_rank_mask(uint32_t m)
 {
     uint64_t r = 0;
     int i = 1;
     while (m) {
-        int c = __ffs(m) - 1;
-        r += binom64(c, i);
+        const int c = __ffs(m) - 1;
+        r += c_binom.v[c][i];  // c <= 31, i <= 32; C(c, i) = 0 for i > c
         ++i;
         m &= m - 1;
     }

@@ -56,6 +56,9 @@ struct EnumArgs {
     int32_t *fb_count;    // [1]
     double *fb_e;         // [rows][FBS] best es^2 of each chunk of an exhaustive row
     unsigned long long *fb_r;  // [rows][FBS] its colex rank
+    float *slots;         // [rows][stride] walk tables
+    uint8_t *perms;       // [rows][PERM] local key order
+    float2 *kg;           // [rows] kappa, |g0| (rounded up)
     int stride;           // floats per row slot (odd)
 };
 
@@ -499,297 +502,332 @@ constexpr int ERW = 16;  // rows per warp (two lanes per row)
 constexpr int MAXT = 3;         // Gram tiles (2 x 4 products) per lane: 33 rows need at most 96
 constexpr int PPL = 8 * MAXT;   // Gram product slots per lane
 
-// ---- the fast kernel: one warp = 16 rows; prologue and re-scoring are
-// warp-cooperative per row, the walk gives each row two lanes that split its
-// removal sets.
+// ---- the search in three kernels.  k_enum_prep: one warp per row builds the
+// row's walk tables (slot, key order, kappa and |g0|) in shared memory and
+// writes them out; k_enum_walk: one warp = ERW rows, two lanes per row split
+// its removal sets; k_enum_rescore: one warp per row re-scores the row's
+// candidates exactly and lists the rows left to the exhaustive path.
+constexpr int PREP_W = 4;  // warps (rows) per block of k_enum_prep
+constexpr int RS_W = 8;    // warps (rows) per block of k_enum_rescore
+
+// per-warp shared memory of k_enum_prep (floats): slot, staged values, a_x,
+// p (double), key order and its inverse; a multiple of 4
+__host__ __device__ constexpr int prep_floats(int stride, int ust)
+{
+    return ((stride + 1) / 2 * 2 + ust + 32 + 64 + (PERM + 32) / 4 + 3) / 4 * 4;
+}
+constexpr int RCB = 8;     // candidates re-scored per pass over the values
+// per-warp shared memory of k_enum_rescore (floats): the staged values
+__host__ __device__ constexpr int rescore_floats(int ust) { return (ust + 3) / 4 * 4; }
+
 template <int DPL, typename VT>
-__global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
+__global__ void __launch_bounds__(32 * PREP_W, 4) k_enum_prep(const EnumArgs a)
 {
     extern __shared__ float smem[];
     constexpr int d = DPL * 32;
     constexpr int DCH = d < 64 ? d : 64;  // dimensions staged at a time
     constexpr int TCH = DCH / 32;         // per-lane dims in one chunk
-    const int lane = threadIdx.x;
-    float *slots = smem;                                                   // [ERW][stride]
-    float *Ust = smem + ERW * a.stride;                                    // [max_n+1][DCH+1]
+    const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
     const int ust_floats = (((a.R.max_n + 1) * (DCH + 1)) + 1) & ~1;
-    float *aX = Ust + ust_floats;                                          // [32]
-    double *pscr = reinterpret_cast<double *>(aX + 32);                    // [32]
-    uint8_t *perms = reinterpret_cast<uint8_t *>(pscr + 32);               // [ERW][PERM]
-    uint8_t *inv = perms + ERW * PERM;                                     // [32]
-    const int64_t row0 = (int64_t)blockIdx.x * ERW;
-
-    Walk my;
-    bool my_walk = false;
-
-    // ------------------------------------------------------------ prologue
-    for (int rr = 0; rr < ERW; ++rr) {
-        const int64_t row = row0 + rr;
-        if (row >= a.R.rows) break;
-        const int64_t g = row / a.R.R;
-        const int64_t ri = row - g * a.R.R;
-        const int n = a.R.n[g];
-        const int k = a.k[row];
-        int status = FW_OK;
-        if (n < 1 || n > a.R.max_n || n > 32 || k < 1 || k > n || k > a.k_max) status = FW_ERR_INVALID_ARG;
-        const float *lg = a.R.logits + a.R.logit_off[g] + ri * (status == FW_OK ? n : 0);
-        const float l = (status == FW_OK && lane < n) ? lg[lane] : -INFINITY;
-        if (status == FW_OK && __any_sync(FW_FULL, lane < n && !isfinite(l))) status = FW_ERR_NONFINITE;
-        if (status != FW_OK) {
-            if (lane == 0) {
-                if (a.row_status) a.row_status[row] = status;
-                a.cand_count[row] = -1;
-                a.best_gap[row] = __int_as_float(0x7fc00000);
-                a.best_rank[row] = ~0ull;
-                if (a.topk_gap) a.topk_gap[row] = __int_as_float(0x7fc00000);
+    float *slot = smem + (size_t)wib * prep_floats(a.stride, ust_floats);  // [stride]
+    float *Ust = slot + (a.stride + 1) / 2 * 2;                             // [max_n+1][DCH+1]
+    float *aX = Ust + ust_floats;                                            // [32]
+    double *pscr = reinterpret_cast<double *>(aX + 32);                      // [32]
+    uint8_t *perms = reinterpret_cast<uint8_t *>(pscr + 32);                 // [PERM]
+    uint8_t *inv = perms + PERM;                                             // [32]
+    const int64_t row = (int64_t)blockIdx.x * PREP_W + wib;
+    if (row >= a.R.rows) return;
+    const int64_t g = row / a.R.R;
+    const int64_t ri = row - g * a.R.R;
+    const int n = a.R.n[g];
+    const int k = a.k[row];
+    int status = FW_OK;
+    if (n < 1 || n > a.R.max_n || n > 32 || k < 1 || k > n || k > a.k_max) status = FW_ERR_INVALID_ARG;
+    const float *lg = a.R.logits + a.R.logit_off[g] + ri * (status == FW_OK ? n : 0);
+    const float l = (status == FW_OK && lane < n) ? lg[lane] : -INFINITY;
+    if (status == FW_OK && __any_sync(FW_FULL, lane < n && !isfinite(l))) status = FW_ERR_NONFINITE;
+    if (status != FW_OK) {
+        if (lane == 0) {
+            if (a.row_status) a.row_status[row] = status;
+            a.cand_count[row] = -1;
+            a.best_gap[row] = __int_as_float(0x7fc00000);
+            a.best_rank[row] = ~0ull;
+            if (a.topk_gap) a.topk_gap[row] = __int_as_float(0x7fc00000);
+        }
+        for (int t = lane; t < a.k_max; t += 32) a.best_idx[row * a.k_max + t] = -1;
+        return;
+    }
+    const VT *V = reinterpret_cast<const VT *>(a.R.v) + a.R.v_off[g];
+    const float M = warp_max(l);
+    double p = lane < n ? exp((double)l - (double)M) : 0.0;
+    p = p / warp_sum_d(p);
+    int rank = 0;
+    for (int s2 = 0; s2 < n; ++s2) {
+        const float ls = __shfl_sync(FW_FULL, l, s2);
+        rank += (ls > l) || (ls == l && s2 < lane);
+    }
+    const bool inA0 = lane < n && rank < k;
+    const uint32_t A0 = __ballot_sync(FW_FULL, inA0);
+    const df pd = df_from_double(p);
+    // local key order: L = first nL keys outside A0, then A0, then H'
+    const int nL = min(EM, n - k);
+    const int nHp = n - k - nL;
+    uint8_t *perm = perms;
+    if (lane < n) {
+        const uint32_t below = (1u << lane) - 1u;
+        const int bo = __popc(~A0 & below);
+        const int bi = __popc(A0 & below);
+        const int loc = inA0 ? EM + bi : (bo < nL ? bo : EM + k + (bo - nL));
+        perm[loc] = (uint8_t)lane;
+        inv[lane] = (uint8_t)loc;
+        pscr[lane] = p;
+    }
+    SlotGeom S;
+    S.slot = slot;
+    S.k = k;
+    S.nL = nL;
+    S.nHp = nHp;
+    S.RA = EM + k + nHp + 2;
+    S.RH = EM + nHp + 2;
+    S.offH = OFF_A + k * S.RA;
+    const int tot = slot_floats(k, nHp);
+    for (int i = lane; i < tot; i += 32) S.slot[i] = (i >= nL && i < EM) ? INFINITY : 0.f;
+    // Gram entries over the n keys plus g0 (index n), staged DCH dimensions at a
+    // time.  The upper triangle is cut into tiles of 2 rows x 4 columns (lane
+    // takes tiles lane, lane + 32, ...); a tile reads 6 staged values per
+    // dimension for its 8 products, and each product is four interleaved
+    // partial sums per chunk.  Slot i = 8 * tile + 4 * (x - x0) + (y - y0);
+    // px_ = -1 marks slots outside the triangle (and |g0|^2, known exactly).
+    const int R1 = n + 1, nby = (R1 + 3) / 4;
+    int tx0[MAXT], ty0[MAXT];
+    int px_[PPL], py_[PPL];
+    float acc[PPL];
+#pragma unroll
+    for (int tl = 0; tl < MAXT; ++tl) {
+        int tid_ = lane + 32 * tl, bx = 0;
+        bool ok = true;
+        for (;;) {  // rows 2bx, 2bx+1 hold tiles by = bx/2 .. nby-1
+            if (2 * bx >= R1) {
+                ok = false;
+                break;
             }
-            for (int t = lane; t < a.k_max; t += 32) a.best_idx[row * a.k_max + t] = -1;
-            continue;
+            const int cnt = nby - bx / 2;
+            if (tid_ < cnt) break;
+            tid_ -= cnt;
+            ++bx;
         }
-        const VT *V = reinterpret_cast<const VT *>(a.R.v) + a.R.v_off[g];
-        const float M = warp_max(l);
-        double p = lane < n ? exp((double)l - (double)M) : 0.0;
-        p = p / warp_sum_d(p);
-        int rank = 0;
-        for (int s2 = 0; s2 < n; ++s2) {
-            const float ls = __shfl_sync(FW_FULL, l, s2);
-            rank += (ls > l) || (ls == l && s2 < lane);
+        tx0[tl] = ok ? 2 * bx : -1;
+        ty0[tl] = ok ? 4 * (bx / 2 + tid_) : -1;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int x = tx0[tl] + (e >> 2), y = ty0[tl] + (e & 3);
+            const bool in = ok && x <= y && y < R1 && x < n;
+            px_[8 * tl + e] = in ? x : -1;
+            py_[8 * tl + e] = y;
+            acc[8 * tl + e] = 0.f;
         }
-        const bool inA0 = lane < n && rank < k;
-        const uint32_t A0 = __ballot_sync(FW_FULL, inA0);
-        const df pd = df_from_double(p);
-        // local key order: L = first nL keys outside A0, then A0, then H'
-        const int nL = min(EM, n - k);
-        const int nHp = n - k - nL;
-        uint8_t *perm = perms + rr * PERM;
-        if (lane < n) {
-            const uint32_t below = (1u << lane) - 1u;
-            const int bo = __popc(~A0 & below);
-            const int bi = __popc(A0 & below);
-            const int loc = inA0 ? EM + bi : (bo < nL ? bo : EM + k + (bo - nL));
-            perm[loc] = (uint8_t)lane;
-            inv[lane] = (uint8_t)loc;
-            pscr[lane] = p;
+    }
+    df g0[DPL];
+#pragma unroll
+    for (int t = 0; t < DPL; ++t) g0[t] = df_zero();
+#pragma unroll
+    for (int ch = 0; ch < DPL / TCH; ++ch) {
+        __syncwarp();
+        // the chunk's values of all n keys into Ust (loads issued back to back)
+        stage_value_cols<DCH>(V, n, d, ch * DCH, Ust, lane);
+        __syncwarp();
+        // mu over the chunk's columns (j ascending, double-float), then
+        // u_j = p_j (v_j - mu) in place
+        df mu[TCH];
+#pragma unroll
+        for (int tt = 0; tt < TCH; ++tt) mu[tt] = df_zero();
+        for (int j = 0; j < n; ++j) {
+            const df pj = shfl_df(pd, j);
+#pragma unroll
+            for (int tt = 0; tt < TCH; ++tt)
+                mu[tt] = df_add(mu[tt], df_mul_f(pj, Ust[j * (DCH + 1) + lane + 32 * tt]));
         }
-        SlotGeom S;
-        S.slot = slots + (size_t)rr * a.stride;
-        S.k = k;
-        S.nL = nL;
-        S.nHp = nHp;
-        S.RA = EM + k + nHp + 2;
-        S.RH = EM + nHp + 2;
-        S.offH = OFF_A + k * S.RA;
-        const int tot = slot_floats(k, nHp);
-        for (int i = lane; i < tot; i += 32) S.slot[i] = (i >= nL && i < EM) ? INFINITY : 0.f;
-        // Gram entries over the n keys plus g0 (index n), staged DCH dimensions at a
-        // time.  The upper triangle is cut into tiles of 2 rows x 4 columns (lane
-        // takes tiles lane, lane + 32, ...); a tile reads 6 staged values per
-        // dimension for its 8 products, and each product is four interleaved
-        // partial sums per chunk.  Slot i = 8 * tile + 4 * (x - x0) + (y - y0);
-        // px_ = -1 marks slots outside the triangle (and |g0|^2, known exactly).
-        const int R1 = n + 1, nby = (R1 + 3) / 4;
-        int tx0[MAXT], ty0[MAXT];
-        int px_[PPL], py_[PPL];
-        float acc[PPL];
+        for (int j = 0; j < n; ++j) {
+            const df pj = shfl_df(pd, j);
+            const bool in = (A0 >> j) & 1u;
+#pragma unroll
+            for (int tt = 0; tt < TCH; ++tt) {
+                const int t = ch * TCH + tt;
+                float *cell = Ust + j * (DCH + 1) + lane + 32 * tt;
+                const df u = df_mul(pj, df_rsub_f(*cell, mu[tt]));
+                *cell = u.hi;
+                if (in) g0[t] = df_add(g0[t], u);
+            }
+        }
+#pragma unroll
+        for (int tt = 0; tt < TCH; ++tt) Ust[n * (DCH + 1) + lane + 32 * tt] = g0[ch * TCH + tt].hi;
+        __syncwarp();
 #pragma unroll
         for (int tl = 0; tl < MAXT; ++tl) {
-            int tid_ = lane + 32 * tl, bx = 0;
-            bool ok = true;
-            for (;;) {  // rows 2bx, 2bx+1 hold tiles by = bx/2 .. nby-1
-                if (2 * bx >= R1) {
-                    ok = false;
-                    break;
-                }
-                const int cnt = nby - bx / 2;
-                if (tid_ < cnt) break;
-                tid_ -= cnt;
-                ++bx;
-            }
-            tx0[tl] = ok ? 2 * bx : -1;
-            ty0[tl] = ok ? 4 * (bx / 2 + tid_) : -1;
+            if (tx0[tl] < 0) continue;
+            const float *ux[2], *uy[4];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const int x = tx0[tl] + (e >> 2), y = ty0[tl] + (e & 3);
-                const bool in = ok && x <= y && y < R1 && x < n;
-                px_[8 * tl + e] = in ? x : -1;
-                py_[8 * tl + e] = y;
-                acc[8 * tl + e] = 0.f;
-            }
-        }
-        df g0[DPL];
+            for (int e = 0; e < 2; ++e) ux[e] = Ust + min(tx0[tl] + e, n) * (DCH + 1);
 #pragma unroll
-        for (int t = 0; t < DPL; ++t) g0[t] = df_zero();
+            for (int e = 0; e < 4; ++e) uy[e] = Ust + min(ty0[tl] + e, n) * (DCH + 1);
+            float sp[8][4];
 #pragma unroll
-        for (int ch = 0; ch < DPL / TCH; ++ch) {
-            __syncwarp();
-            // the chunk's values of all n keys into Ust (loads issued back to back)
-            stage_value_cols<DCH>(V, n, d, ch * DCH, Ust, lane);
-            __syncwarp();
-            // mu over the chunk's columns (j ascending, double-float), then
-            // u_j = p_j (v_j - mu) in place
-            df mu[TCH];
+            for (int e = 0; e < 8; ++e)
 #pragma unroll
-            for (int tt = 0; tt < TCH; ++tt) mu[tt] = df_zero();
-            for (int j = 0; j < n; ++j) {
-                const df pj = shfl_df(pd, j);
+                for (int c4 = 0; c4 < 4; ++c4) sp[e][c4] = 0.f;
+            for (int c = 0; c < DCH; c += 4) {
 #pragma unroll
-                for (int tt = 0; tt < TCH; ++tt)
-                    mu[tt] = df_add(mu[tt], df_mul_f(pj, Ust[j * (DCH + 1) + lane + 32 * tt]));
-            }
-            for (int j = 0; j < n; ++j) {
-                const df pj = shfl_df(pd, j);
-                const bool in = (A0 >> j) & 1u;
+                for (int c4 = 0; c4 < 4; ++c4) {
+                    const float a0 = ux[0][c + c4], a1 = ux[1][c + c4];
 #pragma unroll
-                for (int tt = 0; tt < TCH; ++tt) {
-                    const int t = ch * TCH + tt;
-                    float *cell = Ust + j * (DCH + 1) + lane + 32 * tt;
-                    const df u = df_mul(pj, df_rsub_f(*cell, mu[tt]));
-                    *cell = u.hi;
-                    if (in) g0[t] = df_add(g0[t], u);
-                }
-            }
-#pragma unroll
-            for (int tt = 0; tt < TCH; ++tt) Ust[n * (DCH + 1) + lane + 32 * tt] = g0[ch * TCH + tt].hi;
-            __syncwarp();
-#pragma unroll
-            for (int tl = 0; tl < MAXT; ++tl) {
-                if (tx0[tl] < 0) continue;
-                const float *ux[2], *uy[4];
-#pragma unroll
-                for (int e = 0; e < 2; ++e) ux[e] = Ust + min(tx0[tl] + e, n) * (DCH + 1);
-#pragma unroll
-                for (int e = 0; e < 4; ++e) uy[e] = Ust + min(ty0[tl] + e, n) * (DCH + 1);
-                float sp[8][4];
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-#pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) sp[e][c4] = 0.f;
-                for (int c = 0; c < DCH; c += 4) {
-#pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) {
-                        const float a0 = ux[0][c + c4], a1 = ux[1][c + c4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float b = uy[e][c + c4];
-                            sp[e][c4] = fmaf(a0, b, sp[e][c4]);
-                            sp[4 + e][c4] = fmaf(a1, b, sp[4 + e][c4]);
-                        }
+                    for (int e = 0; e < 4; ++e) {
+                        const float b = uy[e][c + c4];
+                        sp[e][c4] = fmaf(a0, b, sp[e][c4]);
+                        sp[4 + e][c4] = fmaf(a1, b, sp[4 + e][c4]);
                     }
                 }
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[8 * tl + e] += (sp[e][0] + sp[e][1]) + (sp[e][2] + sp[e][3]);
             }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[8 * tl + e] += (sp[e][0] + sp[e][1]) + (sp[e][2] + sp[e][3]);
         }
-        df nrm = df_zero();
+    }
+    df nrm = df_zero();
 #pragma unroll
-        for (int t = 0; t < DPL; ++t) nrm = df_add(nrm, df_mul(g0[t], g0[t]));
-        nrm = warp_sum_df(nrm);
-        const double P0 = warp_sum_d(inA0 ? p : 0.0);
-        const double g0n2 = fmax(df_to_double(nrm), 0.0);
-        const double t = g0n2 / (P0 * P0);  // es(A0)^2
-        const double sqt = sqrt(t);
-        if (lane == 0 && a.topk_gap) a.topk_gap[row] = (float)sqt;
-        // kappa: 2.2x the per-subset error bound of an fp32 evaluation of either form
-        const int Lc = k * (k + 1) / 2 + 2 * n + 16;
-        S.kap = (float)(2.2 * ((double)d * 0.25 + Lc + 16) * 5.9604644775390625e-8);
-        S.g0n = (float)sqrt(g0n2) * 1.0001f;
-        // a_x = |u_x| + sqrt(t) p_x (rounded up) from the diagonal entries
+    for (int t = 0; t < DPL; ++t) nrm = df_add(nrm, df_mul(g0[t], g0[t]));
+    nrm = warp_sum_df(nrm);
+    const double P0 = warp_sum_d(inA0 ? p : 0.0);
+    const double g0n2 = fmax(df_to_double(nrm), 0.0);
+    const double t = g0n2 / (P0 * P0);  // es(A0)^2
+    const double sqt = sqrt(t);
+    if (lane == 0 && a.topk_gap) a.topk_gap[row] = (float)sqt;
+    // kappa: 2.2x the per-subset error bound of an fp32 evaluation of either form
+    const int Lc = k * (k + 1) / 2 + 2 * n + 16;
+    S.kap = (float)(2.2 * ((double)d * 0.25 + Lc + 16) * 5.9604644775390625e-8);
+    S.g0n = (float)sqrt(g0n2) * 1.0001f;
+    // a_x = |u_x| + sqrt(t) p_x (rounded up) from the diagonal entries
 #pragma unroll
-        for (int i = 0; i < PPL; ++i)
-            if (px_[i] >= 0 && px_[i] == py_[i] && px_[i] < n)
-                aX[px_[i]] = sqrtf(fmaxf(acc[i], 0.f)) * 1.0001f + (float)(sqt * pscr[px_[i]]) * 1.0001f;
-        __syncwarp();
-        // scatter the folded entries into the walk tables
-        const float tf = (float)t, P0f = (float)P0;
+    for (int i = 0; i < PPL; ++i)
+        if (px_[i] >= 0 && px_[i] == py_[i] && px_[i] < n)
+            aX[px_[i]] = sqrtf(fmaxf(acc[i], 0.f)) * 1.0001f + (float)(sqt * pscr[px_[i]]) * 1.0001f;
+    __syncwarp();
+    // scatter the folded entries into the walk tables
+    const float tf = (float)t, P0f = (float)P0;
 #pragma unroll
-        for (int i = 0; i < PPL; ++i) {
-            const int x = px_[i], y = py_[i];
-            if (x < 0 || x == n) continue;
-            // G' = u.u - t p p^T in fp32 (a few ulps of a_x a_y, inside kappa's slack)
-            const float tpx = tf * (float)pscr[x];
-            if (y == n) {
-                const float sx = ((A0 >> x) & 1u) ? -2.f : 2.f;
-                put_linear(S, inv[x], sx * fmaf(-tpx, P0f, acc[i]), aX[x]);
+    for (int i = 0; i < PPL; ++i) {
+        const int x = px_[i], y = py_[i];
+        if (x < 0 || x == n) continue;
+        // G' = u.u - t p p^T in fp32 (a few ulps of a_x a_y, inside kappa's slack)
+        const float tpx = tf * (float)pscr[x];
+        if (y == n) {
+            const float sx = ((A0 >> x) & 1u) ? -2.f : 2.f;
+            put_linear(S, inv[x], sx * fmaf(-tpx, P0f, acc[i]), aX[x]);
+        } else {
+            const float gp = fmaf(-tpx, (float)pscr[y], acc[i]);
+            if (x == y) {
+                put_diag(S, inv[x], gp, aX[x]);
             } else {
-                const float gp = fmaf(-tpx, (float)pscr[y], acc[i]);
-                if (x == y) {
-                    put_diag(S, inv[x], gp, aX[x]);
-                } else {
-                    put_entry(S, inv[x], inv[y], gp, aX[x], aX[y]);
-                    put_entry(S, inv[y], inv[x], gp, aX[y], aX[x]);
-                }
+                put_entry(S, inv[x], inv[y], gp, aX[x], aX[y]);
+                put_entry(S, inv[y], inv[x], gp, aX[y], aX[x]);
             }
         }
-        __syncwarp();
-        // Bounds of the walk: the pair terms of the inner set L (G2, x < y) and of
-        // every two keys that can be added back (L x L, H' x H' from HH, H' x L as
-        // twice the folded G'(y, L)); for each list the prefix sums of its
-        // smallest terms (pref[m] = sum of the m smallest) and the sum of |terms|.
-        // The warp takes the smallest remaining term round by round.
-        {
-            const int nLL = EM * (EM - 1) / 2, nHH = nHp * (nHp - 1) / 2, E = nLL + nHH + EM * nHp;
-            float *vals = Ust;
-            float *PF = S.slot + off_pref(k, nHp), *PR = S.slot + off_prefr(k, nHp);
-            if (E <= ust_floats && E <= 512) {
-                for (int e = lane; e < E; e += 32) {
-                    float v;
-                    if (e < nLL) {
-                        int x = 0, rem = e;
-                        while (rem >= EM - 1 - x) {
-                            rem -= EM - 1 - x;
-                            ++x;
-                        }
-                        v = S.slot[3 * EM + x * EM + x + 1 + rem];
-                    } else if (e < nLL + nHH) {
-                        int x = 0, rem = e - nLL;
-                        while (rem >= nHp - 1 - x) {
-                            rem -= nHp - 1 - x;
-                            ++x;
-                        }
-                        v = S.slot[S.offH + x * S.RH + EM + x + 1 + rem];
-                    } else {
-                        const int f = e - nLL - nHH, y = f / EM, j = f - y * EM;
-                        v = 2.f * S.slot[S.offH + y * S.RH + j];
+    }
+    __syncwarp();
+    // Bounds of the walk: the pair terms of the inner set L (G2, x < y) and of
+    // every two keys that can be added back (L x L, H' x H' from HH, H' x L as
+    // twice the folded G'(y, L)); for each list the prefix sums of its
+    // smallest terms (pref[m] = sum of the m smallest) and the sum of |terms|.
+    // The warp takes the smallest remaining term round by round.
+    {
+        const int nLL = EM * (EM - 1) / 2, nHH = nHp * (nHp - 1) / 2, E = nLL + nHH + EM * nHp;
+        float *vals = Ust;
+        float *PF = S.slot + off_pref(k, nHp), *PR = S.slot + off_prefr(k, nHp);
+        if (E <= ust_floats && E <= 512) {
+            for (int e = lane; e < E; e += 32) {
+                float v;
+                if (e < nLL) {
+                    int x = 0, rem = e;
+                    while (rem >= EM - 1 - x) {
+                        rem -= EM - 1 - x;
+                        ++x;
                     }
-                    vals[e] = v;
+                    v = S.slot[3 * EM + x * EM + x + 1 + rem];
+                } else if (e < nLL + nHH) {
+                    int x = 0, rem = e - nLL;
+                    while (rem >= nHp - 1 - x) {
+                        rem -= nHp - 1 - x;
+                        ++x;
+                    }
+                    v = S.slot[S.offH + x * S.RH + EM + x + 1 + rem];
+                } else {
+                    const int f = e - nLL - nHH, y = f / EM, j = f - y * EM;
+                    v = 2.f * S.slot[S.offH + y * S.RH + j];
                 }
-                __syncwarp();
-                // pass 0: the first nLL entries (L x L) for the inner bound; pass 1: all E
-                for (int pass = 0; pass < 2; ++pass) {
-                    const int En = pass == 0 ? nLL : E;
-                    const int need = (pass == 0 ? npref(k) : nprefr(k)) - 1;
-                    smallest_prefix(vals, En, need, pass == 0 ? PF : PR, lane);
-                }
-            } else if (lane == 0) {  // (cannot happen for n <= 32; the bounds then never prune)
-                for (int m = 0; m < npref(k); ++m) PF[m] = -INFINITY;
-                PF[npref(k)] = 0.f;
-                for (int m = 0; m < nprefr(k); ++m) PR[m] = -INFINITY;
-                PR[nprefr(k)] = 0.f;
+                vals[e] = v;
             }
             __syncwarp();
-        }
-        if ((lane & (ERW - 1)) == rr && k <= 31) {
-            my.slot = S.slot;
-            my.perm = perm;
-            my.k = k;
-            my.nL = nL;
-            my.nHp = nHp;
-            my.half = lane / ERW;
-            my.kappa = S.kap;
-            my.g0n = S.g0n;
-            my.cand = a.cand + row * ECAP;
-            my.ccount = a.cand_count + row;
-            my_walk = true;
-        }
-        if (lane == 0) {
-            a.cand_count[row] = k <= 31 ? 0 : ECAP + 1;  // k = 32: the exhaustive path
-            if (a.row_status) a.row_status[row] = FW_OK;
+            // pass 0: the first nLL entries (L x L) for the inner bound; pass 1: all E
+            for (int pass = 0; pass < 2; ++pass) {
+                const int En = pass == 0 ? nLL : E;
+                const int need = (pass == 0 ? npref(k) : nprefr(k)) - 1;
+                smallest_prefix(vals, En, need, pass == 0 ? PF : PR, lane);
+            }
+        } else if (lane == 0) {  // (cannot happen for n <= 32; the bounds then never prune)
+            for (int m = 0; m < npref(k); ++m) PF[m] = -INFINITY;
+            PF[npref(k)] = 0.f;
+            for (int m = 0; m < nprefr(k); ++m) PR[m] = -INFINITY;
+            PR[nprefr(k)] = 0.f;
         }
         __syncwarp();
     }
-    __syncwarp();
+    // the tables out: slot, key order, kappa and |g0|
+    for (int i = lane; i < tot; i += 32) a.slots[row * a.stride + i] = S.slot[i];
+    if (lane < PERM / 4)
+        reinterpret_cast<uint32_t *>(a.perms + row * PERM)[lane] = reinterpret_cast<const uint32_t *>(perm)[lane];
+    if (lane == 0) {
+        a.kg[row] = make_float2(S.kap, S.g0n);
+        a.cand_count[row] = k <= 31 ? 0 : ECAP + 1;  // k = 32: the exhaustive path
+        if (a.row_status) a.row_status[row] = FW_OK;
+    }
+}
 
-    // ------------------------------------------------------------------ walk
+__global__ void __launch_bounds__(32, 1) k_enum_walk(const EnumArgs a)
+{
+    extern __shared__ float smem[];
+    const int lane = threadIdx.x;
+    float *slots = smem;                                                   // [ERW][stride]
+    uint8_t *perms = reinterpret_cast<uint8_t *>(smem + ERW * a.stride);   // [ERW][PERM]
+    const int64_t row0 = (int64_t)blockIdx.x * ERW;
+    const int nrow = (int)min((int64_t)ERW, a.R.rows - row0);
+    {
+        // ERW * stride is a multiple of 4 floats, so every block's tables start 16-byte aligned
+        const float *src = a.slots + row0 * a.stride;
+        const int tot = nrow * a.stride, nv = tot / 4;
+        for (int i = lane; i < nv; i += 32)
+            reinterpret_cast<float4 *>(slots)[i] = reinterpret_cast<const float4 *>(src)[i];
+        for (int i = 4 * nv + lane; i < tot; i += 32) slots[i] = src[i];
+        const int pv = nrow * PERM / 16;
+        for (int i = lane; i < pv; i += 32)
+            reinterpret_cast<uint4 *>(perms)[i] = reinterpret_cast<const uint4 *>(a.perms + row0 * PERM)[i];
+    }
+    __syncwarp();
+    const int rr = lane & (ERW - 1);
+    const int64_t row = row0 + rr;
+    Walk my;
+    const bool my_walk = rr < nrow && a.cand_count[row] == 0;
+    if (my_walk) {
+        const int n = a.R.n[row / a.R.R];
+        my.k = a.k[row];
+        my.nL = min(EM, n - my.k);
+        my.nHp = n - my.k - my.nL;
+        my.slot = slots + rr * a.stride;
+        my.perm = perms + rr * PERM;
+        my.half = lane / ERW;
+        const float2 kg = a.kg[row];
+        my.kappa = kg.x;
+        my.g0n = kg.y;
+        my.cand = a.cand + row * ECAP;
+        my.ccount = a.cand_count + row;
+    }
     {
         const uint32_t wmask = __ballot_sync(FW_FULL, my_walk);
         const int key = my_walk ? (my.k << 8) | (my.nL << 16) | my.nHp : -1;
@@ -798,35 +836,51 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
         my.sync_mask = same ? wmask : 0u;
     }
     if (my_walk) walk_row(my);
-    __syncwarp();
+}
 
-    // ----------------------------------------------------- exact re-scoring
-    for (int rr = 0; rr < ERW; ++rr) {
-        const int64_t row = row0 + rr;
-        if (row >= a.R.rows) break;
-        const int cc = a.cand_count[row];
-        if (cc < 0) continue;  // invalid row, outputs already written
-        if (cc > ECAP || cc == 0) {
-            if (lane == 0) a.fb_list[atomicAdd(a.fb_count, 1)] = (int)row;
-            continue;
+template <int DPL, typename VT>
+__global__ void __launch_bounds__(32 * RS_W) k_enum_rescore(const EnumArgs a)
+{
+    extern __shared__ float smem[];
+    constexpr int d = DPL * 32;
+    constexpr int DCH = d < 64 ? d : 64;
+    constexpr int TCH = DCH / 32;
+    const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+    const int ust_floats = (((a.R.max_n + 1) * (DCH + 1)) + 1) & ~1;
+    float *Ust = smem + (size_t)wib * rescore_floats(ust_floats);  // [max_n+1][DCH+1]
+    const int64_t row = (int64_t)blockIdx.x * RS_W + wib;
+    if (row >= a.R.rows) return;
+    const int cc = a.cand_count[row];
+    if (cc < 0) return;  // invalid row, outputs already written
+    if (cc > ECAP || cc == 0) {
+        if (lane == 0) a.fb_list[atomicAdd(a.fb_count, 1)] = (int)row;
+        return;
+    }
+    const int64_t g = row / a.R.R;
+    const int64_t ri = row - g * a.R.R;
+    const int n = a.R.n[g];
+    const int k = a.k[row];
+    const VT *V = reinterpret_cast<const VT *>(a.R.v) + a.R.v_off[g];
+    const float *lg = a.R.logits + a.R.logit_off[g] + ri * n;
+    const float l = lane < n ? lg[lane] : -INFINITY;
+    const float M = warp_max(l);
+    double p = lane < n ? exp((double)l - (double)M) : 0.0;
+    p = p / warp_sum_d(p);
+    const df pd = df_from_double(p);
+    // candidates in groups of RCB; per 64-column chunk: stage the values, mu over
+    // the chunk, and each candidate's g over the chunk, whose squares add into a
+    // per-lane partial (same order of operations as one pass over all columns)
+    double best = INFINITY;
+    uint64_t brank = ~0ull;
+    uint32_t bmask = 0u;
+    for (int c0 = 0; c0 < cc; c0 += RCB) {
+        uint32_t cm[RCB];
+        df sq[RCB];
+#pragma unroll
+        for (int ci = 0; ci < RCB; ++ci) {
+            cm[ci] = c0 + ci < cc ? a.cand[row * ECAP + c0 + ci] : 0u;
+            sq[ci] = df_zero();
         }
-        const int64_t g = row / a.R.R;
-        const int64_t ri = row - g * a.R.R;
-        const int n = a.R.n[g];
-        const int k = a.k[row];
-        const VT *V = reinterpret_cast<const VT *>(a.R.v) + a.R.v_off[g];
-        const float *lg = a.R.logits + a.R.logit_off[g] + ri * n;
-        const float l = lane < n ? lg[lane] : -INFINITY;
-        const float M = warp_max(l);
-        double p = lane < n ? exp((double)l - (double)M) : 0.0;
-        p = p / warp_sum_d(p);
-        const df pd = df_from_double(p);
-        // per 64-column chunk: stage the values, mu over the chunk, and each
-        // candidate's g over the chunk, whose squares add into a per-lane partial
-        // (kept in the slots, free after the walk); same order of operations as
-        // one pass over all columns
-        df *cacc = reinterpret_cast<df *>(slots);  // [ECAP][32]
-        for (int ci = 0; ci < cc; ++ci) cacc[ci * 32 + lane] = df_zero();
         for (int ch = 0; ch < DPL / TCH; ++ch) {
             __syncwarp();
             stage_value_cols<DCH>(V, n, d, ch * DCH, Ust, lane);
@@ -840,30 +894,27 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
                 for (int tt = 0; tt < TCH; ++tt)
                     mu[tt] = df_add(mu[tt], df_mul_f(pj, Ust[j * (DCH + 1) + lane + 32 * tt]));
             }
-            for (int ci = 0; ci < cc; ++ci) {
-                const uint32_t m = a.cand[row * ECAP + ci];
+#pragma unroll
+            for (int ci = 0; ci < RCB; ++ci) {
                 df gv[TCH];
 #pragma unroll
                 for (int tt = 0; tt < TCH; ++tt) gv[tt] = df_zero();
-                for (uint32_t mm = m; mm; mm &= mm - 1) {
+                for (uint32_t mm = cm[ci]; mm; mm &= mm - 1) {
                     const int j = __ffs(mm) - 1;
                     const df pj = shfl_df(pd, j);
 #pragma unroll
                     for (int tt = 0; tt < TCH; ++tt)
                         gv[tt] = df_add(gv[tt], df_mul(pj, df_rsub_f(Ust[j * (DCH + 1) + lane + 32 * tt], mu[tt])));
                 }
-                df sq = cacc[ci * 32 + lane];
 #pragma unroll
-                for (int tt = 0; tt < TCH; ++tt) sq = df_add(sq, df_mul(gv[tt], gv[tt]));
-                cacc[ci * 32 + lane] = sq;
+                for (int tt = 0; tt < TCH; ++tt) sq[ci] = df_add(sq[ci], df_mul(gv[tt], gv[tt]));
             }
         }
-        double best = INFINITY;
-        uint64_t brank = ~0ull;
-        uint32_t bmask = 0u;
-        for (int ci = 0; ci < cc; ++ci) {
-            const uint32_t m = a.cand[row * ECAP + ci];
-            const df s3 = warp_sum_df(cacc[ci * 32 + lane]);
+#pragma unroll
+        for (int ci = 0; ci < RCB; ++ci) {
+            if (c0 + ci >= cc) break;
+            const uint32_t m = cm[ci];
+            const df s3 = warp_sum_df(sq[ci]);
             const double P = warp_sum_d(((m >> lane) & 1u) ? p : 0.0);
             const double e = fmax(df_to_double(s3), 0.0) / (P * P);
             const uint64_t rk = colex_rank_mask(m);
@@ -873,27 +924,33 @@ __global__ void __launch_bounds__(32, 1) k_enum(const EnumArgs a)
                 bmask = m;
             }
         }
-        if (lane == 0) {
-            a.best_gap[row] = (float)sqrt(best);
-            a.best_rank[row] = brank;
-        }
-        const bool mine = (bmask >> lane) & 1u;
-        const int pos = __popc(bmask & ((1u << lane) - 1u));
-        if (mine) a.best_idx[row * a.k_max + pos] = lane;
-        for (int t = k + lane; t < a.k_max; t += 32) a.best_idx[row * a.k_max + t] = -1;
     }
+    if (lane == 0) {
+        a.best_gap[row] = (float)sqrt(best);
+        a.best_rank[row] = brank;
+    }
+    const bool mine = (bmask >> lane) & 1u;
+    const int pos = __popc(bmask & ((1u << lane) - 1u));
+    if (mine) a.best_idx[row * a.k_max + pos] = lane;
+    for (int t = k + lane; t < a.k_max; t += 32) a.best_idx[row * a.k_max + t] = -1;
 }
 
-// ---- exhaustive fp64 path: one block per listed row, every C(n,k) subset in
-// colex order, each evaluated in the difference form around the top-k set
-// (es^2 = t + val / P^2) so that heavy keys kept in A0 never cancel.
+// ---- exhaustive path: FBS blocks per listed row, every C(n,k) subset in colex
+// order, each evaluated in the difference form around the top-k set
+// (es^2 = t + val / P^2) so that heavy keys kept in A0 never cancel.  A first
+// pass screens every subset in fp32 with a rigorous error bound; the second
+// evaluates in fp64 only those whose lower bound reaches the chunk's smallest
+// upper bound.
 template <int DPL, typename VT>
 __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
 {
     constexpr int d = DPL * 32;
     __shared__ double Gs[33][34];
     __shared__ double Ms[32][33];
+    __shared__ float Mf[32][33];  // Ms in fp32, off-diagonal entries doubled
     __shared__ double ps[32];
+    __shared__ float pf[32];
+    __shared__ float ured_f[256];
     __shared__ double ured_e[256];
     __shared__ unsigned long long ured_r[256];
     __shared__ double s_t, s_P0;
@@ -962,13 +1019,21 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
             }
         }
         __syncthreads();
+        // Gram entries G_xy = u_x . u_y (row n: g0) in double-float, four
+        // interleaved partial sums per product
         for (int q = tid; q < (n + 1) * (n + 1); q += blockDim.x) {
             const int x = q / (n + 1), y = q % (n + 1);
             if (y < x) continue;
-            double s = 0.0;
-            for (int c = 0; c < d; ++c)
-                s += ((double)Ush[x * (d + 1) + c] + (double)Usl[x * d + c]) *
-                     ((double)Ush[y * (d + 1) + c] + (double)Usl[y * d + c]);
+            df s4[4] = {df_zero(), df_zero(), df_zero(), df_zero()};
+            for (int c = 0; c < d; c += 4) {
+#pragma unroll
+                for (int c4 = 0; c4 < 4; ++c4) {
+                    const df ux = {Ush[x * (d + 1) + c + c4], Usl[x * d + c + c4]};
+                    const df uy = {Ush[y * (d + 1) + c + c4], Usl[y * d + c + c4]};
+                    s4[c4] = df_add(s4[c4], df_mul(ux, uy));
+                }
+            }
+            const double s = df_to_double(df_add(df_add(s4[0], s4[1]), df_add(s4[2], s4[3])));
             Gs[x][y] = s;
             Gs[y][x] = s;
         }
@@ -981,6 +1046,8 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
             double m = sx * sy * (Gs[x][y] - t * ps[x] * ps[y]);
             if (x == y) m += 2.0 * sx * (Gs[x][n] - t * P0 * ps[x]);
             Ms[x][y] = m;
+            Mf[x][y] = (float)(x == y ? m : 2.0 * m);
+            if (y == 0) pf[x] = (float)ps[x];
         }
         __syncthreads();
         const uint64_t total = binom64(n, k);
@@ -991,39 +1058,112 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
         const uint64_t per = (span + blockDim.x - 1) / blockDim.x;
         const uint64_t lo = clo + per * tid;
         const uint64_t hi = lo + per < chi ? lo + per : chi;
-        double best = INFINITY;
-        unsigned long long brank = ~0ull;
-        if (lo < hi) {
-            int cmb[32];
-            uint64_t r = lo;
+        // colex unranking, successor and mask of a k-combination
+        auto unrank = [&](uint64_t r, int *cmb) {
             int top = n - 1;
-            for (int i = k; i >= 1; --i) {  // unrank: largest c with C(c, i) <= r
+            for (int i = k; i >= 1; --i) {  // largest c with C(c, i) <= r
                 int c = i - 1;
                 while (c + 1 <= top && binom64(c + 1, i) <= r) ++c;
                 r -= binom64(c, i);
                 cmb[i - 1] = c;
                 top = c - 1;
             }
+        };
+        auto succ = [&](int *cmb) {
+            int i = 0;
+            while (i < k - 1 && cmb[i] + 1 == cmb[i + 1]) ++i;
+            ++cmb[i];
+            for (int q2 = 0; q2 < i; ++q2) cmb[q2] = q2;
+        };
+        auto mask_of = [&](const int *cmb) {
+            uint32_t am = 0u;
+            for (int i = 0; i < k; ++i) am |= 1u << cmb[i];
+            return am;
+        };
+        // fp32 value of es^2 in the difference form with a rigorous bound on
+        // its error: the fp32 entries are the fp64 ones rounded (relative error
+        // u), the sum of N terms adds at most N u times the sum of their
+        // magnitudes, P(A) sums k positive terms, and the reciprocal, products
+        // and the final sum add a few u more (plus the denormal floor per term)
+        const float tf = (float)t;
+        auto screen = [&](uint32_t am, float &elo, float &ehi) {
+            const uint32_t S = am ^ A0;
+            float val = 0.f, ab = 0.f;
+            for (uint32_t m1 = S; m1; m1 &= m1 - 1) {
+                const int x = __ffs(m1) - 1;
+                for (uint32_t m2 = m1; m2; m2 &= m2 - 1) {
+                    const float v = Mf[x][__ffs(m2) - 1];
+                    val += v;
+                    ab += fabsf(v);
+                }
+            }
+            float P = 0.f;
+            for (uint32_t m1 = am; m1; m1 &= m1 - 1) P += pf[__ffs(m1) - 1];
+            if (!(P > 1e-17f)) {
+                elo = -INFINITY;
+                ehi = INFINITY;
+                return;
+            }
+            const int sz = __popc(S);
+            const float N = (float)(sz * (sz + 1) / 2);
+            const float u = 5.9604645e-8f;
+            const float inv = __frcp_rn(P * P);
+            const float e = tf + val * inv;
+            const float err = 1.05f * inv * ((N + 2.f) * u * ab + fabsf(val) * (float)(2 * k + 6) * u +
+                                             (N + 2.f) * 1.4013e-45f) +
+                              2.f * u * (fabsf(tf) + fabsf(e));
+            if (!(fabsf(e) < INFINITY) || !(err < INFINITY)) {
+                elo = -INFINITY;
+                ehi = INFINITY;
+                return;
+            }
+            elo = e - err;
+            ehi = e + err;
+        };
+        // pass 1: the smallest upper bound over the chunk
+        float ub = INFINITY;
+        int cmb[32];
+        if (lo < hi) {
+            unrank(lo, cmb);
             for (uint64_t rk = lo; rk < hi; ++rk) {
-                uint32_t am = 0u;
-                for (int i = 0; i < k; ++i) am |= 1u << cmb[i];
-                const uint32_t S = am ^ A0;
-                double val = 0.0, P = P0;
-                for (uint32_t m1 = S; m1; m1 &= m1 - 1) {
-                    const int x = __ffs(m1) - 1;
-                    P += ((A0 >> x) & 1u) ? -ps[x] : ps[x];
-                    val += Ms[x][x];
-                    for (uint32_t m2 = m1 & (m1 - 1); m2; m2 &= m2 - 1) val += 2.0 * Ms[x][__ffs(m2) - 1];
+                float elo, ehi;
+                screen(mask_of(cmb), elo, ehi);
+                ub = fminf(ub, fmaxf(ehi, 0.f));
+                succ(cmb);
+            }
+        }
+        ured_f[tid] = ub;
+        __syncthreads();
+        for (int s = blockDim.x / 2; s > 0; s >>= 1) {
+            if (tid < s) ured_f[tid] = fminf(ured_f[tid], ured_f[tid + s]);
+            __syncthreads();
+        }
+        ub = ured_f[0];
+        // pass 2: fp64 values of the subsets that may reach that bound
+        double best = INFINITY;
+        unsigned long long brank = ~0ull;
+        if (lo < hi) {
+            unrank(lo, cmb);
+            for (uint64_t rk = lo; rk < hi; ++rk) {
+                const uint32_t am = mask_of(cmb);
+                float elo, ehi;
+                screen(am, elo, ehi);
+                if (elo <= ub) {
+                    const uint32_t S = am ^ A0;
+                    double val = 0.0, P = P0;
+                    for (uint32_t m1 = S; m1; m1 &= m1 - 1) {
+                        const int x = __ffs(m1) - 1;
+                        P += ((A0 >> x) & 1u) ? -ps[x] : ps[x];
+                        val += Ms[x][x];
+                        for (uint32_t m2 = m1 & (m1 - 1); m2; m2 &= m2 - 1) val += 2.0 * Ms[x][__ffs(m2) - 1];
+                    }
+                    const double e = fmax(t + val / (P * P), 0.0);
+                    if (e < best) {
+                        best = e;
+                        brank = rk;
+                    }
                 }
-                const double e = fmax(t + val / (P * P), 0.0);
-                if (e < best) {
-                    best = e;
-                    brank = rk;
-                }
-                int i = 0;  // colex successor
-                while (i < k - 1 && cmb[i] + 1 == cmb[i + 1]) ++i;
-                ++cmb[i];
-                for (int q2 = 0; q2 < i; ++q2) cmb[q2] = q2;
+                succ(cmb);
             }
         }
         ured_e[tid] = best;
@@ -1097,11 +1237,16 @@ static int enum_stride(int max_n, int k_max)
     return best | 1;
 }
 
+// Slot stride of the workspace: the largest over every k <= max_n, so that it
+// bounds the stride of any k_max.
+static int enum_ws_stride(const RowsDev &R) { return enum_stride(R.max_n, R.max_n < 32 ? R.max_n : 32); }
+
 size_t enum_workspace(const RowsDev &R)
 {
     const size_t rows = (size_t)R.rows;
     return align256(rows * ECAP * 4) + align256(rows * 4) + align256(rows * 4) + 256 +
-           2 * align256(rows * FBS * 8);
+           2 * align256(rows * FBS * 8) + align256(rows * (size_t)enum_ws_stride(R) * 4) +
+           align256(rows * PERM) + align256(rows * 8);
 }
 
 fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, float *best_gap, int32_t *best_idx,
@@ -1130,16 +1275,28 @@ fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, f
     a.fb_e = (double *)w;
     w += align256((size_t)R.rows * FBS * 8);
     a.fb_r = (unsigned long long *)w;
+    w += align256((size_t)R.rows * FBS * 8);
+    a.slots = (float *)w;
+    w += align256((size_t)R.rows * (size_t)enum_ws_stride(R) * 4);
+    a.perms = (uint8_t *)w;
+    w += align256((size_t)R.rows * PERM);
+    a.kg = (float2 *)w;
     a.stride = enum_stride(R.max_n, k_max);
     FW_CUDA_CHECK(cudaMemsetAsync(a.fb_count, 0, sizeof(int32_t), s));
     FW_DISPATCH(R.d, R.v_dtype, {
         constexpr int DCH = DPL * 32 < 64 ? DPL * 32 : 64;
-        const size_t ust = (((size_t)(R.max_n + 1) * (DCH + 1)) + 1) & ~(size_t)1;
-        const size_t smem = ((size_t)ERW * a.stride + ust + 32) * sizeof(float) + 32 * sizeof(double) +
-                            ERW * PERM + 32;
-        FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        const unsigned grid = (unsigned)((R.rows + ERW - 1) / ERW);
-        FW_LAUNCH((k_enum<DPL, VT>), grid, 32, smem, s, a);
+        const int ust = (((R.max_n + 1) * (DCH + 1)) + 1) & ~1;
+        const size_t smem_p = (size_t)PREP_W * prep_floats(a.stride, ust) * sizeof(float);
+        FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum_prep<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem_p));
+        FW_LAUNCH((k_enum_prep<DPL, VT>), (unsigned)((R.rows + PREP_W - 1) / PREP_W), 32 * PREP_W, smem_p, s, a);
+        const size_t smem_w = (size_t)ERW * a.stride * sizeof(float) + ERW * PERM;
+        FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_w));
+        FW_LAUNCH(k_enum_walk, (unsigned)((R.rows + ERW - 1) / ERW), 32, smem_w, s, a);
+        const size_t smem_r = (size_t)RS_W * rescore_floats(ust) * sizeof(float);
+        FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum_rescore<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem_r));
+        FW_LAUNCH((k_enum_rescore<DPL, VT>), (unsigned)((R.rows + RS_W - 1) / RS_W), 32 * RS_W, smem_r, s, a);
         const size_t smem2 = (size_t)33 * (2 * DPL * 32 + 1) * sizeof(float);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum_exhaustive<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)smem2));

@@ -227,6 +227,19 @@ def test_best_degenerate_rows_take_the_exhaustive_path(fw):
     check_best(fw, rows_batch(L, V, np.full((4, 1), k)))
 
 
+@pytest.mark.parametrize("eps,d", [(1e-2, 64), (1e-3, 128), (1e-5, 64)])
+def test_best_near_duplicate_values(fw, eps, d):
+    # values scattered by eps around one point: many subsets within the fp32
+    # bounds of the best, so rows overflow the candidate buffer and the
+    # exhaustive path screens and re-scores them
+    rng = np.random.default_rng(int(eps * 1e6) + d)
+    rows, n, k = 8, 24, 6
+    L = (rng.gumbel(size=(rows, n)) * rng.uniform(0.5, 2.0, size=(rows, 1))).astype(np.float32)
+    base = rng.normal(size=(rows, 1, d))
+    V = (base + eps * rng.normal(size=(rows, n, d))).astype(np.float32)
+    check_best(fw, rows_batch(L, V, np.full((rows, 1), k)))
+
+
 def test_best_hardness_instance(fw):
     # App. A.2 construction: d=1 padded to 32 dims with zeros, uniform masses, integer points
     m = 16
