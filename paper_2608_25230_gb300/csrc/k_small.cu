@@ -216,7 +216,10 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
         for (int t = 0; t < DPL; ++t) mu[t] = df_add(mu[t], df_mul_f(pj, Uhi[j * (d + 1) + lane + 32 * t]));
     }
     // u_j = p_j (v_j - mu): high parts in place in Uhi (the exact re-scoring
-    // recomputes the double-float value from V), ||u_j||^2 held by lane j
+    // recomputes the double-float value from V); ||u_j||^2, held by lane j, only
+    // where a budget restricts the pool (E < n - k)
+    bool need_e2 = false;
+    for (int b = 0; b < nb; ++b) need_e2 |= a.E < n - a.k[row * nb + b];
     double e2 = 0.0;
     for (int j = 0; j < n; ++j) {
         const df pj = shfl_df(pd, j);
@@ -226,10 +229,12 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
             const int c = lane + 32 * t;
             const df u = df_mul(pj, df_rsub_f(Uhi[j * (d + 1) + c], mu[t]));
             Uhi[j * (d + 1) + c] = u.hi;
-            s = df_add(s, df_mul(u, u));
+            if (need_e2) s = df_add(s, df_mul(u, u));
         }
-        s = warp_sum_df(s);
-        if (lane == j) e2 = df_to_double(s);
+        if (need_e2) {
+            s = warp_sum_df(s);
+            if (lane == j) e2 = df_to_double(s);
+        }
     }
     __syncwarp();
     // fp32 Gram matrix, four interleaved partial sums per dot product
