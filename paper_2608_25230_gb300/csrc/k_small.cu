@@ -104,7 +104,7 @@ __global__ void __launch_bounds__(256) k_small_gap(const SmallGapArgs a)
     }
     if (a.out.o) {
 #pragma unroll
-        for (int t = 0; t < DPL; ++t) a.out.o[row * d + lane + 32 * t] = (float)df_to_double(mu[t]);
+        for (int t = 0; t < DPL; ++t) a.out.o[row * d + lane + 32 * t] = mu[t].hi + mu[t].lo;  // rounded once
     }
 #pragma unroll
     for (int b = 0; b < 4; ++b) {
@@ -123,11 +123,13 @@ __global__ void __launch_bounds__(256) k_small_gap(const SmallGapArgs a)
             a.out.dropped[rb] = (float)PD;
             if (a.out.phi) a.out.phi[rb] = (float)phi;
         }
-        if (a.out.o_kept) {
+        if (a.out.o_kept) {  // mu + g_A / P(A) in double-float, rounded once
+            const df invP = df_from_double(1.0 / PA);
 #pragma unroll
-            for (int t = 0; t < DPL; ++t)
-                a.out.o_kept[rb * d + lane + 32 * t] =
-                    (float)(df_to_double(mu[t]) + df_to_double(gA[b][t]) / PA);
+            for (int t = 0; t < DPL; ++t) {
+                const df ok = df_add(mu[t], df_mul(gA[b][t], invP));
+                a.out.o_kept[rb * d + lane + 32 * t] = ok.hi + ok.lo;
+            }
         }
     }
     if (lane == 0) {
@@ -304,7 +306,11 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
             }
             S = warp_sum(inp && cnt <= kb ? unorm : 0.f) * 1.0001f;
         }
+        // bound on the fp32 error of a screened score, times P(A - i + j)^2: the
+        // Gram entries and sums (CB S^2), and 8 ulps of Q <= S^2 for the rounded
+        // P(A - i + j) and its inverse square
         const float CB = 2.0f * ((float)d * 0.25f + 2.0f * (float)kb + 12.0f) * 5.9604645e-8f;
+        const float CBS = (CB + 8.f * 5.9604645e-8f) * S * S;
         // u_j in double-float, recomputed from V (the expression of the pass above)
         auto u_df = [&](int j, int t) {
             return df_mul(shfl_df(pd, j), df_rsub_f(load_v(V, (int64_t)j * d + lane + 32 * t), mu[t]));
@@ -340,45 +346,35 @@ __global__ void __launch_bounds__(64) k_small_swap(const SmallSwapArgs a)
             if (lane < n)
                 for (uint32_t m = A; m; m &= m - 1) h += G[lane * 33 + __ffs(m) - 1];
             const float QA = warp_sum(((A >> lane) & 1u) ? h : 0.f);
-            // fp32 screening of every (kept i, added j) pair:
-            // Q(A - i + j) = Q_A - 2 h_i + G_ii + 2 h_j - 2 G_ij + G_jj
-            const int np = na * nadd;  // <= 256
-            float sc[8], bd[8];
-            int pi_[8], pj_[8];
+            // fp32 screening of every (kept i, added j) pair, lane j taking the
+            // added key j: Q(A - i + j) = (Q_A - 2 h_i + G_ii) + (2 h_j + G_jj) - 2 G_ij,
+            // P(A - i + j) = P(A - i) + p_j (two positive terms)
+            const bool isadd = (add >> lane) & 1u;
+            const float cj = lane < n ? 2.f * h + G[lane * 33 + lane] : 0.f;
+            const float pjf = (float)p;
             float best_up = INFINITY;
-#pragma unroll
-            for (int s8 = 0; s8 < 8; ++s8) {
-                const int q = lane + 32 * s8;
-                const bool valid = q < np;
-                const int qq = valid ? q : 0;
-                const int i = __fns(A, 0, qq / nadd + 1);
-                const int j = __fns(add, 0, qq % nadd + 1);
-                const float hi = __shfl_sync(FW_FULL, h, i);
-                const float hj = __shfl_sync(FW_FULL, h, j);
-                const double ppi = __shfl_sync(FW_FULL, p, i);
-                const double ppj = __shfl_sync(FW_FULL, p, j);
-                const float Qp = QA - 2.f * hi + G[i * 33 + i] + 2.f * hj - 2.f * G[i * 33 + j] +
-                                 G[j * 33 + j];
-                const float Pp = (float)(PA - ppi + ppj);
+            for (uint32_t mi = A; mi; mi &= mi - 1) {
+                const int i = __ffs(mi) - 1;
+                const float ci = QA - 2.f * __shfl_sync(FW_FULL, h, i) + G[i * 33 + i];
+                const float Pp = (float)(PA - __shfl_sync(FW_FULL, p, i)) + pjf;
                 const float inv = 1.f / (Pp * Pp);
-                sc[s8] = valid ? Qp * inv : INFINITY;
-                bd[s8] = CB * S * S * inv;
-                pi_[s8] = i;
-                pj_[s8] = j;
-                if (valid) best_up = fminf(best_up, sc[s8] + bd[s8]);
+                const float sc = (ci + cj - 2.f * G[i * 33 + (lane < n ? lane : 0)]) * inv;
+                if (isadd) best_up = fminf(best_up, sc + CBS * inv);
             }
             best_up = warp_min(best_up);
             // exact re-scoring, in (i, j) order, of every pair that may be the best
             double best = INFINITY;
             int bi = -1, bj = -1;
-#pragma unroll
-            for (int s8 = 0; s8 < 8; ++s8) {
-                uint32_t cand = __ballot_sync(FW_FULL, sc[s8] - bd[s8] <= best_up);
+            for (uint32_t mi = A; mi; mi &= mi - 1) {
+                const int i = __ffs(mi) - 1;
+                const float ci = QA - 2.f * __shfl_sync(FW_FULL, h, i) + G[i * 33 + i];
+                const float Pp = (float)(PA - __shfl_sync(FW_FULL, p, i)) + pjf;
+                const float inv = 1.f / (Pp * Pp);
+                const float sc = (ci + cj - 2.f * G[i * 33 + (lane < n ? lane : 0)]) * inv;
+                uint32_t cand = __ballot_sync(FW_FULL, isadd && sc - CBS * inv <= best_up);
                 while (cand) {
-                    const int src = __ffs(cand) - 1;
+                    const int j = __ffs(cand) - 1;
                     cand &= cand - 1;
-                    const int i = __shfl_sync(FW_FULL, pi_[s8], src);
-                    const int j = __shfl_sync(FW_FULL, pj_[s8], src);
                     df gn[DPL];
 #pragma unroll
                     for (int t = 0; t < DPL; ++t) {
