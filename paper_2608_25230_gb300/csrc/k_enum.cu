@@ -35,7 +35,7 @@ namespace {
 
 constexpr int EM = 12;    // inner key set size
 constexpr int ECAP = 32;  // candidate masks per row
-constexpr int FBS = 16;   // chunks (blocks) per row on the exhaustive path
+constexpr int FBS = 64;   // chunks (blocks) per row on the exhaustive path
 constexpr int MAXD = 24;  // depth bound of the phase-2 walk
 constexpr int PERM = 48;  // local index space per row: NS <= EM + 32
 
@@ -532,8 +532,8 @@ __global__ void __launch_bounds__(32 * PREP_W, 4) k_enum_prep(const EnumArgs a)
     float *slot = smem + (size_t)wib * prep_floats(a.stride, ust_floats);  // [stride]
     float *Ust = slot + (a.stride + 1) / 2 * 2;                             // [max_n+1][DCH+1]
     float *aX = Ust + ust_floats;                                            // [32]
-    double *pscr = reinterpret_cast<double *>(aX + 32);                      // [32]
-    uint8_t *perms = reinterpret_cast<uint8_t *>(pscr + 32);                 // [PERM]
+    float *pfl = aX + 32;                                                    // [32] p (rounded)
+    uint8_t *perms = reinterpret_cast<uint8_t *>(aX + 96);                   // [PERM]
     uint8_t *inv = perms + PERM;                                             // [32]
     const int64_t row = (int64_t)blockIdx.x * PREP_W + wib;
     if (row >= a.R.rows) return;
@@ -580,7 +580,7 @@ __global__ void __launch_bounds__(32 * PREP_W, 4) k_enum_prep(const EnumArgs a)
         const int loc = inA0 ? EM + bi : (bo < nL ? bo : EM + k + (bo - nL));
         perm[loc] = (uint8_t)lane;
         inv[lane] = (uint8_t)loc;
-        pscr[lane] = p;
+        pfl[lane] = (float)p;
     }
     SlotGeom S;
     S.slot = slot;
@@ -708,7 +708,7 @@ __global__ void __launch_bounds__(32 * PREP_W, 4) k_enum_prep(const EnumArgs a)
 #pragma unroll
     for (int i = 0; i < PPL; ++i)
         if (px_[i] >= 0 && px_[i] == py_[i] && px_[i] < n)
-            aX[px_[i]] = sqrtf(fmaxf(acc[i], 0.f)) * 1.0001f + (float)(sqt * pscr[px_[i]]) * 1.0001f;
+            aX[px_[i]] = sqrtf(fmaxf(acc[i], 0.f)) * 1.0001f + ((float)sqt * pfl[px_[i]]) * 1.0001f;
     __syncwarp();
     // scatter the folded entries into the walk tables
     const float tf = (float)t, P0f = (float)P0;
@@ -717,12 +717,12 @@ __global__ void __launch_bounds__(32 * PREP_W, 4) k_enum_prep(const EnumArgs a)
         const int x = px_[i], y = py_[i];
         if (x < 0 || x == n) continue;
         // G' = u.u - t p p^T in fp32 (a few ulps of a_x a_y, inside kappa's slack)
-        const float tpx = tf * (float)pscr[x];
+        const float tpx = tf * pfl[x];
         if (y == n) {
             const float sx = ((A0 >> x) & 1u) ? -2.f : 2.f;
             put_linear(S, inv[x], sx * fmaf(-tpx, P0f, acc[i]), aX[x]);
         } else {
-            const float gp = fmaf(-tpx, (float)pscr[y], acc[i]);
+            const float gp = fmaf(-tpx, pfl[y], acc[i]);
             if (x == y) {
                 put_diag(S, inv[x], gp, aX[x]);
             } else {
@@ -1040,14 +1040,15 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
         __syncthreads();
         const double t = s_t, P0 = s_P0;
         const uint32_t A0 = s_A0;
-        for (int q = tid; q < n * n; q += blockDim.x) {
+        for (int q = tid; q < n * n; q += blockDim.x) {  // x <= y, mirrored (exactly symmetric)
             const int x = q / n, y = q % n;
+            if (y < x) continue;
             const double sx = ((A0 >> x) & 1u) ? -1.0 : 1.0, sy = ((A0 >> y) & 1u) ? -1.0 : 1.0;
             double m = sx * sy * (Gs[x][y] - t * ps[x] * ps[y]);
             if (x == y) m += 2.0 * sx * (Gs[x][n] - t * P0 * ps[x]);
-            Ms[x][y] = m;
-            Mf[x][y] = (float)(x == y ? m : 2.0 * m);
-            if (y == 0) pf[x] = (float)ps[x];
+            Ms[x][y] = Ms[y][x] = m;
+            Mf[x][y] = Mf[y][x] = (float)(x == y ? m : 2.0 * m);
+            if (y == x) pf[x] = (float)ps[x];
         }
         __syncthreads();
         const uint64_t total = binom64(n, k);
@@ -1075,37 +1076,19 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
             ++cmb[i];
             for (int q2 = 0; q2 < i; ++q2) cmb[q2] = q2;
         };
-        auto mask_of = [&](const int *cmb) {
-            uint32_t am = 0u;
-            for (int i = 0; i < k; ++i) am |= 1u << cmb[i];
-            return am;
-        };
         // fp32 value of es^2 in the difference form with a rigorous bound on
         // its error: the fp32 entries are the fp64 ones rounded (relative error
-        // u), the sum of N terms adds at most N u times the sum of their
-        // magnitudes, P(A) sums k positive terms, and the reciprocal, products
-        // and the final sum add a few u more (plus the denormal floor per term)
+        // u), a sum over N terms in any order adds at most N u times the sum of
+        // their magnitudes, P(A) sums k positive terms, and the reciprocal,
+        // products and the final sum add a few u more (plus the denormal floor
+        // per term)
         const float tf = (float)t;
-        auto screen = [&](uint32_t am, float &elo, float &ehi) {
-            const uint32_t S = am ^ A0;
-            float val = 0.f, ab = 0.f;
-            for (uint32_t m1 = S; m1; m1 &= m1 - 1) {
-                const int x = __ffs(m1) - 1;
-                for (uint32_t m2 = m1; m2; m2 &= m2 - 1) {
-                    const float v = Mf[x][__ffs(m2) - 1];
-                    val += v;
-                    ab += fabsf(v);
-                }
-            }
-            float P = 0.f;
-            for (uint32_t m1 = am; m1; m1 &= m1 - 1) P += pf[__ffs(m1) - 1];
+        auto bound = [&](float val, float ab, float P, float N, float &elo, float &ehi) {
             if (!(P > 1e-17f)) {
                 elo = -INFINITY;
                 ehi = INFINITY;
                 return;
             }
-            const int sz = __popc(S);
-            const float N = (float)(sz * (sz + 1) / 2);
             const float u = 5.9604645e-8f;
             const float inv = __frcp_rn(P * P);
             const float e = tf + val * inv;
@@ -1120,18 +1103,58 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
             elo = e - err;
             ehi = e + err;
         };
-        // pass 1: the smallest upper bound over the chunk
-        float ub = INFINITY;
-        int cmb[32];
-        if (lo < hi) {
+        // The chunk's ranks in colex order.  Consecutive ranks mostly differ in
+        // the lowest member z only, so for each set of the other k - 1 members
+        // ("rest") the part over S_r = rest xor A0 is summed once, and each z
+        // adds (z not in A0) or removes (z in A0, hence in S_r) its own row:
+        // val(S_r xor {z}) = val(S_r) +- (M'_zz + sum_{y in S_r, y != z} M'_zy),
+        // M' = Mf (off-diagonal entries doubled).  f(mask, rank, val, sum of
+        // |terms|, P, number of terms).
+        auto visit = [&](auto &&f) {
+            if (lo >= hi) return;
+            int cmb[32];
             unrank(lo, cmb);
-            for (uint64_t rk = lo; rk < hi; ++rk) {
-                float elo, ehi;
-                screen(mask_of(cmb), elo, ehi);
-                ub = fminf(ub, fmaxf(ehi, 0.f));
+            uint64_t rk = lo;
+            for (;;) {
+                uint32_t rest = 0u;
+                for (int i = 1; i < k; ++i) rest |= 1u << cmb[i];
+                const uint32_t Sr = rest ^ A0;
+                float vr = 0.f, ar = 0.f, Pr = 0.f;
+                for (uint32_t m1 = Sr; m1; m1 &= m1 - 1) {
+                    const int x = __ffs(m1) - 1;
+                    for (uint32_t m2 = m1; m2; m2 &= m2 - 1) {
+                        const float v = Mf[x][__ffs(m2) - 1];
+                        vr += v;
+                        ar += fabsf(v);
+                    }
+                }
+                for (uint32_t m1 = rest; m1; m1 &= m1 - 1) Pr += pf[__ffs(m1) - 1];
+                const int sr = __popc(Sr);
+                const float Nr = (float)(sr * (sr + 1) / 2 + sr + 1);
+                const int zmax = k > 1 ? cmb[1] : n;
+                for (int z = cmb[0]; z < zmax; ++z) {
+                    float r2 = Mf[z][z], a2 = fabsf(r2);
+                    for (uint32_t m1 = Sr & ~(1u << z); m1; m1 &= m1 - 1) {
+                        const float v = Mf[z][__ffs(m1) - 1];
+                        r2 += v;
+                        a2 += fabsf(v);
+                    }
+                    const float val = ((A0 >> z) & 1u) ? vr - r2 : vr + r2;
+                    f(rest | (1u << z), rk, val, ar + a2, Pr + pf[z], Nr);
+                    if (++rk >= hi) return;
+                }
+                if (k == 1) return;  // (all n ranks visited)
+                cmb[0] = zmax - 1;   // the run of z is over: next rest
                 succ(cmb);
             }
-        }
+        };
+        // pass 1: the smallest upper bound over the chunk
+        float ub = INFINITY;
+        visit([&](uint32_t, uint64_t, float val, float ab, float P, float N) {
+            float elo, ehi;
+            bound(val, ab, P, N, elo, ehi);
+            ub = fminf(ub, fmaxf(ehi, 0.f));
+        });
         ured_f[tid] = ub;
         __syncthreads();
         for (int s = blockDim.x / 2; s > 0; s >>= 1) {
@@ -1142,30 +1165,24 @@ __global__ void __launch_bounds__(256) k_enum_exhaustive(const EnumArgs a)
         // pass 2: fp64 values of the subsets that may reach that bound
         double best = INFINITY;
         unsigned long long brank = ~0ull;
-        if (lo < hi) {
-            unrank(lo, cmb);
-            for (uint64_t rk = lo; rk < hi; ++rk) {
-                const uint32_t am = mask_of(cmb);
-                float elo, ehi;
-                screen(am, elo, ehi);
-                if (elo <= ub) {
-                    const uint32_t S = am ^ A0;
-                    double val = 0.0, P = P0;
-                    for (uint32_t m1 = S; m1; m1 &= m1 - 1) {
-                        const int x = __ffs(m1) - 1;
-                        P += ((A0 >> x) & 1u) ? -ps[x] : ps[x];
-                        val += Ms[x][x];
-                        for (uint32_t m2 = m1 & (m1 - 1); m2; m2 &= m2 - 1) val += 2.0 * Ms[x][__ffs(m2) - 1];
-                    }
-                    const double e = fmax(t + val / (P * P), 0.0);
-                    if (e < best) {
-                        best = e;
-                        brank = rk;
-                    }
-                }
-                succ(cmb);
+        visit([&](uint32_t am, uint64_t rk, float val, float ab, float P, float N) {
+            float elo, ehi;
+            bound(val, ab, P, N, elo, ehi);
+            if (!(elo <= ub)) return;
+            const uint32_t S = am ^ A0;
+            double dv = 0.0, Pd = P0;
+            for (uint32_t m1 = S; m1; m1 &= m1 - 1) {
+                const int x = __ffs(m1) - 1;
+                Pd += ((A0 >> x) & 1u) ? -ps[x] : ps[x];
+                dv += Ms[x][x];
+                for (uint32_t m2 = m1 & (m1 - 1); m2; m2 &= m2 - 1) dv += 2.0 * Ms[x][__ffs(m2) - 1];
             }
-        }
+            const double e = fmax(t + dv / (Pd * Pd), 0.0);
+            if (e < best) {
+                best = e;
+                brank = rk;
+            }
+        });
         ured_e[tid] = best;
         ured_r[tid] = brank;
         __syncthreads();
