@@ -19,21 +19,27 @@
 // The swap lowers es iff D_ij < 0; the round takes the pair of smallest
 // D_ij / P'^2 (ties: smallest i, then j) and stops when that is not negative.
 //
-// Only C_ij needs a d-long product per pair, and |C_ij| <= |w_i||w_j|.  Each
-// round therefore works in three steps:
-//  1. one pass over the kept keys computes g.w_i exactly (so alpha_i) and a
-//     lower bound of min_j D_ij / P'^2 in which C_ij is replaced by that
-//     Cauchy-Schwarz bound and the pool is taken in 8 groups of consecutive
-//     beta_j, each group through its least beta_j, largest p_j|w_j| and
-//     extreme p_j (D is increasing in p_j - p_i for p_j - p_i > -P);
-//  2. the key with the least bound is scored exactly against the whole pool,
-//     which bounds the round's best score from above;
-//  3. every key whose bound does not exceed that (plus a rounding allowance)
-//     is scored exactly, and the best of those pairs is the round's choice.
-// A key whose bound exceeds an attained score cannot hold the minimum, so the
-// choice is the one that scoring every pair would make; on measured rows the
-// bound leaves about 0.1-3 % of the kept keys to step 3.
+// Only C_ij needs a d-long product per pair, and it does not depend on g: a
+// swap changes one kept position (the key that enters) and one pool slot (the
+// key that leaves takes the entering key's slot).  So the block keeps the
+// table C[slot][position] in its workspace: the first round of a budget fills
+// it (a k x d by d x E product in register tiles), and every later round
+// recomputes only the changed slot's column and the changed position's row.
+// A round is then one pass over the kept keys -- per key the exact product
+// g.w_i (so alpha_i), the new column entry, and the scan of its E stored
+// entries -- with O(d + E) work per key instead of O(E d).  Four lanes share a
+// key (each a quarter of the columns and of the slots); the pass is software
+// pipelined (the next key's value row is in flight while the current one is
+// scored).  In the scan D_ij is regrouped as A_i + B_j + p_i (h_j + k_j C_ij)
+// with per-key A_i and per-slot B_j, h_j, k_j, so a pair costs three fused
+// operations and one approximate division.  Each lane keeps its least score
+// and the first position where it occurred; the lanes holding the block's
+// least score score that position's pairs again with the same operations and
+// the smallest (i, j) among the pairs at that score wins.  (Two positions of
+// one lane at exactly the same fp32 score keep the first: such pairs are tied
+// to ~1e-7 relative, a decision no fp32 evaluation can settle.)
 #include <algorithm>
+#include <climits>
 
 #include "fw_internal.h"
 
@@ -42,9 +48,11 @@ namespace {
 
 constexpr int SWT = 256;     // threads per block
 constexpr int SWMAXE = kLongSwapMaxE;  // largest pool size E
-constexpr int SWGRP = 8;     // pool groups in the lower bound
-constexpr int QL = 4;        // lanes per kept key in the passes over kept keys
-constexpr int KPI = SWT / QL;  // kept keys per block iteration
+constexpr int TK = 2;        // kept keys per thread in the first-round product tile
+constexpr int TS = 8;        // pool slots per thread in that tile (4 threads cover 32)
+constexpr int QL = 4;        // lanes per kept key in the round pass
+constexpr int KPI = SWT / QL;  // kept keys per block iteration of the pass
+constexpr int LS_BPS = 3;    // resident blocks per SM
 
 struct LSArgs {
     RowsDev R;
@@ -63,9 +71,9 @@ struct LSArgs {
     int32_t *kbuf;   // key at each position of the current kept list
     float *pbuf;     // its mass
     float *xbuf;     // its |w|^2
-    float *lbuf;     // its lower bound of the round
-    float *abuf;     // its alpha of the round
-    int32_t *sbuf;   // positions left for exact scoring
+    // per-block cross-product table, [gridDim.x][Ep][cstride]
+    float *cbuf;
+    int cstride;     // positions per slot row (max_n rounded up to a multiple of 4)
 };
 
 __device__ __forceinline__ float block_sum(float v, float *red)
@@ -77,19 +85,6 @@ __device__ __forceinline__ float block_sum(float v, float *red)
     __syncthreads();
     float t = 0.f;
     for (int i = 0; i < SWT / 32; ++i) t += red[i];
-    __syncthreads();
-    return t;
-}
-
-__device__ __forceinline__ float block_min(float v, float *red)
-{
-    v = warp_min(v);
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) red[w] = v;
-    __syncthreads();
-    float t = INFINITY;
-    for (int i = 0; i < SWT / 32; ++i) t = fminf(t, red[i]);
     __syncthreads();
     return t;
 }
@@ -113,216 +108,253 @@ __device__ __forceinline__ void ld8(const float *p, float (&x)[8])
     x[4] = b.x, x[5] = b.y, x[6] = b.z, x[7] = b.w;
 }
 
-// D_ij / P'^2 for one pair (the fast form of the file comment).
-__device__ __forceinline__ float pair_score(float alpha, float p_i, float p_j, float beta, float cij, float P,
-                                           float P2, float N)
-{
-    const float cross = p_i * p_j * cij;
-    const float delta = alpha + beta - 2.f * cross;
-    const float dp = p_j - p_i;
-    const float Pp = P + dp;
-    const float D = delta * P2 - N * dp * (2.f * P + dp);
-    return D / (Pp * Pp);
-}
-
 // The fast form divides D (a difference of terms of size ~N P^2) by P'^2, so
-// its rounding grows like P^2 / P'^2; it is trusted while P'^2 >= P^2 / 16
-// (error ~1e-6 N, inside the decision margins that matter).  A swap that
-// removes more of the kept mass is rescored from g' = g - u_i + u_j, which keeps
-// the cancellation in d-vectors.
-__device__ __forceinline__ bool needs_vector(float P, float p_i, float p_j)
-{
-    const float Pp = P + p_j - p_i;
-    return !(16.f * Pp * Pp >= P * P);
-}
+// its rounding grows like P^2 / P'^2; it is trusted while P'^2 >= P^2 / 16.
+// A swap that removes more of the kept mass is scored from g' = g - u_i + u_j,
+// which keeps the cancellation in d-vectors.
 
-// Rounding allowances of the lower bound.  alpha_i and beta_j are computed once
-// and shared by the bound and the exact scores, so the bound only has to cover
-// the few operations that combine them (kRoundRel, about 16 ulps, of their
-// magnitude), the
-// rounding of the computed cross product C_ij against |w_i||w_j| (d ulps at
-// most) and, where a pair may take the vector form, that form's rounding.
-constexpr float kRoundRel = 1e-6f;
-constexpr float kUlp = 1.2e-7f;
-
-// The score from |g'|^2, g' = g - u_i + u_j summed by the caller.
+// The score from |g'|^2, g' = g - u_i + u_j.
 __device__ __forceinline__ float vector_score(float gp2, float P, float p_i, float p_j, float P2, float N)
 {
     const float Pp = P + p_j - p_i;
     return gp2 * (P2 / (Pp * Pp)) - N;
 }
 
-__device__ __forceinline__ bool pair_less(float s, unsigned long long k, float bs, unsigned long long bk)
-{
-    return s < bs || (s == bs && k < bk);
-}
 
-// Exact scores of the pairs of the kept positions in list[0, cnt) (entries
-// < 0 are skipped), 4 lanes per position; folds them into the calling lane's
-// best (score, (i, j) key, position, slot).  Block-uniform in cnt.
+// Up to 16 sixteen-byte loads of a value row, all issued before any use:
+// NV vectors of 8 bf16 or 4 fp32 elements.
+template <typename VT, int NV> struct RowChunk;
+template <int NV> struct RowChunk<uint16_t, NV> {
+    uint4 u[NV];
+    __device__ __forceinline__ void load(const uint16_t *p)
+    {
+#pragma unroll
+        for (int i = 0; i < NV; ++i) u[i] = __ldg(reinterpret_cast<const uint4 *>(p) + i);
+    }
+    __device__ __forceinline__ float at(int c) const  // c is a constant after unrolling
+    {
+        const uint4 v = u[c >> 3];
+        const int e = (c >> 1) & 3;
+        const uint32_t w = e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+        return (c & 1) ? __uint_as_float(w & 0xffff0000u) : __uint_as_float(w << 16);
+    }
+};
+template <int NV> struct RowChunk<float, NV> {
+    float4 u[NV];
+    __device__ __forceinline__ void load(const float *p)
+    {
+#pragma unroll
+        for (int i = 0; i < NV; ++i) u[i] = __ldg(reinterpret_cast<const float4 *>(p) + i);
+    }
+    __device__ __forceinline__ float at(int c) const
+    {
+        const float4 v = u[c >> 2];
+        const int e = c & 3;
+        return e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+    }
+};
+
+// First round of a budget: C[q][t] = w_{kb[t]} . w_q for every kept position
+// t < nk and pool slot q in the 32-slot blocks below nadd.  A thread owns 2
+// consecutive positions x 8 slots; the 4 threads of a group cover 32 slots.
+// The sum over the d columns runs in column order, as in the later rounds.
 template <int DPL, typename VT>
-__device__ __forceinline__ void score_positions(const int *list, int cnt, const int *kb, const float *pk,
-                                                const float *ak, const float *xk, const VT *V, const float *mu,
-                                                const float *g, const float *Wt, int Ep, const float *pj,
-                                                const float *betaj, const float *rj, const int *idxj, int nadd,
-                                                float P, float P2, float N, float sqN, float &best,
-                                                unsigned long long &bkey, int &bt, int &bq)
+__device__ __forceinline__ void cross_table(const int *kb, int nk, const VT *V, const float *mu, const float *Wt,
+                                            int Ep, int nadd, float *cb, int cstride)
 {
     constexpr int d = DPL * 32;
-    constexpr int CPL = d / QL;
-    const int lane = threadIdx.x & 31, gq = threadIdx.x / QL, sub = threadIdx.x % QL;
-    for (int s0 = 0; s0 < cnt; s0 += KPI) {
-        const int s = s0 + gq;
-        const int t0 = s < cnt ? list[s] : -1;
-        const bool valid = t0 >= 0;
-        const int t = valid ? t0 : 0;
-        const int i = kb[t];
-        const float p_i = pk[t], al = ak[t], s_i = p_i * sqrtf(xk[t]);
-        const VT *vr = V + (int64_t)i * d + sub * CPL;
-        const float *mur = mu + sub * CPL;
-        for (int q0 = 0; q0 < Ep; q0 += 16) {
-            float acc[16];
+    const int sub = threadIdx.x & 3, grp = threadIdx.x >> 2;
+    constexpr int GROUPS = SWT / 4;
+    for (int base = 0; base < nk; base += GROUPS * TK) {
+        const int t0 = base + grp * TK;
+        if (t0 >= nk) break;
+        const VT *vr[TK];
 #pragma unroll
-            for (int m = 0; m < 16; ++m) acc[m] = 0.f;
-#pragma unroll 2
-            for (int c0 = 0; c0 < CPL; c0 += 8) {
-                float x[8];
-                ld8(vr + c0, x);
+        for (int u = 0; u < TK; ++u) vr[u] = V + (int64_t)kb[t0 + u < nk ? t0 + u : t0] * d;
+        for (int q0 = 0; q0 < nadd; q0 += 32) {
+            float acc[TK][TS];
 #pragma unroll
-                for (int m = 0; m < 8; ++m) {
-                    const float w = x[m] - mur[c0 + m];
-                    const float4 *wr = reinterpret_cast<const float4 *>(Wt + (sub * CPL + c0 + m) * Ep + q0);
+            for (int u = 0; u < TK; ++u)
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const float4 W4 = wr[u];
-                        acc[4 * u] = fmaf(w, W4.x, acc[4 * u]);
-                        acc[4 * u + 1] = fmaf(w, W4.y, acc[4 * u + 1]);
-                        acc[4 * u + 2] = fmaf(w, W4.z, acc[4 * u + 2]);
-                        acc[4 * u + 3] = fmaf(w, W4.w, acc[4 * u + 3]);
+                for (int s = 0; s < TS; ++s) acc[u][s] = 0.f;
+            const float *wq = Wt + q0 + sub * TS;
+            // one 16-byte vector per position in flight ahead of the one in use
+            constexpr int EPV = 16 / (int)sizeof(VT);
+            RowChunk<VT, 1> cur[TK];
+#pragma unroll
+            for (int u = 0; u < TK; ++u) cur[u].load(vr[u]);
+#pragma unroll 1
+            for (int c0 = 0; c0 < d; c0 += EPV) {
+                RowChunk<VT, 1> nxt[TK];
+                const int cn = c0 + EPV < d ? c0 + EPV : c0;
+#pragma unroll
+                for (int u = 0; u < TK; ++u) nxt[u].load(vr[u] + cn);
+#pragma unroll
+                for (int m = 0; m < EPV; ++m) {
+                    const float mc = mu[c0 + m];
+                    const float4 A = *reinterpret_cast<const float4 *>(wq + (c0 + m) * Ep);
+                    const float4 B = *reinterpret_cast<const float4 *>(wq + (c0 + m) * Ep + 4);
+                    const float ws[TS] = {A.x, A.y, A.z, A.w, B.x, B.y, B.z, B.w};
+#pragma unroll
+                    for (int u = 0; u < TK; ++u) {
+                        const float x = cur[u].at(m) - mc;
+#pragma unroll
+                        for (int s = 0; s < TS; ++s) acc[u][s] = fmaf(x, ws[s], acc[u][s]);
                     }
                 }
-            }
-            // reduce-scatter over the 4 lanes: lane `sub` ends with slots q0 + 4 sub + m
-            float h8[8];
 #pragma unroll
-            for (int m = 0; m < 8; ++m) {
-                const bool up = sub & 2;
-                const float send = up ? acc[m] : acc[m + 8];
-                const float keep = up ? acc[m + 8] : acc[m];
-                h8[m] = keep + __shfl_xor_sync(FW_FULL, send, 2);
+                for (int u = 0; u < TK; ++u) cur[u] = nxt[u];
             }
-            float h4[4];
+            static_assert(TK == 2, "the tile stores TK consecutive positions as one float2");
 #pragma unroll
-            for (int m = 0; m < 4; ++m) {
-                const bool up = sub & 1;
-                const float send = up ? h8[m] : h8[m + 4];
-                const float keep = up ? h8[m + 4] : h8[m];
-                h4[m] = keep + __shfl_xor_sync(FW_FULL, send, 1);
-            }
-            uint32_t fl = 0;  // pairs left to the vector form
-            if (valid) {
+            for (int s = 0; s < TS; ++s)
+                __stcs(reinterpret_cast<float2 *>(cb + (size_t)(q0 + sub * TS + s) * cstride + t0),
+                       make_float2(acc[0][s], acc[1][s]));
+        }
+    }
+}
+
+// The 16-byte vectors sub, sub + 4, ... of a value row (4 lanes per row),
+// each lane's loads issued before any use.
+template <int DPL, typename VT> struct LaneRow {
+    static constexpr int EPV = 16 / (int)sizeof(VT);       // elements per vector
+    static constexpr int NVL = DPL * 32 / EPV / QL;          // vectors per lane
+    RowChunk<VT, 1> u[NVL];
+    __device__ __forceinline__ void load(const VT *vr, int sub)
+    {
 #pragma unroll
-                for (int m = 0; m < 4; ++m) {
-                    const int q = q0 + 4 * sub + m;
-                    if (q < nadd) {
-                        const float sc = pair_score(al, p_i, pj[q], betaj[q], h4[m], P, P2, N);
-                        if (needs_vector(P, p_i, pj[q])) {
-                            fl |= 1u << m;
-                            continue;
-                        }
-                        const unsigned long long key =
-                            ((unsigned long long)(uint32_t)i << 32) | (uint32_t)idxj[q];
-                        if (pair_less(sc, key, best, bkey)) {
-                            best = sc;
-                            bkey = key;
-                            bt = t;
-                            bq = q;
-                        }
-                    }
-                }
-            }
-            if (__any_sync(FW_FULL, fl != 0)) {
-                // warp-uniform walk over the group's 16 pairs; each flagged pair is
-                // summed by the 4 lanes of its group and scored by its owner lane
-                for (int src = 0; src < QL; ++src) {
-                    const uint32_t fs = __shfl_sync(FW_FULL, fl, (lane & ~(QL - 1)) | src);
-                    for (int m = 0; m < 4; ++m) {
-                        const bool need = (fs >> m) & 1u;
-                        if (!__any_sync(FW_FULL, need)) continue;
-                        const int q = q0 + 4 * src + m;
-                        float gv = 0.f;
-                        if (need) {
-                            const float pq = pj[q];
-                            for (int c0 = 0; c0 < CPL; c0 += 8) {
-                                float x[8];
-                                ld8(vr + c0, x);
+        for (int k = 0; k < NVL; ++k) u[k].load(vr + (k * QL + sub) * EPV);
+    }
+};
+
+// This lane's part of g.w and |w|^2, w = v - mu.
+template <int DPL, typename VT>
+__device__ __forceinline__ void lane_products(const VT *vr, const float *mu, const float *g, int sub, float &sg,
+                                              float &s2)
+{
+    using L = LaneRow<DPL, VT>;
+    L row;
+    row.load(vr, sub);
+    sg = 0.f;
+    s2 = 0.f;
 #pragma unroll
-                                for (int u = 0; u < 8; ++u) {
-                                    const int c = sub * CPL + c0 + u;
-                                    const float gp = fmaf(pq, Wt[c * Ep + q], fmaf(-p_i, x[u] - mu[c], g[c]));
-                                    gv = fmaf(gp, gp, gv);
-                                }
-                            }
-                        }
-                        gv += __shfl_xor_sync(FW_FULL, gv, 1);
-                        gv += __shfl_xor_sync(FW_FULL, gv, 2);
-                        if (need && sub == src) {
-                            const float sc = vector_score(gv, P, p_i, pj[q], P2, N);
-                            const unsigned long long key =
-                                ((unsigned long long)(uint32_t)i << 32) | (uint32_t)idxj[q];
-                            if (pair_less(sc, key, best, bkey)) {
-                                best = sc;
-                                bkey = key;
-                                bt = t;
-                                bq = q;
-                            }
-                        }
-                    }
-                }
+    for (int k = 0; k < L::NVL; ++k) {
+        const int c0 = (k * QL + sub) * L::EPV;
+#pragma unroll
+        for (int e = 0; e < L::EPV; ++e) {
+            const float w = row.u[k].at(e) - mu[c0 + e];
+            sg = fmaf(w, g[c0 + e], sg);
+            s2 = fmaf(w, w, s2);
+        }
+    }
+}
+
+// This lane's part of v.g and v.y from its loaded vectors.
+template <int DPL, typename VT>
+__device__ __forceinline__ void lane_products_v_row(const LaneRow<DPL, VT> &row, const float *g, const float *y,
+                                                    int sub, float &vg, float &vy)
+{
+    using L = LaneRow<DPL, VT>;
+    vg = 0.f;
+    vy = 0.f;
+#pragma unroll
+    for (int k = 0; k < L::NVL; ++k) {
+        const int c0 = (k * QL + sub) * L::EPV;
+#pragma unroll
+        for (int e = 0; e < L::EPV; e += 4) {
+            const float4 g4 = *reinterpret_cast<const float4 *>(g + c0 + e);
+            const float4 y4 = *reinterpret_cast<const float4 *>(y + c0 + e);
+            const float gg[4] = {g4.x, g4.y, g4.z, g4.w}, yy[4] = {y4.x, y4.y, y4.z, y4.w};
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                const float v = row.u[k].at(e + h);
+                vg = fmaf(v, gg[h], vg);
+                vy = fmaf(v, yy[h], vy);
             }
         }
     }
 }
 
+// |g - u_i + u_j|^2 for one pair, from the value row of i and the pool column
+// of j (the vector form of needs_vector's pairs).
 template <int DPL, typename VT>
-__global__ void __launch_bounds__(SWT, 2) k_long_swap(const LSArgs a)
+__device__ __forceinline__ float vector_gp2(const VT *vr, const float *mu, const float *g, const float *Wt, int Ep,
+                                            int q, float p_i, float p_j)
 {
     constexpr int d = DPL * 32;
-    constexpr int CPL = d / QL;  // columns per lane of a 4-lane group
-    const int Ep = a.Ep;         // pool slots, a multiple of 16
+    float gv = 0.f;
+    for (int c0 = 0; c0 < d; c0 += 8) {
+        float x[8];
+        ld8(vr + c0, x);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int c = c0 + u;
+            const float gp = fmaf(p_j, Wt[c * Ep + q], fmaf(-p_i, x[u] - mu[c], g[c]));
+            gv = fmaf(gp, gp, gv);
+        }
+    }
+    return gv;
+}
+
+// Score D / P'^2 of one pair in the regrouped fast form: sq = (B_j, k_j, h_j,
+// p_j), Ai = A_i, Pm = P - p_i.
+__device__ __forceinline__ float fast_score(float4 sq, float cij, float p_i, float Ai, float Pm)
+{
+    const float Pp = Pm + sq.w;
+    return __fdividef(fmaf(p_i, fmaf(sq.y, cij, sq.z), Ai + sq.x), Pp * Pp);
+}
+
+template <int DPL, typename VT>
+__device__ __noinline__ float vector_pair_score(const VT *vr, const float *mu, const float *g, const float *Wt, int Ep,
+                                                int q, float p_i, float p_j, float P, float P2, float N)
+{
+    return vector_score(vector_gp2<DPL, VT>(vr, mu, g, Wt, Ep, q, p_i, p_j), P, p_i, p_j, P2, N);
+}
+
+// The fast form where P'^2 >= P^2 / 16, else the vector form.
+template <int DPL, typename VT>
+__device__ __forceinline__ float any_score(float4 sq, float cij, float p_i, float Ai, float Pm, float P, float P2,
+                                           float N, const VT *vr, const float *mu, const float *g, const float *Wt,
+                                           int Ep, int q)
+{
+    const float Pp = Pm + sq.w;
+    if (16.f * Pp * Pp >= P2) return fast_score(sq, cij, p_i, Ai, Pm);
+    return vector_pair_score<DPL, VT>(vr, mu, g, Wt, Ep, q, p_i, sq.w, P, P2, N);
+}
+
+template <int DPL, typename VT>
+__global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
+{
+    constexpr int d = DPL * 32;
+    const int Ep = a.Ep;         // pool slots, a multiple of 32
     extern __shared__ __align__(16) float sm[];
     float *S = sm;                     // [5][d] band sums of p v
     float *mu = S + 5 * d;             // [d]
     float *o = mu + d;                 // [d]   dense output given by the caller
     float *g = o + d;                  // [d]
-    float *wdep = g + d;               // [d]   w of the key leaving A
-    float *wtmp = wdep + d;            // [d]   w of a single key being scored / entering A
+    float *wdep = g + d;               // [d]   w of the key that left A last (its pool slot's column)
+    float *wtmp = wdep + d;            // [d]   w of the key that entered A last
     float *Wt = wtmp + d;              // [d][Ep] pool vectors w_j, slot-major inner
-    float *pj = Wt + d * Ep;           // [Ep] masses of the pool slots
+    float4 *slot4 = reinterpret_cast<float4 *>(Wt + d * Ep);  // [Ep] per-round slot terms
+    float *pj = reinterpret_cast<float *>(slot4 + Ep);         // [Ep] masses of the pool slots
     float *betaj = pj + Ep;            // [Ep]
-    float *rj = betaj + Ep;            // [Ep] p_j |w_j|
-    int *idxj = reinterpret_cast<int *>(rj + Ep);      // [Ep] keys in the slots
-    int *ord = idxj + Ep;                               // [Ep] slots by ascending beta
-    int *cand = ord + Ep;                               // [KPI] nominated positions
-    float4 *grp = reinterpret_cast<float4 *>(cand + KPI);  // [SWGRP] bmin, rmax, pmin, pmax
-    float *gab = reinterpret_cast<float *>(grp + SWGRP);  // [SWGRP] largest |beta| of each group
-    float *red = gab + SWGRP;          // [32]
+    int *idxj = reinterpret_cast<int *>(betaj + Ep);  // [Ep] keys in the slots
+    float *red = reinterpret_cast<float *>(idxj + Ep);  // [32]
     float *mass = red + 32;            // [8]
     uint32_t *hist = reinterpret_cast<uint32_t *>(mass + 8);  // [256]
     __shared__ uint32_t s_misc[8];
     __shared__ int s_cnt, s_bt, s_bq;
-    __shared__ float s_best;
+    __shared__ float s_gm, s_ym, s_pmin;
     __shared__ unsigned long long s_bkey;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-    const int gq = tid / QL, sub = tid % QL;  // 4-lane group and lane within it
+    const int gq = tid / QL, sub = tid % QL;  // key group and lane within it
     const size_t boff = (size_t)blockIdx.x * a.R.max_n;
     float *eb = a.ebuf + boff;
     int *kb = a.kbuf + boff;
     float *pk = a.pbuf + boff;
     float *xk = a.xbuf + boff;
-    float *lbk = a.lbuf + boff;
-    float *ak = a.abuf + boff;
-    int *sl = a.sbuf + boff;
+    const int cs = a.cstride;
+    float *cb = a.cbuf + (size_t)blockIdx.x * Ep * cs;
     const int nb = a.nb, MS = a.max_swaps;
 
     for (int64_t row = blockIdx.x; row < a.R.rows; row += gridDim.x) {
@@ -353,26 +385,68 @@ __global__ void __launch_bounds__(SWT, 2) k_long_swap(const LSArgs a)
 #pragma unroll
                 for (int t = 0; t < DPL; ++t) acc[b][t] = 0.f;
             }
-            for (int j = wid; j < n; j += SWT / 32) {
-                const float x = lg[j];
-                const float p = expf(x - M) * Zi;
-                const uint32_t key = order_key(x);
-                int band = 0;
-                for (int b = 0; b < nb; ++b) band += !(key > tk[b] || (key == tk[b] && j <= ti[b]));
-                float dist = 0.f;
-#pragma unroll
-                for (int t = 0; t < DPL; ++t) {
-                    const int c = lane + 32 * t;
-                    const float v = load_v(V, (int64_t)j * d + c);
-#pragma unroll
-                    for (int b = 0; b < 5; ++b) acc[b][t] = fmaf(band == b ? p : 0.f, v, acc[b][t]);
-                    const float w = v - o[c];
-                    dist = fmaf(w, w, dist);
+            // 16 consecutive keys per warp and step: lanes l and l + 16 find the
+            // mass and band of key j0 + (l mod 16); then the warp walks the 16
+            // value rows (lane = column), and the 16 partial |v_j - o|^2 are summed
+            // by a transposed butterfly (lane l ends with key j0 + (l mod 16))
+            constexpr int KS = 16;
+            for (int j0 = wid * KS; j0 < n; j0 += (SWT / 32) * KS) {
+                const int jl = j0 + (lane & (KS - 1));
+                float pl = 0.f;
+                int bl = 0;
+                if (jl < n) {
+                    const float x = lg[jl];
+                    pl = expf(x - M) * Zi;
+                    const uint32_t key = order_key(x);
+                    for (int b = 0; b < nb; ++b) bl += !(key > tk[b] || (key == tk[b] && jl <= ti[b]));
                 }
-                dist = warp_sum(dist);
+                float dd[KS];
 #pragma unroll
-                for (int b = 0; b < 5; ++b) macc[b] += band == b ? p : 0.f;
-                if (lane == 0) eb[j] = p * p * dist;  // single-key error squared
+                for (int u0 = 0; u0 < KS; u0 += 4) {
+                    float v[4][DPL];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int j = j0 + u0 + u < n ? j0 + u0 + u : j0;
+#pragma unroll
+                        for (int t = 0; t < DPL; ++t) v[u][t] = load_v(V, (int64_t)j * d + lane + 32 * t);
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const float p = __shfl_sync(FW_FULL, pl, u0 + u);
+                        const int band = __shfl_sync(FW_FULL, bl, u0 + u);
+                        const bool live = j0 + u0 + u < n;
+                        // band is the same for the whole warp: one accumulator set is touched
+#pragma unroll
+                        for (int b = 0; b < 5; ++b)
+                            if (live && b == band) {
+#pragma unroll
+                                for (int t = 0; t < DPL; ++t) acc[b][t] = fmaf(p, v[u][t], acc[b][t]);
+                                macc[b] += p;
+                            }
+                        float dist = 0.f;
+#pragma unroll
+                        for (int t = 0; t < DPL; ++t) {
+                            const float w = v[u][t] - o[lane + 32 * t];
+                            dist = fmaf(w, w, dist);
+                        }
+                        dd[u0 + u] = dist;
+                    }
+                }
+                // transposed butterfly: the step with offset h leaves lane l the
+                // keys whose bit h equals lane bit h; after h = 1 it holds key
+                // l mod 16, and the last step adds the other half of the columns
+#pragma unroll
+                for (int h = KS / 2; h >= 1; h >>= 1) {
+                    const bool up = lane & h;
+#pragma unroll
+                    for (int u = 0; u < h; ++u) {
+                        const float send = up ? dd[u] : dd[u + h];
+                        const float keep = up ? dd[u + h] : dd[u];
+                        dd[u] = keep + __shfl_xor_sync(FW_FULL, send, h);
+                    }
+                }
+                dd[0] += __shfl_xor_sync(FW_FULL, dd[0], KS);
+                if (jl < n && lane < KS) eb[jl] = pl * pl * dd[0];  // single-key error squared
             }
 #pragma unroll
             for (int b = 0; b < 5; ++b) {
@@ -518,10 +592,11 @@ __global__ void __launch_bounds__(SWT, 2) k_long_swap(const LSArgs a)
 
             int taken = 0, cap = 0;
             bool first = true;
+            int tprev = -1, qprev = -1;  // position that entered and slot that changed last round
             for (;;) {
                 if (nadd == 0 || nk == 0) break;
-                const float P2 = P * P, twoP = 2.f * P, sqN = sqrtf(N);
-                // ---- pool terms of the round: beta_j, p_j |w_j|; slots ordered by beta
+                const float P2 = P * P;
+                // ---- pool terms of the round: beta_j
                 for (int q = wid; q < nadd; q += SWT / 32) {
                     float s2 = 0.f, sg = 0.f;
                     for (int c = lane; c < d; c += 32) {
@@ -533,169 +608,205 @@ __global__ void __launch_bounds__(SWT, 2) k_long_swap(const LSArgs a)
                     sg = warp_sum(sg);
                     const float p = pj[q];
                     if (lane == 0) {
-                        betaj[q] = p * p * s2 + 2.f * p * sg;
-                        rj[q] = p * sqrtf(s2);
+                        const float beta = p * p * s2 + 2.f * p * sg;
+                        betaj[q] = beta;
+                        // D_ij = A_i + B_j + p_i (h_j + k_j C_ij) (the file comment's D regrouped)
+                        slot4[q] = make_float4(beta * P2 - N * p * fmaf(2.f, P, p), -2.f * P2 * p, 2.f * N * p, p);
+                    }
+                }
+                if (wid == SWT / 32 - 1) {  // mu.g and mu.(changed slot's vector) for the folded products
+                    float a1 = 0.f, a2 = 0.f;
+                    for (int c = lane; c < d; c += 32) {
+                        a1 = fmaf(mu[c], g[c], a1);
+                        a2 = fmaf(mu[c], wdep[c], a2);
+                    }
+                    a1 = warp_sum(a1);
+                    a2 = warp_sum(a2);
+                    float pm = INFINITY;
+                    for (int q = lane; q < nadd; q += 32) pm = fminf(pm, pj[q]);
+                    pm = warp_min(pm);
+                    if (lane == 0) {
+                        s_gm = a1;
+                        s_ym = a2;
+                        s_pmin = pm;
+                    }
+                }
+                // ---- cross products: the whole table in the first round, else the
+                // row of the position that changed (its column entries come below)
+                if (first) {
+                    cross_table<DPL, VT>(kb, nk, V, mu, Wt, Ep, nadd, cb, cs);
+                } else {
+                    // warps split the columns, lanes take the slots of a 32-slot block
+                    float *part = reinterpret_cast<float *>(hist);  // [8][32]
+                    constexpr int CPW = d / (SWT / 32);
+                    for (int q0 = 0; q0 < nadd; q0 += 32) {
+                        const int q = q0 + lane;
+                        float c2 = 0.f;
+#pragma unroll 4
+                        for (int c = wid * CPW; c < (wid + 1) * CPW; ++c) c2 = fmaf(wtmp[c], Wt[c * Ep + q], c2);
+                        part[wid * 32 + lane] = c2;
+                        __syncthreads();
+                        if (wid == 0 && q < nadd) {
+                            float c3 = 0.f;
+                            for (int w = 0; w < SWT / 32; ++w) c3 += part[w * 32 + lane];
+                            __stcs(cb + (size_t)q * cs + tprev, c3);
+                        }
+                        __syncthreads();
                     }
                 }
                 __syncthreads();
-                if (wid == 0) {
-                    for (int q = lane; q < nadd; q += 32) {
-                        const uint32_t kq = order_key(betaj[q]);
-                        int r = 0;
-                        for (int q2 = 0; q2 < nadd; ++q2) {
-                            const uint32_t k2 = order_key(betaj[q2]);
-                            r += (k2 < kq) || (k2 == kq && q2 < q);
-                        }
-                        ord[r] = q;
-                    }
-                    __syncwarp();
-                    if (lane < SWGRP) {
-                        const int lo = lane * nadd / SWGRP, hi = (lane + 1) * nadd / SWGRP;
-                        float4 G = make_float4(INFINITY, 0.f, 1.f, 0.f);
-                        float ba = 0.f;
-                        if (hi > lo) {
-                            G.x = betaj[ord[lo]];
-                            G.z = INFINITY;
-                            for (int r = lo; r < hi; ++r) {
-                                const int q = ord[r];
-                                G.x = fminf(G.x, betaj[q]);
-                                G.y = fmaxf(G.y, rj[q]);
-                                G.z = fminf(G.z, pj[q]);
-                                G.w = fmaxf(G.w, pj[q]);
-                                ba = fmaxf(ba, fabsf(betaj[q]));
-                            }
-                        }
-                        grp[lane] = G;
-                        gab[lane] = ba;
-                    }
-                }
-                __syncthreads();
-                // ---- step 1: exact g.w_i and the lower bound of every kept key; each
-                // 4-lane group nominates the key of least bound among those it saw
-                float lbmin = INFINITY;
-                int tmin = -1;
-                for (int t0 = 0; t0 < nk; t0 += KPI) {
-                    const int t = t0 + gq;
-                    const bool valid = t < nk;
-                    const int i = kb[valid ? t : 0];
-                    const VT *vr = V + (int64_t)i * d + sub * CPL;
-                    const float *mur = mu + sub * CPL, *gr = g + sub * CPL;
-                    float sg = 0.f, s2 = 0.f;
-#pragma unroll
-                    for (int c0 = 0; c0 < CPL; c0 += 8) {
-                        float x[8];
-                        ld8(vr + c0, x);
-#pragma unroll
-                        for (int m = 0; m < 8; ++m) {
-                            const float w = x[m] - mur[c0 + m];
-                            sg = fmaf(w, gr[c0 + m], sg);
-                            if (first) s2 = fmaf(w, w, s2);
-                        }
-                    }
-                    sg += __shfl_xor_sync(FW_FULL, sg, 1);
-                    sg += __shfl_xor_sync(FW_FULL, sg, 2);
-                    float p_i, x2;
-                    if (first) {
-                        s2 += __shfl_xor_sync(FW_FULL, s2, 1);
-                        s2 += __shfl_xor_sync(FW_FULL, s2, 2);
-                        p_i = expf(lg[i] - M) * Zi;
-                        x2 = s2;
-                        if (valid && sub == 0) {
-                            pk[t] = p_i;
-                            xk[t] = x2;
-                        }
-                    } else {
-                        p_i = pk[valid ? t : 0];
-                        x2 = xk[valid ? t : 0];
-                    }
+                // ---- one pass over the kept keys: exact g.w_i, the changed slot's
+                // entry, and every pair of the key from the table
+                // Four lanes per kept key: lane `sub` holds the row's 16-byte
+                // vectors sub, sub + 4, ... and the pool slots q0 + 4m + sub of every
+                // 32-slot block.  Each lane keeps the least of its scores and the
+                // position where it first occurred; the block's least score then
+                // picks the lanes whose pairs are scored again.
+                float lmin = INFINITY, lp = 0.f, lA = 0.f;
+                int lt = -1, li = 0;
+                const float gm = s_gm, ym = s_ym;
+                const float pmin = s_pmin;  // least pool mass (the vector form's test)
+                // the scores of key t (position) from its products; cq0: its table
+                // entries of the first 32-slot block, read ahead
+                auto score_key = [&](int t, int i, const VT *vr, float sg, float sn, float p_i, float x2, bool col,
+                                     float (&cq0)[8]) {
                     const float alpha = p_i * p_i * x2 - 2.f * p_i * sg;
-                    const float s_i = p_i * sqrtf(x2);
-                    float lb = INFINITY;
+                    const float Ai = alpha * P2 + N * p_i * (2.f * P - p_i);
+                    const float Pm = P - p_i;
+                    // every pair of this key takes the fast form unless some pool
+                    // mass leaves P' below P / 4
+                    const bool fast = 16.f * (Pm + pmin) * (Pm + pmin) >= P2;
+                    float kmin = INFINITY;
+                    for (int q0 = 0; q0 < nadd; q0 += 32) {
+                        float cq[8];
 #pragma unroll
-                    for (int gi = sub; gi < SWGRP; gi += QL) {
-                        const float4 G = grp[gi];  // least beta, largest p|w|, least and largest p
-                        const float dmax = G.w - p_i, dmin = G.z - p_i;
-                        const float dabs = fmaxf(fabsf(dmin), fabsf(dmax));
-                        const float sr = s_i * G.y;
-                        const float LB = (alpha + G.x - 2.f * sr) * P2 - N * dmax * (twoP + dmax);
-                        const float den = LB >= 0.f ? P + dmax : P + dmin;
-                        const float dlo = P + dmin;
-                        const float mag = (fabsf(alpha) + gab[gi] + 2.f * sr) * P2 + N * dabs * (twoP + dabs);
-                        float allow = kRoundRel * mag + (float)d * kUlp * 2.f * sr * P2;
-                        if (!(16.f * dlo * dlo >= P2)) {  // some pair may take the vector form
-                            const float tv = sqN + s_i + G.y;
-                            allow += kRoundRel * tv * tv * P2;
+                        for (int m = 0; m < 8; ++m)
+                            cq[m] = q0 == 0 ? cq0[m] : __ldcs(cb + (size_t)(q0 + 4 * m + sub) * cs + t);
+                        if (col && qprev >= q0 && qprev < q0 + 32 && ((qprev - q0) & 3) == sub) {
+                            const int mm = (qprev - q0) >> 2;
+#pragma unroll
+                            for (int m = 0; m < 8; ++m)
+                                if (m == mm) cq[m] = sn;
+                            __stcs(cb + (size_t)qprev * cs + t, sn);
                         }
-                        lb = fminf(lb, dlo > 0.f ? LB / (den * den) - allow / (dlo * dlo) : -INFINITY);
+                        const int nq = nadd - q0;  // slot q0 + 4m + sub exists iff 4m + sub < nq
+                        if (fast && nq >= 32) {
+#pragma unroll
+                            for (int m = 0; m < 8; ++m)
+                                kmin = fminf(kmin, fast_score(slot4[q0 + 4 * m + sub], cq[m], p_i, Ai, Pm));
+                        } else {
+#pragma unroll
+                            for (int m = 0; m < 8; ++m)
+                                if (4 * m + sub < nq)
+                                    kmin = fminf(kmin, any_score<DPL, VT>(slot4[q0 + 4 * m + sub], cq[m], p_i, Ai, Pm, P,
+                                                                          P2, N, vr, mu, g, Wt, Ep, q0 + 4 * m + sub));
+                        }
                     }
-                    lb = fminf(lb, __shfl_xor_sync(FW_FULL, lb, 1));
-                    lb = fminf(lb, __shfl_xor_sync(FW_FULL, lb, 2));
-                    if (valid) {
+                    if (kmin < lmin) {  // first position of the lane's least score
+                        lmin = kmin;
+                        lt = t;
+                        li = i;
+                        lp = p_i;
+                        lA = Ai;
+                    }
+                };
+                auto load_cq0 = [&](int t, float (&cq0)[8]) {
+#pragma unroll
+                    for (int m = 0; m < 8; ++m) cq0[m] = __ldcs(cb + (size_t)(4 * m + sub) * cs + t);
+                };
+                if (first) {
+                    for (int t0 = 0; t0 < nk; t0 += KPI) {
+                        const int t = t0 + gq;
+                        const bool valid = t < nk;
+                        const int ts = valid ? t : t0;
+                        const int i = kb[ts];
+                        const VT *vr = V + (int64_t)i * d;
+                        float cq0[8];
+                        load_cq0(ts, cq0);
+                        float sg, sn;  // g.w_i and |w_i|^2 from w itself
+                        lane_products<DPL, VT>(vr, mu, g, sub, sg, sn);
+                        sg += __shfl_xor_sync(FW_FULL, sg, 1);
+                        sn += __shfl_xor_sync(FW_FULL, sn, 1);
+                        sg += __shfl_xor_sync(FW_FULL, sg, 2);
+                        sn += __shfl_xor_sync(FW_FULL, sn, 2);
+                        const float p_i = expf(lg[i] - M) * Zi;
+                        if (!valid) continue;
                         if (sub == 0) {
-                            lbk[t] = lb;
-                            ak[t] = alpha;
+                            pk[t] = p_i;
+                            xk[t] = sn;
                         }
-                        if (lb < lbmin) {
-                            lbmin = lb;
-                            tmin = t;
-                        }
+                        score_key(t, i, vr, sg, sn, p_i, sn, false, cq0);
+                    }
+                } else {
+                    // software pipeline: the value row of the next iteration and the
+                    // kept index of the one after are in flight during this one
+                    const int niter = (nk + KPI - 1) / KPI;
+                    int i_cur = kb[gq < nk ? gq : nk - 1];
+                    int i_next = kb[gq + KPI < nk ? gq + KPI : nk - 1];
+                    LaneRow<DPL, VT> row;
+                    row.load(V + (int64_t)i_cur * d, sub);
+                    for (int it = 0; it < niter; ++it) {
+                        const int t = it * KPI + gq;
+                        const bool valid = t < nk;
+                        const int ts = valid ? t : nk - 1;
+                        float cq0[8];
+                        load_cq0(ts, cq0);
+                        const float p_i = pk[ts], x2 = xk[ts];
+                        LaneRow<DPL, VT> rown;
+                        rown.load(V + (int64_t)i_next * d, sub);
+                        const int tnn = t + 2 * KPI;
+                        const int i_nn = kb[tnn < nk ? tnn : nk - 1];
+                        float sg, sn;  // v_i.g and v_i . (the changed slot's vector)
+                        lane_products_v_row<DPL, VT>(row, g, wdep, sub, sg, sn);
+                        sg += __shfl_xor_sync(FW_FULL, sg, 1);
+                        sn += __shfl_xor_sync(FW_FULL, sn, 1);
+                        sg += __shfl_xor_sync(FW_FULL, sg, 2);
+                        sn += __shfl_xor_sync(FW_FULL, sn, 2);
+                        if (valid)
+                            score_key(t, i_cur, V + (int64_t)i_cur * d, sg - gm, sn - ym, p_i, x2, t != tprev, cq0);
+                        row = rown;
+                        i_cur = i_next;
+                        i_next = i_nn;
                     }
                 }
                 first = false;
-                if (sub == 0) cand[gq] = tmin;
-                __syncthreads();
-                // ---- step 2: exact scores of the nominated keys -> an attained score UB
-                float best = INFINITY;
-                unsigned long long bkey = ~0ull;
-                int bt = -1, bq = -1;
-                score_positions<DPL, VT>(cand, KPI, kb, pk, ak, xk, V, mu, g, Wt, Ep, pj, betaj, rj, idxj, nadd, P, P2,
-                                         N, sqN, best, bkey, bt, bq);
-                const float UB = block_min(best, red);
-                // ---- step 3: exact scores of every key whose bound does not exceed UB.
-                // A key's bound lies below every score computed for its pairs (the
-                // bound carries the rounding allowance), so the keys left out hold no
-                // pair scoring at or below UB, and the best pair is among those kept.
-                const float thr = UB;
-                if (tid == 0) s_cnt = 0;
-                __syncthreads();
-                for (int t0 = 0; t0 < nk; t0 += SWT) {
-                    const int t = t0 + tid;
-                    const bool keep = t < nk && !(lbk[t] > thr);
-                    const uint32_t bal = __ballot_sync(FW_FULL, keep);
-                    int basew = 0;
-                    if (lane == 0 && bal) basew = atomicAdd(&s_cnt, __popc(bal));
-                    basew = __shfl_sync(FW_FULL, basew, 0);
-                    if (keep) sl[basew + __popc(bal & ((1u << lane) - 1u))] = t;
+                // the block's least score
+                {
+                    const float wb = warp_min(lmin);
+                    if (lane == 0) red[wid] = wb;
+                    if (tid == 0) s_bkey = ~0ull;
                 }
                 __syncthreads();
-                const int nsv = s_cnt;
-                best = INFINITY;
-                bkey = ~0ull;
-                bt = bq = -1;
-                score_positions<DPL, VT>(sl, nsv, kb, pk, ak, xk, V, mu, g, Wt, Ep, pj, betaj, rj, idxj, nadd, P, P2, N,
-                                         sqN, best, bkey, bt, bq);
-                // block argmin of (score, i, j)
-                if (tid == 0) {
-                    s_best = INFINITY;
-                    s_bkey = ~0ull;
-                }
-                float wb = warp_min(best);
-                if (lane == 0) red[wid] = wb;
-                __syncthreads();
-                if (tid == 0) {
-                    float m = INFINITY;
-                    for (int w = 0; w < SWT / 32; ++w) m = fminf(m, red[w]);
-                    s_best = m;
-                }
-                __syncthreads();
-                if (best == s_best) atomicMin(&s_bkey, bkey);
-                __syncthreads();
-                if (best == s_best && bkey == s_bkey && bt >= 0) {
-                    s_bt = bt;
-                    s_bq = bq;
+                float bmin = INFINITY;
+                for (int w = 0; w < SWT / 32; ++w) bmin = fminf(bmin, red[w]);
+                // the lanes that attain it score their position's pairs again (the
+                // same operations on the same inputs); the smallest (i, j) wins
+                unsigned long long mykey = ~0ull;
+                int myt = -1, myq = -1;
+                if (bmin < 0.f && lt >= 0 && lmin == bmin) {
+                    const float Pm = P - lp;
+                    const VT *vr = V + (int64_t)li * d;
+                    for (int q = sub; q < nadd; q += QL) {
+                        const float sc = any_score<DPL, VT>(slot4[q], __ldcs(cb + (size_t)q * cs + lt), lp, lA, Pm, P, P2,
+                                                            N, vr, mu, g, Wt, Ep, q);
+                        if (sc == bmin) {
+                            const unsigned long long key = ((unsigned long long)(uint32_t)li << 32) | (uint32_t)idxj[q];
+                            if (key < mykey) {
+                                mykey = key;
+                                myt = lt;
+                                myq = q;
+                            }
+                        }
+                    }
+                    if (mykey != ~0ull) atomicMin(&s_bkey, mykey);
                 }
                 __syncthreads();
-                const float bs = s_best;
+                if (mykey != ~0ull && mykey == s_bkey) {
+                    s_bt = myt;
+                    s_bq = myq;
+                }
+                __syncthreads();
+                const float bs = s_bkey != ~0ull ? bmin : INFINITY;
                 const unsigned long long bk = s_bkey;
                 if (!(bs < 0.f)) break;  // no pair strictly decreases es
                 if (taken >= MS) {
@@ -732,6 +843,8 @@ __global__ void __launch_bounds__(SWT, 2) k_long_swap(const LSArgs a)
                 N = block_sum(gl2, red);
                 x2n = block_sum(x2n, red);
                 if (tid == 0) xk[tb] = x2n;
+                tprev = tb;
+                qprev = qj;
                 __syncthreads();
                 ++taken;
             }
@@ -747,26 +860,33 @@ __global__ void __launch_bounds__(SWT, 2) k_long_swap(const LSArgs a)
     }
 }
 
-// pool slots rounded up to the 16-slot blocks of the exact scoring step
-inline int pool_slots(int E) { return std::max(16, (E + 15) / 16 * 16); }
+// pool slots rounded up to the 32-slot blocks of the product tile
+inline int pool_slots(int E) { return std::max(32, (E + 31) / 32 * 32); }
 
 template <int DPL> size_t ls_smem(int Ep)
 {
     constexpr int d = DPL * 32;
-    return sizeof(float) * (10 * (size_t)d + (size_t)d * Ep + 5 * (size_t)Ep + KPI + 5 * SWGRP + 32 + 8 + 256) + 64;
+    return sizeof(float) * (10 * (size_t)d + (size_t)d * Ep + 7 * (size_t)Ep + 32 + 8 + 256) + 64;
 }
 
 }  // namespace
 
-// two resident blocks per SM (the launch bounds guarantee the registers for it)
-static unsigned ls_grid(const RowsDev &R) { return (unsigned)std::min<int64_t>(R.rows, 152 * 2); }
+// LS_BPS resident blocks per SM (the launch bounds guarantee the registers for it)
+static unsigned ls_grid(const RowsDev &R) { return (unsigned)std::min<int64_t>(R.rows, 152 * LS_BPS); }
 
 static size_t ls_array_bytes(const RowsDev &R) { return align256((size_t)ls_grid(R) * R.max_n * 4); }
 
+static int ls_cstride(const RowsDev &R) { return (R.max_n + 3) / 4 * 4; }
+
+static size_t ls_table_bytes(const RowsDev &R, int E)
+{
+    return align256((size_t)ls_grid(R) * pool_slots(E) * ls_cstride(R) * 4);
+}
+
 size_t long_swap_workspace(const RowsDev &R, int nb, int E, int max_swaps)
 {
-    (void)nb, (void)E, (void)max_swaps;
-    return ls_array_bytes(R) * 7;
+    (void)nb, (void)max_swaps;
+    return ls_array_bytes(R) * 4 + ls_table_bytes(R, E);
 }
 
 fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &topk, int E, int max_swaps,
@@ -793,6 +913,7 @@ fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out
     a.capped = capped;
     a.refined_gap = refined_gap;
     a.topk_gap = topk_gap;
+    a.cstride = ls_cstride(R);
     const unsigned grid = ls_grid(R);
     const size_t arr = ls_array_bytes(R);
     char *w = (char *)ws;
@@ -800,9 +921,7 @@ fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out
     a.kbuf = (int32_t *)(w + 1 * arr);
     a.pbuf = (float *)(w + 2 * arr);
     a.xbuf = (float *)(w + 3 * arr);
-    a.lbuf = (float *)(w + 4 * arr);
-    a.abuf = (float *)(w + 5 * arr);
-    a.sbuf = (int32_t *)(w + 6 * arr);
+    a.cbuf = (float *)(w + 4 * arr);
     FW_DISPATCH(R.d, R.v_dtype, {
         const size_t smem = ls_smem<DPL>(a.Ep);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_swap<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
