@@ -12,7 +12,10 @@
 //   o_A - mu = (pbar(A) N_A - p(A) N_{A^c}) / p(A),
 // which never subtracts two rounded outputs and keeps the gap accurate when it
 // is small; pbar(A) is summed over the dropped keys.
+#include <algorithm>
+
 #include "fw_internal.h"
+#include "tc_sm100.cuh"
 
 namespace fw {
 namespace {
@@ -28,6 +31,8 @@ struct SelArgs {
     int nb;
     fw_gap_out out;
     LongWs ws;
+    int32_t *redo_list;   // rows the register select leaves to the radix select
+    int32_t *redo_count;  // (device) entries of redo_list; NULL: one CTA per row
 };
 
 __device__ __forceinline__ void block_max_sum(float &m, float &s, float *red_m, float *red_s)
@@ -77,7 +82,7 @@ __device__ __forceinline__ float key_float(uint32_t k)
 }
 
 template <bool STAGED>
-__global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
+__device__ __forceinline__ void select_row(const SelArgs &a, const int64_t row)
 {
     extern __shared__ uint32_t skeys[];  // [n] order keys when STAGED
     __shared__ uint32_t hist[4][256];
@@ -88,7 +93,6 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
     __shared__ uint32_t wcnt[LT / 32];
     __shared__ int s_found;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-    const int64_t row = blockIdx.x;
     const int64_t g = row / a.R.R;
     const int64_t ri = row - g * a.R.R;
     const int n = a.R.n[g];
@@ -256,6 +260,314 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
                 const uint32_t bal = __ballot_sync(FW_FULL, kept);
                 if (lane == 0 && (j >> 5) < nw) wbits[j >> 5] = bal;
             }
+        }
+    }
+}
+
+template <bool STAGED>
+__global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
+{
+    if (!a.redo_count) {
+        select_row<STAGED>(a, blockIdx.x);
+        return;
+    }
+    const int cnt = *a.redo_count;
+    for (int i = blockIdx.x; i < cnt; i += gridDim.x) {
+        select_row<STAGED>(a, a.redo_list[i]);
+        __syncthreads();
+    }
+}
+
+// ------------------------------------------------------ linear-bin select
+// Rows of at most SEL_MAX_N keys.  Persistent CTAs walk rows; a row's logits
+// arrive in shared memory by bulk copy.  The k-th largest key of every budget
+// comes from one histogram of SNB linear bins over [min, max] of the row (a
+// monotone map of the float, so the bins split the key order), the bin holding
+// the k-th key, and an exact rank among that bin's keys.  Rows whose threshold
+// bin holds more than SCAP keys (heavy ties) are listed for the radix select,
+// which runs on them after this kernel.
+constexpr int SEL_MAX_N = 32768;  // longest row of the linear-bin select
+constexpr int SNB = 2048;         // linear bins
+constexpr int SCAP = 1024;        // keys of a threshold bin ranked directly
+constexpr uint32_t SEL_WAIT = 1u << 22;  // polls of a row-copy wait before it gives up
+constexpr uint32_t SEL_CHUNK = 32768;    // bytes per bulk-copy instruction
+
+__device__ __forceinline__ bool row_bulk_ok(const RowsDev &R, int64_t row, int &n, const float *&lg)
+{
+    const int64_t g = row / R.R;
+    const int64_t ri = row - g * R.R;
+    n = R.n[g];
+    const int64_t off = R.logit_off[g] + ri * n;
+    lg = R.logits + off;
+    return (n & 3) == 0 && (reinterpret_cast<uintptr_t>(lg) & 15) == 0;
+}
+
+template <int NT>
+__global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
+{
+    extern __shared__ __align__(16) float sbuf[];  // [max_n] the row's logits
+    __shared__ uint32_t hist[SNB];
+    __shared__ uint32_t ckey[4][SCAP];
+    __shared__ int32_t cidx[4][SCAP];
+    __shared__ float red_a[32], red_b[32];
+    __shared__ uint32_t wsum[32];
+    __shared__ int s_tb[4], s_cnt[4], s_ti[4], s_kv[4], s_rem[4], s_bcnt[4], s_err;
+    __shared__ uint32_t s_T[4];
+    __shared__ __align__(8) uint64_t full;
+    constexpr int NW = NT / 32;
+    constexpr int BPT = SNB / NT;  // bins per thread in the scan
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int nb = a.nb;
+    if (tid == 0) {
+        tc::mbar_init(&full, 1);
+        tc::mbar_init_fence();
+        s_err = 0;
+    }
+    __syncthreads();
+    uint32_t phase = 0;
+    int64_t fail_row = -1;
+    for (int64_t row = blockIdx.x; row < a.R.rows; row += gridDim.x) {
+        int n;
+        const float *lg;
+        const bool bulk = row_bulk_ok(a.R, row, n, lg);
+        // ---- the row into shared memory; max, min and finiteness on the way
+        if (bulk) {
+            if (tid == 0) {
+                tc::fence_async_smem();
+                const uint32_t bytes = (uint32_t)n * 4u;
+                tc::mbar_arrive_expect_tx(&full, bytes);
+                for (uint32_t o = 0; o < bytes; o += SEL_CHUNK) {
+                    const uint32_t c = bytes - o < SEL_CHUNK ? bytes - o : SEL_CHUNK;
+                    tc::bulk_g2s(reinterpret_cast<char *>(sbuf) + o, reinterpret_cast<const char *>(lg) + o, c,
+                                 &full);
+                }
+            }
+            if (wid == 0 && !tc::mbar_wait(&full, phase, SEL_WAIT)) s_err = 1;  // (every writer stores 1)
+            phase ^= 1u;
+            __syncthreads();
+            if (s_err) {
+                fail_row = row;
+                break;
+            }
+        } else {
+            for (int j = tid; j < n; j += NT) sbuf[j] = lg[j];
+            __syncthreads();
+        }
+        // the next row heads for L2 while this one is processed
+        if (tid == 0 && row + gridDim.x < a.R.rows) {
+            int n2;
+            const float *lg2;
+            if (row_bulk_ok(a.R, row + gridDim.x, n2, lg2)) {
+                const uint32_t bytes = (uint32_t)n2 * 4u;
+                for (uint32_t o = 0; o < bytes; o += SEL_CHUNK)
+                    tc::bulk_prefetch_l2(reinterpret_cast<const char *>(lg2) + o,
+                                         bytes - o < SEL_CHUNK ? bytes - o : SEL_CHUNK);
+            }
+        }
+        // f(j, x) for every key, four per shared-memory load
+        auto for_keys = [&](auto &&f) {
+            const int n4 = n >> 2;
+            for (int q = tid; q < n4; q += NT) {
+                const float4 v = reinterpret_cast<const float4 *>(sbuf)[q];
+                f(4 * q, v.x);
+                f(4 * q + 1, v.y);
+                f(4 * q + 2, v.z);
+                f(4 * q + 3, v.w);
+            }
+            for (int j = 4 * n4 + tid; j < n; j += NT) f(j, sbuf[j]);
+        };
+        float m = -INFINITY, mn = INFINITY;
+        bool nan = false;
+        for_keys([&](int, float x) {
+            nan |= x != x;
+            m = fmaxf(m, x);
+            mn = fminf(mn, x);
+        });
+        m = warp_max(m);
+        mn = warp_min(mn);
+        if (lane == 0) {
+            red_a[wid] = m;
+            red_b[wid] = mn;
+        }
+        for (int i = tid; i < SNB; i += NT) hist[i] = 0u;
+        if (tid < 4) s_cnt[tid] = 0;
+        if (tid < nb) s_kv[tid] = a.k[row * nb + tid];
+        bool bad = __syncthreads_or(nan) || n < 1;
+        m = red_a[0];
+        mn = red_b[0];
+        for (int w = 1; w < NW; ++w) {
+            m = fmaxf(m, red_a[w]);
+            mn = fminf(mn, red_b[w]);
+        }
+        bad |= !isfinite(m) || !isfinite(mn);  // (an infinite key is the max or the min)
+        int status = bad ? FW_ERR_NONFINITE : FW_OK;
+        for (int b = 0; b < nb; ++b) {
+            const int kb = s_kv[b];
+            if (kb < 1 || kb > n) status = status == FW_OK ? FW_ERR_INVALID_ARG : status;
+        }
+        // ---- sum of exponentials and the histogram of linear bins over [mn, m]
+        // (halves keep m - mn finite)
+        const float hmn = mn * 0.5f, den = m * 0.5f - hmn;
+        float scl = den > 0.f ? (float)SNB / den : 0.f;
+        if (!(scl < 1e30f)) scl = 0.f;
+        auto bin_of = [&](float v) { return (int)fminf((v * 0.5f - hmn) * scl, (float)(SNB - 1)); };
+        float se = 0.f;
+        if (status == FW_OK) {
+            for_keys([&](int, float x) {
+                se += __expf(x - m);
+                atomicAdd(&hist[bin_of(x)], 1u);
+            });
+        }
+        se = warp_sum(se);
+        __syncthreads();  // red_a reads above are done
+        if (lane == 0) red_a[wid] = se;
+        __syncthreads();
+        float Z = 0.f;
+        for (int w = 0; w < NW; ++w) Z += red_a[w];
+        if (tid == 0) {
+            a.ws.M[row] = m;
+            a.ws.Z[row] = Z;
+            a.ws.status[row] = status;
+            if (a.out.row_max) a.out.row_max[row] = m;
+            if (a.out.row_sum) a.out.row_sum[row] = Z;
+            if (a.out.row_status) a.out.row_status[row] = status;
+        }
+        if (status != FW_OK) continue;  // (uniform)
+        // ---- keys above each bin (bins from the top), the bin of each budget's k-th key
+        uint32_t hv[BPT], loc = 0;
+#pragma unroll
+        for (int i = 0; i < BPT; ++i) {
+            hv[i] = hist[SNB - 1 - (tid * BPT + i)];
+            loc += hv[i];
+        }
+        uint32_t inc = loc;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(FW_FULL, inc, o);
+            if (lane >= o) inc += y;
+        }
+        if (lane == 31) wsum[wid] = inc;
+        __syncthreads();
+        uint32_t above = inc - loc;
+        for (int w = 0; w < wid; ++w) above += wsum[w];
+#pragma unroll
+        for (int i = 0; i < BPT; ++i) {
+            const int bn = SNB - 1 - (tid * BPT + i);
+            for (int b = 0; b < nb; ++b) {
+                const uint32_t kb = (uint32_t)s_kv[b];
+                if (above < kb && kb <= above + hv[i]) {
+                    s_tb[b] = bn;
+                    s_rem[b] = (int)(kb - above);
+                    s_bcnt[b] = (int)hv[i];
+                }
+            }
+            above += hv[i];
+        }
+        __syncthreads();
+        // a budget whose threshold bin is crowded (heavy ties) leaves the row to
+        // the radix select, which runs after this kernel on the listed rows
+        bool crowded = false;
+        for (int b = 0; b < nb; ++b) crowded |= s_bcnt[b] > SCAP;
+        if (crowded) {
+            if (tid == 0) a.redo_list[atomicAdd(a.redo_count, 1)] = (int32_t)row;
+            __syncthreads();
+            continue;
+        }
+        // ---- the threshold bins' keys, then their exact ranks
+        int gb[4], glo = SNB, ghi = -1;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            gb[b] = b < nb ? s_tb[b] : -1;
+            if (b < nb) {
+                glo = min(glo, gb[b]);
+                ghi = max(ghi, gb[b]);
+            }
+        }
+        for_keys([&](int j, float x) {
+            const int bn = bin_of(x);
+            if (bn < glo || bn > ghi) return;
+#pragma unroll
+            for (int b = 0; b < 4; ++b)
+                if (bn == gb[b]) {
+                    const int p = atomicAdd(&s_cnt[b], 1);
+                    ckey[b][p] = order_key(x);
+                    cidx[b][p] = j;
+                }
+        });
+        __syncthreads();
+        // thread t ranks candidate t mod 256 (and every 256th after it) of
+        // budget t / 256, so the budgets' ranks run side by side
+        {
+            constexpr int CPB = NT / 4;  // threads per budget
+            const int b = tid / CPB;
+            if (b < nb) {
+                const int cb = s_bcnt[b];
+                const int want = s_rem[b] - 1;
+                for (int c = tid % CPB; c < cb; c += CPB) {
+                    const uint32_t kc = ckey[b][c];
+                    const int ic = cidx[b][c];
+                    int r = 0;
+#pragma unroll 4
+                    for (int c2 = 0; c2 < cb; ++c2) {
+                        const uint32_t k2 = ckey[b][c2];
+                        r += k2 > kc || (k2 == kc && cidx[b][c2] < ic);
+                    }
+                    if (r == want) {
+                        s_T[b] = kc;
+                        s_ti[b] = ic;
+                    }
+                }
+            }
+        }
+        __syncthreads();
+        // ---- thresholds and kept bits (a warp per 32 consecutive keys)
+        if (tid < nb) {
+            a.ws.tk[row * nb + tid] = s_T[tid];
+            a.ws.ti[row * nb + tid] = s_ti[tid];
+            if (a.out.thr_key) a.out.thr_key[row * nb + tid] = s_T[tid];
+            if (a.out.thr_idx) a.out.thr_idx[row * nb + tid] = s_ti[tid];
+        }
+        if (a.out.kept_bits) {
+            // keys strictly above each threshold by one compare and a ballot; the
+            // keys equal to it (all in its bin, so among the candidates) up to
+            // the tie index are added after
+            const int nw = a.out.kept_words;
+            float xt[4];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) xt[b] = b < nb ? key_float(s_T[b]) : INFINITY;
+            for (int w = wid; w < nw; w += NW) {
+                const int j = w * 32 + lane;
+                const float x = j < n ? sbuf[j] : -INFINITY;
+                uint32_t mine = 0u;  // lane b keeps budget b's word
+#pragma unroll
+                for (int b = 0; b < 4; ++b) {
+                    const uint32_t word = __ballot_sync(FW_FULL, x > xt[b]);
+                    if (lane == b) mine = word;
+                }
+                if (lane < nb) a.out.kept_bits[(row * nb + lane) * (int64_t)nw + w] = mine;
+            }
+            __syncthreads();  // the words above are visible to the block
+            constexpr int CPB = NT / 4;
+            const int b = tid / CPB;
+            if (b < nb) {
+                const uint32_t T = s_T[b];
+                const int ti = s_ti[b];
+                for (int c = tid % CPB; c < s_bcnt[b]; c += CPB) {
+                    const int ic = cidx[b][c];
+                    if (ckey[b][c] == T && ic <= ti)
+                        atomicOr(&a.out.kept_bits[(row * nb + b) * (int64_t)nw + (ic >> 5)], 1u << (ic & 31));
+                }
+            }
+        }
+        __syncthreads();  // sbuf, s_T, s_ti, hist and candidates are reused by the next row
+    }
+    if (fail_row >= 0 && tid == 0) {
+        // a row copy did not arrive in time: after a last bounded wait for it,
+        // that row and the rest of this CTA's rows are marked
+        (void)tc::mbar_wait(&full, phase ^ 1u, SEL_WAIT);
+        for (int64_t row = fail_row; row < a.R.rows; row += gridDim.x) {
+            a.ws.status[row] = FW_ERR_TIMEOUT;
+            if (a.out.row_status) a.out.row_status[row] = FW_ERR_TIMEOUT;
         }
     }
 }
@@ -432,18 +744,45 @@ static LongWs carve(const RowsDev &R, int nb, void *ws)
     return L;
 }
 
-size_t long_gap_workspace(const RowsDev &R, int nb)
+// after the LongWs arrays: the redo list [rows] and its count
+static size_t carve_bytes(const RowsDev &R, int nb)
 {
     return align256(R.rows * 4) * 2 + align256(R.rows * nb * 4) * 2 + align256(R.rows * 4);
 }
+
+size_t long_gap_workspace(const RowsDev &R, int nb) { return carve_bytes(R, nb) + align256(R.rows * 4) + 256; }
 
 fw_status long_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, void *ws, size_t ws_bytes,
                    cudaStream_t s)
 {
     (void)ws_bytes;
     const LongWs L = carve(R, nb, ws);
-    const SelArgs sa{R, k, nb, out, L};
-    if (R.max_n <= kSelStageMax) {
+    int32_t *redo_list = (int32_t *)((char *)ws + carve_bytes(R, nb));
+    int32_t *redo_count = (int32_t *)((char *)redo_list + align256(R.rows * 4));
+    SelArgs sa{R, k, nb, out, L, redo_list, nullptr};
+    if (R.max_n <= SEL_MAX_N) {
+        FW_CUDA_CHECK(cudaMemsetAsync(redo_count, 0, sizeof(int32_t), s));
+        sa.redo_count = redo_count;
+        int dev = 0, sms = 0;
+        FW_CUDA_CHECK(cudaGetDevice(&dev));
+        FW_CUDA_CHECK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+        auto launch = [&](auto kernel, int nt) -> fw_status {
+            const size_t smem = (size_t)R.max_n * 4;
+            FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+            int per_sm = 0;
+            FW_CUDA_CHECK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, nt, smem));
+            const int64_t grid = std::min<int64_t>(R.rows, (int64_t)sms * std::max(per_sm, 1));
+            FW_LAUNCH(kernel, (unsigned)grid, nt, smem, s, sa);
+            return FW_OK;
+        };
+        const fw_status st = R.max_n <= 8192 ? launch(k_long_select_bins<512>, 512)
+                                              : launch(k_long_select_bins<1024>, 1024);
+        if (st != FW_OK) return st;
+        // the listed rows (crowded threshold bins) by the radix select
+        const size_t smem = (size_t)R.max_n * 4;
+        FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_select<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        FW_LAUNCH(k_long_select<true>, (unsigned)std::min<int64_t>(R.rows, sms), LT, smem, s, sa);
+    } else if (R.max_n <= kSelStageMax) {
         const size_t smem = (size_t)R.max_n * 4;
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_select<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
         FW_LAUNCH(k_long_select<true>, (unsigned)R.rows, LT, smem, s, sa);
