@@ -248,9 +248,10 @@ def cpu_baseline(seed, rows_per_group=40):
 
 # ----------------------------------------------------------------- sections
 
-def section_long_rows(fw, device, K, W, flush, peaks):
-    """a1-a4 (top-k gap) and a5 (swap rule, E=32) on 4,096 rows x 32,768 keys."""
-    b = workloads.long_rows(seed=0, backend="torch", device=device)
+def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
+    """a1-a4 (top-k gap) and a5 (swap rule, E=32) on 8 heads x rows_per_head rows
+    x 32,768 keys (4,096 rows at the default)."""
+    b = workloads.long_rows(seed=0, rows_per_head=rows_per_head, backend="torch", device=device)
     rows = fw.rows_from_batch(b, device)
     rows_k = b.k
     holder = {}
@@ -261,17 +262,35 @@ def section_long_rows(fw, device, K, W, flush, peaks):
     total, _ = time_steps(gap_step, K, W, flush, lambda: None)
     ms_gap = total / K
     top = holder["top"]
-    total, _ = time_steps(lambda: fw.swap_refine(rows, rows_k, top, E=32, max_swaps=64), max(2, K // 2), 2,
-                          flush, lambda: None)
-    ms_swap = total / max(2, K // 2)
-    nbytes = (rows.logits.numel() * 4 + rows.v.numel() * 2 + rows.num_rows * (128 * 4 * 4 + 3 * 4 * 4 + 3 * 4096 * 4))
+
+    def swap_step():
+        holder["sw"] = fw.swap_refine(rows, rows_k, top, E=32, max_swaps=64)
+
+    ks = max(2, K // 2)
+    total, _ = time_steps(swap_step, ks, 2, flush, lambda: None)
+    ms_swap = total / ks
+    ns = holder["sw"]["n_swaps"].float()
+    R, n, d, nb = rows.num_rows, int(b.n_host[0]), b.d, rows_k.shape[1]
+    # algorithmic bytes of the gap call: logits once, the value blocks once,
+    # outputs (o, three o_A, gap / dropped / phi, thresholds, kept bits)
+    nbytes = (rows.logits.numel() * 4 + rows.v.numel() * 2
+              + R * (d * 4 * (1 + nb) + nb * 3 * 4 + nb * 8 + nb * (n // 8)))
     ach = nbytes / (ms_gap * 1e-3) / 1e9
-    return dict(workload="long_rows: 8 heads x 512 rows, n=32768, d=128, bf16 V, k in {2048,4096,8192}",
+    # the swap rounds: per round one pass over the k kept keys (a d-long product
+    # with g and one with the changed pool vector, E table entries)
+    rounds = float((ns + 1).sum().item())
+    return dict(workload=f"long_rows: 8 heads x {rows_per_head} rows, n=32768, d=128, bf16 V, k in {{2048,4096,8192}}",
                 path="a1-a4 (fw_dense_and_topk_gap) then a5 (fw_swap_refine, E=32)", metric="rows/s",
-                value=rows.num_rows / ((ms_gap + ms_swap) * 1e-3), gap_rows_per_s=rows.num_rows / (ms_gap * 1e-3),
-                swap_rows_per_s=rows.num_rows / (ms_swap * 1e-3), ms_gap=ms_gap, ms_swap=ms_swap,
-                roofline=dict(bound="hbm", kernel="k_long_select + k_long_pv", achieved=ach, peak=peaks["hbm_gbs"],
-                              unit="GB/s", frac=ach / peaks["hbm_gbs"], traffic=None, algorithmic_bytes=nbytes))
+                value=R / ((ms_gap + ms_swap) * 1e-3), gap_rows_per_s=R / (ms_gap * 1e-3),
+                swap_rows_per_s=R / (ms_swap * 1e-3), ms_gap=ms_gap, ms_swap=ms_swap,
+                swaps_per_row_budget=float(ns.mean().item()), swap_rounds=rounds,
+                roofline=dict(bound="hbm", kernel="k_long_select_bins + k_long_pv_tc (fw_dense_and_topk_gap)",
+                              achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s", frac=ach / peaks["hbm_gbs"],
+                              traffic=None, algorithmic_bytes=nbytes,
+                              tensor_flops_executed=2 * 3 * (nb + 1) * n * d * R,
+                              tensor_tflops=2 * 3 * (nb + 1) * n * d * R / (ms_gap * 1e-3) / 1e12,
+                              tensor_basis="P.V as a bf16 GEMM: 3 bf16 terms per probability, nb + 1 band rows; "
+                                           "time of the whole gap call (the select kernel included)"))
 
 
 def section_contour(fw, device, K, W, flush, peaks):
@@ -307,6 +326,10 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--rows-scale", type=float, default=1.0,
                     help="fraction of the headline rows (profiling captures of a smaller case)")
+    ap.add_argument("--only", default="all", choices=["all", "long_rows", "contour"],
+                    help="run one section alone and print its line (profiling captures)")
+    ap.add_argument("--long-rows-per-head", type=int, default=512,
+                    help="rows per head of the long-row section (profiling captures of a smaller case)")
     args = ap.parse_args()
     K, W = args.steps, max(3, args.warmup)
 
@@ -349,6 +372,16 @@ def main():
 
     peaks = read_peaks()
     flush = L2Flush(device)
+    if args.only != "all":
+        if rank == 0:
+            if args.only == "long_rows":
+                sec = section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=args.long_rows_per_head)
+            else:
+                sec = section_contour(fw, device, K, W, flush, peaks)
+            print(json.dumps(dict(section=args.only, **sec)), flush=True)
+        if dist:
+            dist.destroy_process_group()
+        return
     barrier = (lambda: dist.barrier()) if dist else (lambda: None)
 
     wl = EnumWorkload(fw, seed=rank, device=device, rows_scale=args.rows_scale)
@@ -370,11 +403,12 @@ def main():
     alg_flops = sum(r.num_rows * SUBSETS_PER_ROW * 4 * b.d for r, b in zip(wl.rows, wl.batches))  # 4d flops per subset
     alu_ach = alg_flops / (enum_ms * 1e-3) / 1e12
     lane_frac = wl.subsets * ALU_OPS_PER_SUBSET / (enum_ms * 1e-3) / (152 * 128 * sm_mhz * 1e6)
-    # DRAM traffic of one launch from the ncu capture (group of 36,864 rows, d = 128:
-    # 930.1 MB), scaled to the average launch by its input bytes
+    # DRAM traffic of one call from the ncu capture of its prep and walk kernels
+    # (group of 36,864 rows, d = 128: 522.3 + 85.7 MB), scaled to the average
+    # call by its input bytes
     cap_in = 36864 * (24 * 128 * 4 + 24 * 4)
     avg_in = sum(r.num_rows * (24 * b.d * 4 + 24 * 4) for r, b in zip(wl.rows, wl.batches)) / len(wl.batches)
-    traffic = 930.1e6 * avg_in / cap_in if args.rows_scale == 1.0 else None
+    traffic = (522.3e6 + 85.7e6) * avg_in / cap_in if args.rows_scale == 1.0 else None
 
     # end to end through the public API with host buffers
     e2e = EnumE2E(wl)
@@ -407,8 +441,9 @@ def main():
                               lane_issue_frac=lane_frac,
                               peak_basis=f"152 SMs x 128 fp32 lanes x 2 x {sm_mhz:.0f} MHz (median SM clock under "
                                          f"load)",
-                              traffic_basis="ncu dram bytes of one full-size launch, scaled to the average launch "
-                                            "by input bytes"),
+                              traffic_basis="ncu dram bytes of k_enum_prep + k_enum_walk for one full-size group, "
+                                            "scaled to the average call by input bytes (the rescore and exhaustive "
+                                            "kernels of the call are not included)"),
                 e2e=dict(value=e2e_value, unit="subsets/s",
                          h2d_bytes_per_step=e2e.h2d, d2h_bytes_per_step=e2e.d2h),
                 gpu_launches=int(launches_timed), clocks=clocks, peaks_source=peaks["source"])
