@@ -14,10 +14,12 @@
 // by cp.async in the 128-byte-swizzled MN-major layout; one thread issues
 // tcgen05.mma and tcgen05.commit frees each stage.  The tensor core rounds its
 // fp32 accumulation toward zero, which over thousands of additions into one
-// accumulator biases the sums by ~1e-3; so every stage accumulates into a fresh
-// TMEM buffer (three in rotation) and the producers add it into fp32 registers
-// with round-to-nearest two stages later, when its MMAs have long completed,
-// so that no producer ever waits on the MMAs it has just enabled.  The epilogue combines
+// accumulator biases the sums by ~1e-3; so every chunk of CH = 8 stages (512
+// keys, about 100 accumulation steps: a bias below ~1e-5 of the partial sums)
+// accumulates into a fresh TMEM buffer (two in rotation) and the producers add
+// it into fp32 registers with round-to-nearest two stages after the chunk ends,
+// when its MMAs have long completed, so that no producer ever waits on the MMAs
+// it has just enabled.  The epilogue combines
 // the bands exactly as the CUDA-core kernel does:
 //   N_A = sum of the bands inside A, N_{A^c} = the rest,
 //   p(A) (m_A - mu) = pbar(A) N_A - p(A) N_{A^c}.
@@ -31,13 +33,14 @@ namespace {
 
 constexpr int TM = 128;       // rows of the MMA tile: (band, row) pairs, band-major
 constexpr int KS = 64;        // keys per stage: one 128-byte swizzle atom of bf16
-constexpr int PW = 8;         // producer warps
-constexpr int NT = (PW + 1) * 32;
-constexpr int NPROD = PW * 32;
+// producer warps: 16 for d = 128, 8 for d = 64 (each warp flushes 32 TMEM columns)
+template <int D> __host__ __device__ constexpr int prod_warps() { return D == 128 ? 16 : 8; }
+template <int D> __host__ __device__ constexpr int pv_threads() { return (prod_warps<D>() + 1) * 32; }
 constexpr int NSPLIT = 3;     // bf16 terms per probability
 constexpr int ASLOTS = 2;     // A tiles in flight
 constexpr int BSLOTS = 4;     // V / logit tiles in flight (prefetch distance 2)
-constexpr int NACC = 3;       // stage accumulators in TMEM (added two stages late)
+constexpr int NACC = 2;       // chunk accumulators in TMEM (added two stages after a chunk ends)
+constexpr int CH = 8;         // stages (of KS keys) accumulated in TMEM between flushes
 constexpr int MAXRT = 32;     // rows per tile
 constexpr uint32_t WAIT_POLLS = 1u << 20;  // polls before a wait gives up (well over a second)
 constexpr int A_SPLIT_BYTES = TM * 128;            // 16 KB
@@ -70,8 +73,13 @@ __device__ __forceinline__ uint32_t bf16_bits_rn(float x)
 }
 
 template <int D>
-__global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
+__global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs a)
 {
+    constexpr int PW = prod_warps<D>();
+    constexpr int NT = pv_threads<D>();
+    constexpr int NPROD = PW * 32;
+    constexpr int TPR = NPROD / MAXRT;  // producer threads per row
+    constexpr int KPTH = KS / TPR;      // keys per producer thread and stage (4 or 8)
     constexpr int B_SLOT_BYTES = D * 128;  // KS keys x D bf16
     constexpr uint32_t TCOLS = NACC * D <= 256 ? 256u : 512u;  // TMEM columns (a power of two)
     constexpr int NC = D / 8;              // 16-byte chunks per V row
@@ -99,6 +107,8 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
     const int n = a.R.n[g];
     const uint16_t *V = reinterpret_cast<const uint16_t *>(a.R.v) + a.R.v_off[g];
     const float *LG = a.R.logits + a.R.logit_off[g];
+    // rows start on 16-byte boundaries: logit copies of 16 bytes
+    const bool lg16 = (n & 3) == 0 && (reinterpret_cast<uintptr_t>(LG) & 15) == 0;
     const int nst = (n + KS - 1) / KS;
 
     if (tid < MAXRT) {
@@ -145,12 +155,15 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
             for (int it = 0; it < nst && ok; ++it) {
                 const int bs = it % BSLOTS, as = it % ASLOTS;
                 ok = tc::mbar_wait(&full[bs], (uint32_t)(it / BSLOTS) & 1u, WAIT_POLLS);
-                // accumulator it % NACC was last read by the producers after stage it - NACC
-                if (ok && it >= NACC)
-                    ok = tc::mbar_wait(&accfree[it % NACC], (uint32_t)((it - NACC) / NACC) & 1u, WAIT_POLLS);
+                // chunk c = it / CH accumulates in buffer c % NACC, last read by the
+                // producers when they flushed chunk c - NACC
+                const int ch = it / CH;
+                if (ok && it % CH == 0 && ch >= NACC)
+                    ok = tc::mbar_wait(&accfree[ch % NACC], (uint32_t)((ch - NACC) / NACC) & 1u, WAIT_POLLS);
                 if (!ok) break;
                 tc::fence_after_sync();
-                const uint32_t dacc = taddr + (uint32_t)((it % NACC) * D);
+                const uint32_t dacc = taddr + (uint32_t)(((it / CH) % NACC) * D);
+                const bool fresh = it % CH == 0;  // first stage of a chunk overwrites the buffer
 #pragma unroll
                 for (int ks = 0; ks < KS / 16; ++ks) {
                     const uint64_t bd = tc::sdesc_sw128(b0 + bs * B_SLOT_BYTES + ks * 2048, KS * 128, 1024);
@@ -158,7 +171,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
                     for (int sp = 0; sp < NSPLIT; ++sp) {
                         const uint64_t ad =
                             tc::sdesc_sw128(a0 + as * A_SLOT_BYTES + sp * A_SPLIT_BYTES + ks * 32, 16, 1024);
-                        tc::mma_bf16(dacc, ad, bd, idesc, ks > 0 || sp > 0);
+                        tc::mma_bf16(dacc, ad, bd, idesc, !fresh || ks > 0 || sp > 0);
                     }
                 }
                 tc::commit(&empty[bs]);
@@ -168,35 +181,34 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ producers
-        const int ptid = tid;                 // 0..NPROD-1
-        const int kc = ptid & 7;              // 8-key chunk of the stage
-        const int rr0 = ptid >> 3;            // the row handled (tiles have at most 32 rows)
-        float bm[2][5];
+        const int ptid = tid;                       // 0..NPROD-1
+        const int rr0 = ptid / TPR;                 // the row handled (tiles have at most 32 rows)
+        const int kc = (ptid % TPR) * KPTH / 8;     // 8-key chunk of the stage
+        const int hk = (ptid % TPR) * KPTH % 8;     // first key of this thread in the chunk
+        float bm[5];
 #pragma unroll
-        for (int q = 0; q < 2; ++q)
-#pragma unroll
-            for (int b = 0; b < 5; ++b) bm[q][b] = 0.f;
+        for (int b = 0; b < 5; ++b) bm[b] = 0.f;
         bool ok = true;
         const uint32_t bbase = tc::smem_u32(sB), lbase = tc::smem_u32(sL);
-        // this thread's accumulator entries: TMEM lane 32 (wid % 4) + lane, columns of half wid / 4
-        const int quarter = wid & 3, half = wid >> 2;
-        float racc[D / 2];
+        // this thread's accumulator entries: TMEM lane 32 (wid % 4) + lane, the
+        // 32 columns of part wid / 4
+        const int quarter = wid & 3, part = wid >> 2;
+        float racc[32];
 #pragma unroll
-        for (int i = 0; i < D / 2; ++i) racc[i] = 0.f;
-        auto flush = [&](int st) {  // add the accumulator of stage st once its MMAs completed
+        for (int i = 0; i < 32; ++i) racc[i] = 0.f;
+        // stage st closes its chunk: the chunk's buffer is added once its MMAs completed
+        auto chunk_end = [&](int st) { return st % CH == CH - 1 || st == nst - 1; };
+        auto flush = [&](int st) {
             if (ok) ok = tc::mbar_wait(&empty[st % BSLOTS], (uint32_t)(st / BSLOTS) & 1u, WAIT_POLLS);
             tc::fence_after_sync();
             const uint32_t base =
-                taddr + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((st % NACC) * D + half * (D / 2));
+                taddr + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(((st / CH) % NACC) * D + part * 32);
+            float v[32];
+            tc::ld32(base, v);
 #pragma unroll
-            for (int c0 = 0; c0 < D / 2; c0 += 32) {
-                float v[32];
-                tc::ld32(base + c0, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) racc[c0 + i] += v[i];
-            }
+            for (int i = 0; i < 32; ++i) racc[i] += v[i];
             tc::fence_before_sync();
-            tc::mbar_arrive(&accfree[st % NACC]);
+            tc::mbar_arrive(&accfree[(st / CH) % NACC]);
         };
         auto issue = [&](int st) {  // cp.async of stage st's V tile and this thread's logits
             if (st < nst) {
@@ -213,11 +225,21 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
                 for (int r = rr0; r < RT; r += 32) {
                     const bool live = r < nr && rok[r];
                     const float *lrow = LG + (int64_t)(r0 + (live ? r : 0)) * n;
+                    const uint32_t ldst = lbase + ((bs * RT + r) * KS + kc * 8 + hk) * 4;
+                    if (lg16) {  // 16-byte copies, zero-filled past the row's end
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) {
-                        const int j = j0 + kc * 8 + u;
-                        const bool in = live && j < n;
-                        cp_async4(lbase + ((bs * RT + r) * KS + kc * 8 + u) * 4, lrow + (in ? j : 0), in ? 4u : 0u);
+                        for (int h = 0; h < KPTH / 4; ++h) {
+                            const int j = j0 + kc * 8 + hk + 4 * h;
+                            const int nv = live ? min(max(n - j, 0), 4) : 0;
+                            cp_async16(ldst + 16 * h, lrow + (nv > 0 ? j : 0), 4u * (uint32_t)nv);
+                        }
+                    } else {
+#pragma unroll
+                        for (int u = 0; u < KPTH; ++u) {
+                            const int j = j0 + kc * 8 + hk + u;
+                            const bool in = live && j < n;
+                            cp_async4(ldst + 4 * u, lrow + (in ? j : 0), in ? 4u : 0u);
+                        }
                     }
                 }
             }
@@ -226,11 +248,14 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
         // this thread's row: thresholds, softmax statistics and the band rows of its chunk
         const bool live = rr0 < nr && rok[rr0];
         const float Mr = live ? rowM[rr0] : 0.f, Zr = live ? rowZi[rr0] : 0.f;
-        uint32_t mtk[4];
+        // thresholds as floats: key > T <=> x > xT and key == T <=> x == xT
+        // for finite logits (order keys fold -0 onto +0, as float compares do)
+        float mxt[4];
         int mti[4];
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
-            mtk[b] = live ? rtk[rr0][b] : 0u;
+            const uint32_t tk = live ? rtk[rr0][b] : 0u;
+            mxt[b] = __uint_as_float((tk & 0x80000000u) ? (tk & 0x7fffffffu) : ~tk);
             mti[b] = live ? rti[rr0][b] : -1;
         }
         uint32_t boff[5];
@@ -254,63 +279,81 @@ __global__ void __launch_bounds__(NT, 1) k_long_pv_tc(const TcArgs a)
             uint8_t *aslot = sA + as * A_SLOT_BYTES;
             const int j0 = it * KS;
             if (rr0 < RT) {  // (threads past the tile's rows have no band rows)
-                const float *lr = sL + (bs * RT + rr0) * KS + kc * 8;
-                // zero this thread's chunk of every band row, then put each key's three
-                // bf16 terms into the row of its own band (same thread: ordered)
+                const float *lr = sL + (bs * RT + rr0) * KS + kc * 8 + hk;
+                // this thread's KPTH keys of its row: mass, band and three bf16
+                // terms (keys past the row's end or in a dead row get mass 0)
+                float xs[KPTH];
 #pragma unroll
-                for (int b = 0; b < 5; ++b)
-                    if (b < nbb)
+                for (int q = 0; q < KPTH / 4; ++q) {
+                    const float4 x4 = *reinterpret_cast<const float4 *>(lr + 4 * q);
+                    xs[4 * q] = x4.x, xs[4 * q + 1] = x4.y, xs[4 * q + 2] = x4.z, xs[4 * q + 3] = x4.w;
+                }
+                uint32_t h16[KPTH], m16[KPTH], l16[KPTH];
+                int bdv[KPTH];
 #pragma unroll
-                        for (int sp = 0; sp < NSPLIT; ++sp)
-                            *reinterpret_cast<uint4 *>(aslot + sp * A_SPLIT_BYTES + boff[b]) = make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const int j = j0 + kc * 8 + u;
-                    if (!(live && j < n)) continue;
-                    const float x = lr[u];
-                    const float p = expf(x - Mr) * Zr;
-                    const uint32_t key = order_key(x);
+                for (int u = 0; u < KPTH; ++u) {
+                    const int j = j0 + kc * 8 + hk + u;
+                    const float x = xs[u];
+                    const float p = (live && j < n) ? __expf(x - Mr) * Zr : 0.f;
                     int bd = 0;
 #pragma unroll
                     for (int b = 0; b < 4; ++b)
-                        if (b < nb) bd += !(key > mtk[b] || (key == mtk[b] && j <= mti[b]));
+                        if (b < nb) bd += !(x > mxt[b] || (x == mxt[b] && j <= mti[b]));
+                    bdv[u] = bd;
 #pragma unroll
-                    for (int b = 0; b < 5; ++b) bm[0][b] += bd == b ? p : 0.f;
-                    const uint32_t h16 = bf16_bits_rn(p);
-                    const float r1 = p - __uint_as_float(h16 << 16);
-                    const uint32_t m16 = bf16_bits_rn(r1);
-                    const uint32_t l16 = bf16_bits_rn(r1 - __uint_as_float(m16 << 16));
-                    const uint32_t off = (bd == 0 ? boff[0] : bd == 1 ? boff[1] : bd == 2 ? boff[2]
-                                          : bd == 3 ? boff[3] : boff[4]) + 2u * u;
-                    *reinterpret_cast<uint16_t *>(aslot + off) = (uint16_t)h16;
-                    *reinterpret_cast<uint16_t *>(aslot + A_SPLIT_BYTES + off) = (uint16_t)m16;
-                    *reinterpret_cast<uint16_t *>(aslot + 2 * A_SPLIT_BYTES + off) = (uint16_t)l16;
+                    for (int b = 0; b < 5; ++b) bm[b] += bd == b ? p : 0.f;
+                    h16[u] = bf16_bits_rn(p);
+                    const float r1 = p - __uint_as_float(h16[u] << 16);
+                    m16[u] = bf16_bits_rn(r1);
+                    l16[u] = bf16_bits_rn(r1 - __uint_as_float(m16[u] << 16));
+                }
+                // one vector per (band row, term): each key's terms in its own
+                // band's row, zeros in the others
+#pragma unroll
+                for (int b = 0; b < 5; ++b) {
+                    if (b >= nbb) continue;
+                    uint32_t wh[KPTH / 2], wm[KPTH / 2], wl[KPTH / 2];
+#pragma unroll
+                    for (int q = 0; q < KPTH / 2; ++q) {
+                        const bool e0 = bdv[2 * q] == b, e1 = bdv[2 * q + 1] == b;
+                        wh[q] = (e0 ? h16[2 * q] : 0u) | ((e1 ? h16[2 * q + 1] : 0u) << 16);
+                        wm[q] = (e0 ? m16[2 * q] : 0u) | ((e1 ? m16[2 * q + 1] : 0u) << 16);
+                        wl[q] = (e0 ? l16[2 * q] : 0u) | ((e1 ? l16[2 * q + 1] : 0u) << 16);
+                    }
+                    uint8_t *dst = aslot + boff[b] + 2 * hk;
+                    if constexpr (KPTH == 8) {
+                        *reinterpret_cast<uint4 *>(dst) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+                        *reinterpret_cast<uint4 *>(dst + A_SPLIT_BYTES) = make_uint4(wm[0], wm[1], wm[2], wm[3]);
+                        *reinterpret_cast<uint4 *>(dst + 2 * A_SPLIT_BYTES) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+                    } else {
+                        *reinterpret_cast<uint2 *>(dst) = make_uint2(wh[0], wh[1]);
+                        *reinterpret_cast<uint2 *>(dst + A_SPLIT_BYTES) = make_uint2(wm[0], wm[1]);
+                        *reinterpret_cast<uint2 *>(dst + 2 * A_SPLIT_BYTES) = make_uint2(wl[0], wl[1]);
+                    }
                 }
             }
             tc::fence_async_smem();
             tc::mbar_arrive(&full[bs]);
-            if (it >= 2) flush(it - 2);
+            if (it >= 2 && chunk_end(it - 2)) flush(it - 2);
         }
-        for (int st = nst - 2 < 0 ? 0 : nst - 2; st < nst; ++st) flush(st);
-        // band masses: the 8 threads of a row sit in consecutive lanes
+        for (int st = nst - 2 < 0 ? 0 : nst - 2; st < nst; ++st)
+            if (chunk_end(st)) flush(st);
+        // band masses: the TPR threads of a row sit in consecutive lanes
 #pragma unroll
-        for (int q = 0; q < 2; ++q)
+        for (int b = 0; b < 5; ++b) {
+            float v = bm[b];
 #pragma unroll
-            for (int b = 0; b < 5; ++b) {
-                float v = bm[q][b];
-                v += __shfl_xor_sync(FW_FULL, v, 1);
-                v += __shfl_xor_sync(FW_FULL, v, 2);
-                v += __shfl_xor_sync(FW_FULL, v, 4);
-                bm[q][b] = v;
-            }
-        if (kc == 0 && rr0 < RT)
-            for (int b = 0; b < 5; ++b) bmass[rr0][b] = bm[0][b];
+            for (int o = 1; o < TPR; o <<= 1) v += __shfl_xor_sync(FW_FULL, v, o);
+            bm[b] = v;
+        }
+        if (ptid % TPR == 0 && rr0 < RT)
+            for (int b = 0; b < 5; ++b) bmass[rr0][b] = bm[b];
         // accumulators -> shared for the per-row epilogue (the stage buffers are idle now)
         if (!ok) atomicOr(&s_err, 1);
         {
             const int m = quarter * 32 + lane;
 #pragma unroll
-            for (int i = 0; i < D / 2; ++i) acc[m * (D + 1) + half * (D / 2) + i] = racc[i];
+            for (int i = 0; i < 32; ++i) acc[m * (D + 1) + part * 32 + i] = racc[i];
         }
     }
     tc::fence_before_sync();
@@ -412,11 +455,11 @@ fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_ou
     if (R.d == 128) {
         const size_t smem = tc_smem<128>(a.RT);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_pv_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        FW_LAUNCH(k_long_pv_tc<128>, grid, NT, smem, s, a);
+        FW_LAUNCH(k_long_pv_tc<128>, grid, pv_threads<128>(), smem, s, a);
     } else {
         const size_t smem = tc_smem<64>(a.RT);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_pv_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        FW_LAUNCH(k_long_pv_tc<64>, grid, NT, smem, s, a);
+        FW_LAUNCH(k_long_pv_tc<64>, grid, pv_threads<64>(), smem, s, a);
     }
     return FW_OK;
 }
