@@ -190,7 +190,7 @@ fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t
  * cudaMalloc would synchronise the device -- and cannot provide the
  * workspace fw_contour_alloc asks for.  This variant takes the same
  * arguments minus the workspace and uses a scratch area compiled into the
- * library instead (about 50 KB, held by every GPU that loads the library
+ * library instead (about 83 KB, held by every GPU that loads the library
  * until the process exits).
  *   - cells must be <= FW_CONTOUR_NOALLOC_MAX_CELLS, otherwise the call
  *     returns FW_ERR_WORKSPACE and launches nothing; the other argument

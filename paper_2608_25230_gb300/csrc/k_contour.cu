@@ -7,8 +7,11 @@
 // (score desc, cell asc, position asc), so ties at tau are split exactly.
 //
 // tau is found by a global radix select (4 passes x 8 bits).  Every pass is a
-// histogram launch over all cells followed by a one-block scan launch: no
-// kernel ever waits on another block.  Then per-cell counts, an exclusive
+// histogram launch (a block per cell) into its own global histogram; each
+// block of the next launch derives the digits fixed so far from those
+// histograms (a warp scan), so no kernel ever waits on another block.  The same passes carry each cell's own
+// top-uniform_s select (the uniform-budget dropped mass): its histogram is
+// the cell's alone, so the cell's block fixes its digit at the end of the pass.  Then per-cell counts, an exclusive
 // prefix sum into ragged offsets, and per-cell ordered compaction of the kept
 // positions.  The compaction copy moves 16-byte vectors, a row per 16 lanes.
 #include <algorithm>
@@ -32,7 +35,7 @@ struct CArgs {
     const float *scores;
     int cells, T, F;
     int64_t K;
-    uint32_t *hist;      // [256]
+    uint32_t *hist;      // [4][256] global histograms of the four passes
     CState *st;          // [1]
     int32_t *gt;         // [cells] non-floor keys above tau
     int32_t *eq;         // [cells] non-floor keys equal to tau
@@ -43,6 +46,8 @@ struct CArgs {
     float *tau;
     float *dropped_uniform, *dropped_alloc;
     int uniform_s;
+    uint32_t *uprefix;   // [cells] bits of the cell's uniform-budget threshold fixed so far
+    uint32_t *urem;      // [cells] rank still to find inside that prefix (0: no uniform set)
 };
 
 __global__ void k_c_init(CArgs a)
@@ -52,58 +57,139 @@ __global__ void k_c_init(CArgs a)
         a.st->rem = (uint32_t)a.K;
         a.st->K_lo = (uint32_t)a.K;
     }
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) a.hist[i] = 0u;
+    for (int i = threadIdx.x; i < 4 * 256; i += blockDim.x) a.hist[i] = 0u;
+    const uint32_t su = a.dropped_uniform ? (uint32_t)max(min(a.uniform_s, a.T), 0) : 0u;
+    for (int c = threadIdx.x; c < a.cells; c += blockDim.x) {
+        a.uprefix[c] = 0u;
+        a.urem[c] = su;
+    }
 }
 
-// histogram of digit `pass` among non-floor keys matching the prefix
-__global__ void __launch_bounds__(CT) k_c_hist(CArgs a, int pass)
+// The radix state after `npass` passes: the bits of tau's key fixed so far
+// and the rank still to find inside them, from the passes' global
+// histograms.  One warp; lane l takes bins 255 - 8l .. 248 - 8l of a pass.
+__device__ __forceinline__ void select_state(const uint32_t *hist4, int npass, uint32_t K, uint32_t &prefix,
+                                             uint32_t &rem)
 {
-    __shared__ uint32_t h[256];
-    for (int i = threadIdx.x; i < 256; i += CT) h[i] = 0u;
+    const int lane = threadIdx.x & 31;
+    prefix = 0u;
+    rem = K;
+    for (int p = 0; p < npass; ++p) {
+        uint32_t c[8], loc = 0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            c[i] = hist4[p * 256 + 255 - 8 * lane - i];
+            loc += c[i];
+        }
+        uint32_t inc = loc;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(FW_FULL, inc, o);
+            if (lane >= o) inc += y;
+        }
+        const uint32_t exc = inc - loc;
+        const bool mine = exc < rem && rem <= inc;
+        uint32_t v = 0u, nr = 0u;
+        if (mine) {
+            uint32_t cum = exc;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                if (v == 0u && cum + c[i] >= rem) {
+                    v = 256u + 255u - 8u * lane - i;  // (+256: found)
+                    nr = rem - cum;
+                }
+                cum += c[i];
+            }
+        }
+        const int src = __ffs(__ballot_sync(FW_FULL, mine)) - 1;
+        v = __shfl_sync(FW_FULL, v, src < 0 ? 0 : src);
+        nr = __shfl_sync(FW_FULL, nr, src < 0 ? 0 : src);
+        prefix |= (v & 255u) << (24 - 8 * p);
+        rem = nr;
+    }
+}
+
+// One radix pass, a block per cell.  The cell's non-floor keys matching the
+// global prefix go to the global histogram of digit `pass` (the threshold
+// tau); all of the cell's keys matching its own uniform prefix go to a cell
+// histogram, which the block scans at once to fix the digit of the cell's own
+// top-uniform_s threshold (the uniform-budget dropped mass).
+constexpr int CPT = 512;  // threads of a pass block
+__global__ void __launch_bounds__(CPT) k_c_pass(CArgs a, int pass)
+{
+    __shared__ uint32_t hg[256], hu[256];
+    __shared__ uint32_t s_prefix;
+    for (int i = threadIdx.x; i < 256; i += CPT) hg[i] = hu[i] = 0u;
+    const bool glob = a.K > 0;
+    if (threadIdx.x < 32) {  // the global state after the earlier passes
+        uint32_t pf = 0u, rm = 0u;
+        if (glob) select_state(a.hist, pass, (uint32_t)a.K, pf, rm);
+        if (threadIdx.x == 0) s_prefix = pf;
+    }
     __syncthreads();
+    const int c = blockIdx.x;
     const int shift = 24 - 8 * pass;
     const uint32_t pmask = pass == 0 ? 0u : (0xffffffffu << (32 - 8 * pass));
-    const uint32_t prefix = a.st->prefix;
-    const int64_t per_cell = a.T - a.F;
-    const int64_t total = (int64_t)a.cells * per_cell;
-    for (int64_t e = (int64_t)blockIdx.x * CT + threadIdx.x; e < total; e += (int64_t)gridDim.x * CT) {
-        const int64_t c = e / per_cell, j = e - c * per_cell;
-        const uint32_t key = order_key(__ldg(a.scores + c * a.T + j));
-        if ((key & pmask) == prefix) atomicAdd(&h[(key >> shift) & 255u], 1u);
+    const uint32_t prefix = s_prefix;
+    const uint32_t upre = a.uprefix[c];
+    const bool uni = a.urem[c] > 0u;
+    const int nf = a.T - a.F;
+    const float *sc = a.scores + (int64_t)c * a.T;
+    auto visit = [&](int j, float x) {
+        const uint32_t key = order_key(x);
+        const uint32_t dg = (key >> shift) & 255u;
+        if (glob && j < nf && (key & pmask) == prefix) atomicAdd(&hg[dg], 1u);
+        if (uni && (key & pmask) == upre) atomicAdd(&hu[dg], 1u);
+    };
+    if ((a.T & 3) == 0 && (reinterpret_cast<uintptr_t>(sc) & 15) == 0) {
+        for (int q = threadIdx.x; q < a.T / 4; q += CPT) {
+            const float4 v = __ldg(reinterpret_cast<const float4 *>(sc) + q);
+            visit(4 * q, v.x);
+            visit(4 * q + 1, v.y);
+            visit(4 * q + 2, v.z);
+            visit(4 * q + 3, v.w);
+        }
+    } else {
+        for (int j = threadIdx.x; j < a.T; j += CPT) visit(j, __ldg(sc + j));
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < 256; i += CT)
-        if (h[i]) atomicAdd(&a.hist[i], h[i]);
-}
-
-__global__ void k_c_scan(CArgs a, int pass)
-{
-    // one thread: walk bins from the top
-    if (threadIdx.x == 0) {
-        const int shift = 24 - 8 * pass;
-        uint32_t cum = 0, rem = a.st->rem;
+    if (glob)
+        for (int i = threadIdx.x; i < 256; i += CPT)
+            if (hg[i]) atomicAdd(&a.hist[pass * 256 + i], hg[i]);
+    if (uni && threadIdx.x == 0) {
+        uint32_t cum = 0, rem = a.urem[c];
         for (int v = 255; v >= 0; --v) {
-            const uint32_t c = a.hist[v];
-            if (cum + c >= rem) {
-                a.st->prefix |= (uint32_t)v << shift;
-                a.st->rem = rem - cum;
+            const uint32_t cc = hu[v];
+            if (cum + cc >= rem) {
+                a.uprefix[c] = upre | ((uint32_t)v << shift);
+                a.urem[c] = rem - cum;
                 break;
             }
-            cum += c;
+            cum += cc;
         }
     }
-    __syncthreads();
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) a.hist[i] = 0u;
 }
 
 // per cell: keys above / equal to tau among the non-floor positions
 __global__ void __launch_bounds__(CT) k_c_count(CArgs a)
 {
     __shared__ int s_gt, s_eq;
+    __shared__ uint32_t s_tk;
     const int c = blockIdx.x;
-    if (threadIdx.x == 0) s_gt = s_eq = 0;
+    if (threadIdx.x < 32) {  // tau's key from the four passes; block 0 records it
+        uint32_t pf = 0u, rm = 0u;
+        if (a.K > 0) select_state(a.hist, 4, (uint32_t)a.K, pf, rm);
+        if (threadIdx.x == 0) {
+            s_tk = pf;
+            s_gt = s_eq = 0;
+            if (c == 0) {
+                a.st->prefix = pf;
+                a.st->rem = rm;
+            }
+        }
+    }
     __syncthreads();
-    const uint32_t tk = a.st->prefix;
+    const uint32_t tk = s_tk;
     int gt = 0, eq = 0;
     if (a.K > 0) {
         for (int j = threadIdx.x; j < a.T - a.F; j += CT) {
@@ -193,169 +279,108 @@ __global__ void __launch_bounds__(1024) k_c_offsets(CArgs a)
     }
 }
 
-// per cell: ordered compaction of kept positions + dropped mass of the allocation
-__global__ void __launch_bounds__(CT) k_c_emit(CArgs a)
+// exclusive and total sums over the warps of the values v[w] (w < NW), for
+// every thread of the block
+template <int NW>
+__device__ __forceinline__ void warp_counts(const int *v, int wid, int lane, int &before, int &total)
 {
-    __shared__ int wc[CT / 32], wt[CT / 32];
-    __shared__ double red[CT / 32], red2[CT / 32];
+    int x = lane < NW ? v[lane] : 0;
+    int inc = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(FW_FULL, inc, o);
+        if (lane >= o) inc += y;
+    }
+    before = __shfl_sync(FW_FULL, inc - x, wid);
+    total = __shfl_sync(FW_FULL, inc, 31);
+}
+
+// per cell, positions in order: the ordered compaction of the kept positions,
+// the dropped mass of the allocation, and the cell's own top-uniform_s set
+// (keys above its threshold, then the first equal ones in position order) with
+// the dropped mass outside it
+constexpr int CTE = 1024;  // threads of an emit block
+__global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
+{
+    constexpr int NW = CTE / 32;
+    __shared__ int wc[NW], wt[NW], wu[NW];
+    __shared__ double red[NW], red2[NW], red3[NW];
     const int c = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const uint32_t tk = a.st->prefix;
     const int take = a.take[c];
     const int64_t base = a.offsets[c];
+    const uint32_t uT = a.uprefix[c];
+    const int uwant = (int)a.urem[c];  // 0: no uniform set (every key dropped)
     const float *s = a.scores + (int64_t)c * a.T;
-    int written = 0, ties_seen = 0;
-    double tot = 0.0, drop = 0.0;
-    for (int j0 = 0; j0 < a.T; j0 += CT) {
+    const uint32_t lmask = (1u << lane) - 1u;
+    int written = 0, ties_seen = 0, uties_seen = 0;
+    // per-thread sums of T / CTE positive terms in fp32 (relative error below
+    // 1e-5); the sums over threads in fp64
+    float tot = 0.f, drop = 0.f, udrop = 0.f;
+    float xn = tid < a.T ? __ldg(s + tid) : 0.f;  // the next chunk's score, loaded a chunk ahead
+    for (int j0 = 0; j0 < a.T; j0 += CTE) {
         const int j = j0 + tid;
-        bool kept = false, tie = false;
-        float x = 0.f;
+        bool kept = false, tie = false, ukept = false, utie = false;
+        const float x = xn;
+        if (j + CTE < a.T) xn = __ldg(s + j + CTE);
         if (j < a.T) {
-            x = __ldg(s + j);
+            const uint32_t key = order_key(x);
             if (j >= a.T - a.F) {
                 kept = true;
             } else if (a.K > 0) {
-                const uint32_t key = order_key(x);
                 kept = key > tk;
                 tie = key == tk;
             }
+            if (uwant > 0) {
+                ukept = key > uT;
+                utie = key == uT;
+            }
         }
-        // rank of this tie among the cell's ties, in position order
-        const uint32_t tb = __ballot_sync(FW_FULL, tie);
-        if (lane == 0) wt[wid] = __popc(tb);
+        // ranks of the ties among the cell's ties, in position order
+        const uint32_t tb = __ballot_sync(FW_FULL, tie), ub = __ballot_sync(FW_FULL, utie);
+        if (lane == 0) {
+            wt[wid] = __popc(tb);
+            wu[wid] = __popc(ub);
+        }
         __syncthreads();
-        int tbefore = 0, ttotal = 0;
-        for (int w = 0; w < CT / 32; ++w) {
-            if (w < wid) tbefore += wt[w];
-            ttotal += wt[w];
-        }
-        if (tie) kept = (ties_seen + tbefore + __popc(tb & ((1u << lane) - 1u))) < take;
+        int tbefore, ttotal, ubefore, utotal;
+        warp_counts<NW>(wt, wid, lane, tbefore, ttotal);
+        warp_counts<NW>(wu, wid, lane, ubefore, utotal);
+        if (tie) kept = ties_seen + tbefore + __popc(tb & lmask) < take;
+        if (utie) ukept = uties_seen + ubefore + __popc(ub & lmask) < uwant;
         ties_seen += ttotal;
+        uties_seen += utotal;
         const uint32_t kb = __ballot_sync(FW_FULL, kept);
         if (lane == 0) wc[wid] = __popc(kb);
         __syncthreads();
-        int before = 0, total = 0;
-        for (int w = 0; w < CT / 32; ++w) {
-            if (w < wid) before += wc[w];
-            total += wc[w];
-        }
-        if (kept) a.kept_pos[base + written + before + __popc(kb & ((1u << lane) - 1u))] = j;
+        int before, total;
+        warp_counts<NW>(wc, wid, lane, before, total);
+        if (kept) a.kept_pos[base + written + before + __popc(kb & lmask)] = j;
         written += total;
         if (j < a.T) {
-            tot += (double)x;
-            if (!kept) drop += (double)x;
+            tot += x;
+            if (!kept) drop += x;
+            if (!ukept) udrop += x;
         }
-        __syncthreads();
+        __syncthreads();  // wt, wu, wc are rewritten by the next chunk
     }
-    tot = warp_sum_d(tot);
-    drop = warp_sum_d(drop);
+    const double tsum = warp_sum_d((double)tot), dsum = warp_sum_d((double)drop), usum = warp_sum_d((double)udrop);
     if (lane == 0) {
-        red[wid] = tot;
-        red2[wid] = drop;
-    }
-    __syncthreads();
-    if (tid == 0 && a.dropped_alloc) {
-        double t = 0.0, dd = 0.0;
-        for (int w = 0; w < CT / 32; ++w) {
-            t += red[w];
-            dd += red2[w];
-        }
-        a.dropped_alloc[c] = t > 0.0 ? (float)(dd / t) : 0.f;
-    }
-}
-
-// per cell: dropped mass outside the cell's own top-s set (ties -> lower position)
-__global__ void __launch_bounds__(CT) k_c_uniform(CArgs a)
-{
-    __shared__ uint32_t hist[256];
-    __shared__ uint32_t s_prefix, s_rem;
-    __shared__ uint32_t wcnt[CT / 32];
-    __shared__ int s_found;
-    __shared__ double red[CT / 32], red2[CT / 32];
-    const int c = blockIdx.x;
-    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-    const int T = a.T;
-    const float *s = a.scores + (int64_t)c * T;
-    const int su = a.uniform_s < T ? a.uniform_s : T;
-    uint32_t tk = 0u;
-    int ti = -1;
-    if (su > 0) {
-        if (tid == 0) {
-            s_prefix = 0u;
-            s_rem = (uint32_t)su;
-        }
-        uint32_t pmask = 0u;
-        for (int pass = 0; pass < 4; ++pass) {
-            const int shift = 24 - 8 * pass;
-            for (int i = tid; i < 256; i += CT) hist[i] = 0u;
-            __syncthreads();
-            const uint32_t pre = s_prefix;
-            for (int j = tid; j < T; j += CT) {
-                const uint32_t key = order_key(__ldg(s + j));
-                if ((key & pmask) == pre) atomicAdd(&hist[(key >> shift) & 255u], 1u);
-            }
-            __syncthreads();
-            if (tid == 0) {
-                uint32_t cum = 0, rem = s_rem;
-                for (int v = 255; v >= 0; --v) {
-                    const uint32_t cc = hist[v];
-                    if (cum + cc >= rem) {
-                        s_prefix |= (uint32_t)v << shift;
-                        s_rem = rem - cum;
-                        break;
-                    }
-                    cum += cc;
-                }
-            }
-            pmask |= 255u << shift;
-            __syncthreads();
-        }
-        tk = s_prefix;
-        const uint32_t want = s_rem;
-        if (tid == 0) s_found = -1;
-        __syncthreads();
-        uint32_t base = 0;
-        for (int j0 = 0; j0 < T; j0 += CT) {
-            const int j = j0 + tid;
-            const bool match = j < T && order_key(__ldg(s + j)) == tk;
-            const uint32_t bal = __ballot_sync(FW_FULL, match);
-            if (lane == 0) wcnt[wid] = __popc(bal);
-            __syncthreads();
-            uint32_t before = 0, total = 0;
-            for (int w = 0; w < CT / 32; ++w) {
-                if (w < wid) before += wcnt[w];
-                total += wcnt[w];
-            }
-            if (match && base + before + __popc(bal & ((1u << lane) - 1u)) + 1u == want) s_found = j;
-            __syncthreads();
-            base += total;
-            if (base >= want) break;
-        }
-        __syncthreads();
-        ti = s_found;
-    }
-    double tot = 0.0, drop = 0.0;
-    for (int j = tid; j < T; j += CT) {
-        const float x = __ldg(s + j);
-        const uint32_t key = order_key(x);
-        const bool kept = su > 0 && (key > tk || (key == tk && j <= ti));
-        tot += (double)x;
-        if (!kept) drop += (double)x;
-    }
-    tot = warp_sum_d(tot);
-    drop = warp_sum_d(drop);
-    if (lane == 0) {
-        red[wid] = tot;
-        red2[wid] = drop;
+        red[wid] = tsum;
+        red2[wid] = dsum;
+        red3[wid] = usum;
     }
     __syncthreads();
     if (tid == 0) {
-        double t = 0.0, dd = 0.0;
-        for (int w = 0; w < CT / 32; ++w) {
+        double t = 0.0, dd = 0.0, du = 0.0;
+        for (int w = 0; w < NW; ++w) {
             t += red[w];
             dd += red2[w];
+            du += red3[w];
         }
-        a.dropped_uniform[c] = t > 0.0 ? (float)(dd / t) : 0.f;
+        if (a.dropped_alloc) a.dropped_alloc[c] = t > 0.0 ? (float)(dd / t) : 0.f;
+        if (a.dropped_uniform) a.dropped_uniform[c] = t > 0.0 ? (float)(du / t) : 0.f;
     }
 }
 
@@ -386,7 +411,7 @@ __global__ void __launch_bounds__(256) k_compact(const uint4 *K, const uint4 *V,
 size_t contour_workspace(int cells, int T)
 {
     (void)T;
-    return align256(256 * 4) + align256(sizeof(CState)) + 3 * align256((size_t)cells * 4);
+    return align256(4 * 256 * 4) + align256(sizeof(CState)) + 5 * align256((size_t)cells * 4);
 }
 
 fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64_t total_budget, int uniform_s,
@@ -403,7 +428,7 @@ fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64
     if (a.K >= ((int64_t)1 << 32)) return FW_ERR_UNSUPPORTED;
     char *w = (char *)ws;
     a.hist = (uint32_t *)w;
-    w += align256(256 * 4);
+    w += align256(4 * 256 * 4);
     a.st = (CState *)w;
     w += align256(sizeof(CState));
     a.gt = (int32_t *)w;
@@ -411,6 +436,10 @@ fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64
     a.eq = (int32_t *)w;
     w += align256((size_t)cells * 4);
     a.take = (int32_t *)w;
+    w += align256((size_t)cells * 4);
+    a.uprefix = (uint32_t *)w;
+    w += align256((size_t)cells * 4);
+    a.urem = (uint32_t *)w;
     a.counts = counts;
     a.offsets = offsets;
     a.kept_pos = kept_pos;
@@ -418,19 +447,13 @@ fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64
     a.dropped_uniform = dropped_uniform;
     a.dropped_alloc = dropped_alloc;
     a.uniform_s = uniform_s;
-    FW_LAUNCH(k_c_init, 1, 256, 0, s, a);
-    if (a.K > 0) {
-        const int64_t keys = (int64_t)cells * (T - a.F);
-        const unsigned hb = (unsigned)std::max<int64_t>(1, std::min<int64_t>(152 * 8, (keys + CT - 1) / CT));
-        for (int pass = 0; pass < 4; ++pass) {
-            FW_LAUNCH(k_c_hist, hb, CT, 0, s, a, pass);
-            FW_LAUNCH(k_c_scan, 1, 256, 0, s, a, pass);
-        }
+    FW_LAUNCH(k_c_init, 1, 1024, 0, s, a);
+    if (a.K > 0 || (dropped_uniform && uniform_s > 0)) {
+        for (int pass = 0; pass < 4; ++pass) FW_LAUNCH(k_c_pass, (unsigned)cells, CPT, 0, s, a, pass);
     }
     FW_LAUNCH(k_c_count, (unsigned)cells, CT, 0, s, a);
     FW_LAUNCH(k_c_offsets, 1, 1024, 0, s, a);
-    FW_LAUNCH(k_c_emit, (unsigned)cells, CT, 0, s, a);
-    if (dropped_uniform) FW_LAUNCH(k_c_uniform, (unsigned)cells, CT, 0, s, a);
+    FW_LAUNCH(k_c_emit, (unsigned)cells, CTE, 0, s, a);
     return FW_OK;
 }
 
@@ -454,8 +477,8 @@ fw_status ragged_compact(const void *K, const void *V, int cells, int T, int row
 namespace fw {
 namespace {
 
-constexpr size_t kNoallocBytes = 256 * 4 + 256 + 3 * (size_t)FW_CONTOUR_NOALLOC_MAX_CELLS * 4;  // >= contour_workspace
-static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocBytes + 3 * 256];
+constexpr size_t kNoallocBytes = 4 * 256 * 4 + 256 + 5 * (size_t)FW_CONTOUR_NOALLOC_MAX_CELLS * 4;  // >= contour_workspace
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocBytes + 5 * 256];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_noalloc_mu;
