@@ -308,17 +308,26 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
                     l16[u] = bf16_bits_rn(r1 - __uint_as_float(m16[u] << 16));
                 }
                 // one vector per (band row, term): each key's terms in its own
-                // band's row, zeros in the others
+                // band's row, zeros in the others.  Keys 2q and 2q + 1 share a
+                // 32-bit word; a 2 x 16-bit compare of their bands gives the mask.
+                uint32_t ph[KPTH / 2], pm[KPTH / 2], pl[KPTH / 2], pb[KPTH / 2];
+#pragma unroll
+                for (int q = 0; q < KPTH / 2; ++q) {
+                    ph[q] = h16[2 * q] | (h16[2 * q + 1] << 16);
+                    pm[q] = m16[2 * q] | (m16[2 * q + 1] << 16);
+                    pl[q] = l16[2 * q] | (l16[2 * q + 1] << 16);
+                    pb[q] = (uint32_t)bdv[2 * q] | ((uint32_t)bdv[2 * q + 1] << 16);
+                }
 #pragma unroll
                 for (int b = 0; b < 5; ++b) {
                     if (b >= nbb) continue;
                     uint32_t wh[KPTH / 2], wm[KPTH / 2], wl[KPTH / 2];
 #pragma unroll
                     for (int q = 0; q < KPTH / 2; ++q) {
-                        const bool e0 = bdv[2 * q] == b, e1 = bdv[2 * q + 1] == b;
-                        wh[q] = (e0 ? h16[2 * q] : 0u) | ((e1 ? h16[2 * q + 1] : 0u) << 16);
-                        wm[q] = (e0 ? m16[2 * q] : 0u) | ((e1 ? m16[2 * q + 1] : 0u) << 16);
-                        wl[q] = (e0 ? l16[2 * q] : 0u) | ((e1 ? l16[2 * q + 1] : 0u) << 16);
+                        const uint32_t msk = __vcmpeq2(pb[q], (uint32_t)b * 0x00010001u);
+                        wh[q] = ph[q] & msk;
+                        wm[q] = pm[q] & msk;
+                        wl[q] = pl[q] & msk;
                     }
                     uint8_t *dst = aslot + boff[b] + 2 * hk;
                     if constexpr (KPTH == 8) {
