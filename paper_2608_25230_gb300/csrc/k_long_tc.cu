@@ -81,11 +81,13 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
     constexpr int TPR = NPROD / MAXRT;  // producer threads per row
     constexpr int KPTH = KS / TPR;      // keys per producer thread and stage (4 or 8)
     constexpr int B_SLOT_BYTES = D * 128;  // KS keys x D bf16
-    constexpr uint32_t TCOLS = NACC * D <= 256 ? 256u : 512u;  // TMEM columns (a power of two)
+    constexpr int MCOL = NACC * D;  // first TMEM column of the band-mass accumulators (16 per buffer)
+    constexpr uint32_t TCOLS = NACC * (D + 16) <= 256 ? 256u : 512u;  // TMEM columns (a power of two)
     constexpr int NC = D / 8;              // 16-byte chunks per V row
     extern __shared__ uint8_t smraw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~(uintptr_t)1023);
-    uint8_t *sA = sm;                                  // [ASLOTS][NSPLIT][TM x 128 B]
+    uint8_t *sOnes = sm;                               // [16 x 128 B] bf16 ones: B of the band-mass MMA
+    uint8_t *sA = sm + 2048;                           // [ASLOTS][NSPLIT][TM x 128 B]
     uint8_t *sB = sA + ASLOTS * A_SLOT_BYTES;          // [BSLOTS][D/64][KS x 128 B]
     float *sL = reinterpret_cast<float *>(sB + BSLOTS * B_SLOT_BYTES);  // [BSLOTS][RT][KS] raw logits
     float *acc = reinterpret_cast<float *>(sA);       // epilogue: [TM][D + 1]
@@ -134,7 +136,12 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
         for (int x = 0; x < NACC; ++x) tc::mbar_init(&accfree[x], NPROD);
         tc::mbar_init_fence();
     }
-    // rows of A past nbb * RT stay zero in every slot
+    // rows of A past nbb * RT stay zero in every slot; the ones tile is
+    // constant (any swizzle of it reads 1.0)
+    for (int e = tid; e < 2048 / 16; e += NT)
+        reinterpret_cast<uint4 *>(sOnes)[e] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    if (tid < MAXRT)
+        for (int b = 0; b < 5; ++b) bmass[tid][b] = 0.f;
     for (int e = tid; e < ASLOTS * NSPLIT * TM * 8; e += NT) {
         const int m = (e / 8) % TM;
         if (m >= nbb * RT) reinterpret_cast<uint4 *>(sA)[e] = make_uint4(0u, 0u, 0u, 0u);
@@ -150,7 +157,8 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
         // ---------------------------------------------------------- MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_bf16_f32(TM, D, false, true);
-            const uint32_t a0 = tc::smem_u32(sA), b0 = tc::smem_u32(sB);
+            constexpr uint32_t idesc_m = tc::idesc_bf16_f32(TM, 16, false, false);
+            const uint32_t a0 = tc::smem_u32(sA), b0 = tc::smem_u32(sB), o0 = tc::smem_u32(sOnes);
             bool ok = true;
             for (int it = 0; it < nst && ok; ++it) {
                 const int bs = it % BSLOTS, as = it % ASLOTS;
@@ -163,6 +171,7 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
                 if (!ok) break;
                 tc::fence_after_sync();
                 const uint32_t dacc = taddr + (uint32_t)(((it / CH) % NACC) * D);
+                const uint32_t dmass = taddr + (uint32_t)(MCOL + ((it / CH) % NACC) * 16);
                 const bool fresh = it % CH == 0;  // first stage of a chunk overwrites the buffer
 #pragma unroll
                 for (int ks = 0; ks < KS / 16; ++ks) {
@@ -172,6 +181,9 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
                         const uint64_t ad =
                             tc::sdesc_sw128(a0 + as * A_SLOT_BYTES + sp * A_SPLIT_BYTES + ks * 32, 16, 1024);
                         tc::mma_bf16(dacc, ad, bd, idesc, !fresh || ks > 0 || sp > 0);
+                        // band masses: the same A tile times a K x 16 tile of ones
+                        tc::mma_bf16(dmass, ad, tc::sdesc_sw128(o0 + ks * 32, 16, 1024), idesc_m,
+                                     !fresh || ks > 0 || sp > 0);
                     }
                 }
                 tc::commit(&empty[bs]);
@@ -185,9 +197,6 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
         const int rr0 = ptid / TPR;                 // the row handled (tiles have at most 32 rows)
         const int kc = (ptid % TPR) * KPTH / 8;     // 8-key chunk of the stage
         const int hk = (ptid % TPR) * KPTH % 8;     // first key of this thread in the chunk
-        float bm[5];
-#pragma unroll
-        for (int b = 0; b < 5; ++b) bm[b] = 0.f;
         bool ok = true;
         const uint32_t bbase = tc::smem_u32(sB), lbase = tc::smem_u32(sL);
         // this thread's accumulator entries: TMEM lane 32 (wid % 4) + lane, the
@@ -196,6 +205,7 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
         float racc[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) racc[i] = 0.f;
+        float rmass = 0.f;  // band mass of TMEM lane 32 quarter + lane (warps of part 0)
         // stage st closes its chunk: the chunk's buffer is added once its MMAs completed
         auto chunk_end = [&](int st) { return st % CH == CH - 1 || st == nst - 1; };
         auto flush = [&](int st) {
@@ -207,6 +217,8 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
             tc::ld32(base, v);
 #pragma unroll
             for (int i = 0; i < 32; ++i) racc[i] += v[i];
+            if (part == 0)
+                rmass += tc::ld1(taddr + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(MCOL + ((st / CH) % NACC) * 16));
             tc::fence_before_sync();
             tc::mbar_arrive(&accfree[(st / CH) % NACC]);
         };
@@ -300,8 +312,6 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
                     for (int b = 0; b < 4; ++b)
                         if (b < nb) bd += !(x > mxt[b] || (x == mxt[b] && j <= mti[b]));
                     bdv[u] = bd;
-#pragma unroll
-                    for (int b = 0; b < 5; ++b) bm[b] += bd == b ? p : 0.f;
                     h16[u] = bf16_bits_rn(p);
                     const float r1 = p - __uint_as_float(h16[u] << 16);
                     m16[u] = bf16_bits_rn(r1);
@@ -347,16 +357,11 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
         }
         for (int st = nst - 2 < 0 ? 0 : nst - 2; st < nst; ++st)
             if (chunk_end(st)) flush(st);
-        // band masses: the TPR threads of a row sit in consecutive lanes
-#pragma unroll
-        for (int b = 0; b < 5; ++b) {
-            float v = bm[b];
-#pragma unroll
-            for (int o = 1; o < TPR; o <<= 1) v += __shfl_xor_sync(FW_FULL, v, o);
-            bm[b] = v;
+        // band masses from the ones MMA: TMEM lane m = (band, row) = (m / RT, m % RT)
+        if (part == 0) {
+            const int m = quarter * 32 + lane;
+            if (m < nbb * RT) bmass[m % RT][m / RT] = rmass;
         }
-        if (ptid % TPR == 0 && rr0 < RT)
-            for (int b = 0; b < 5; ++b) bmass[rr0][b] = bm[b];
         // accumulators -> shared for the per-row epilogue (the stage buffers are idle now)
         if (!ok) atomicOr(&s_err, 1);
         {
@@ -439,7 +444,7 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
 
 template <int D> size_t tc_smem(int RT)
 {
-    return 1024 + (size_t)ASLOTS * A_SLOT_BYTES + (size_t)BSLOTS * D * 128 + (size_t)BSLOTS * RT * KS * 4;
+    return 1024 + 2048 + (size_t)ASLOTS * A_SLOT_BYTES + (size_t)BSLOTS * D * 128 + (size_t)BSLOTS * RT * KS * 4;
 }
 
 }  // namespace

@@ -136,5 +136,17 @@ __device__ __forceinline__ void ld32(uint32_t taddr, float (&v)[32])
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// One fp32 column of this warp's 32 TMEM lanes (lane i reads TMEM lane
+// (taddr >> 16) + i), waited on in the same asm statement.
+__device__ __forceinline__ float ld1(uint32_t taddr)
+{
+    uint32_t r;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];\n\ttcgen05.wait::ld.sync.aligned;"
+                 : "=r"(r)
+                 : "r"(taddr)
+                 : "memory");
+    return __uint_as_float(r);
+}
+
 }  // namespace tc
 }  // namespace fw
