@@ -5,7 +5,7 @@ import pytest
 
 import oracle
 import workloads
-from tests.parity import assert_close, np_, row_onorm
+from tests.parity import assert_close, close, np_, row_onorm
 from tests.test_gpu_small import rows_batch
 
 pytestmark = pytest.mark.gpu
@@ -175,3 +175,105 @@ def test_swap_mixed_profiles_reduced(fw):
     for b in workloads.mixed_profiles(seed=2, rows_scale=6e-4,
                                       profiles=(("A", 36864, 64, 1024), ("B", 24192, 128, 4096))):
         check_swap_long(fw, b)
+
+
+class _PickRagged:
+    """Host copy of a few rows of a device RowBatch whose groups differ in n."""
+
+    def __init__(self, b, rows_index):
+        self.rows_index = np.asarray(rows_index)
+        R = b.rows_per_group
+        d = b.d
+        n_host = np.asarray(b.n_host)
+        lo = b.logit_off.cpu().numpy() if hasattr(b.logit_off, "cpu") else np.asarray(b.logit_off)
+        vo = b.v_off.cpu().numpy() if hasattr(b.v_off, "cpu") else np.asarray(b.v_off)
+        Ls, Vs, ns = [], [], []
+        for r in self.rows_index:
+            g = int(r) // R
+            n = int(n_host[g])
+            off = int(lo[g]) + (int(r) - g * R) * n
+            Ls.append(b.logits[off:off + n].cpu().numpy())
+            Vs.append(b.v[int(vo[g]):int(vo[g]) + n * d].view(torch.int16).cpu().numpy().view(np.uint16))
+            ns.append(n)
+        ns = np.asarray(ns, np.int32)
+        k = b.k[torch.as_tensor(self.rows_index, device=b.k.device)].cpu().numpy()
+        batch = workloads.RowBatch(rows_per_group=1, d=d, n=ns, logits=np.concatenate(Ls),
+                                   logit_off=np.concatenate([[0], np.cumsum(ns)[:-1]]).astype(np.int64),
+                                   v=np.concatenate(Vs),
+                                   v_off=np.concatenate([[0], np.cumsum(ns.astype(np.int64) * d)[:-1]]).astype(np.int64),
+                                   v_dtype="bf16", k=k, nb=k.shape[1], n_host=ns)
+        self.H = oracle.HostRows(batch)
+
+
+def _compare_swap(sw, o, sel, on):
+    """Swap outputs of the sampled rows against the oracle.  Over ~30 rounds of
+    up to 8,192 x 32 candidate pairs, most (row, budget) chains contain a
+    decision closer than 1e-6 relative (the oracle's `margin`), after which the
+    greedy paths may part; those chains are checked for validity only (the
+    refined gap does not exceed the top-k gap), the others exactly."""
+    from tests.parity import NEAR_TIE
+
+    exempt = (o["margin"] < NEAR_TIE) | (o["pool_margin"] < NEAR_TIE)
+    strict = ~exempt
+    assert_close(np_(sw["topk_gap"])[sel], o["topk_gap"], on, "swap topk_gap")
+    for key in ("n_swaps", "capped", "swap_out", "swap_in"):
+        np.testing.assert_array_equal(np_(sw[key])[sel][strict], o[key][strict])
+    rg = np_(sw["refined_gap"])[sel]
+    ok = close(rg, o["refined_gap"], on)
+    assert np.all(ok[strict]), "refined_gap differs on a chain without near-ties"
+    assert np.all(rg <= np_(sw["topk_gap"])[sel] * (1 + 1e-6))
+    return int(strict.sum())
+
+
+def test_swap_long_rows_full_scale_sampled(fw):
+    """The swap rule on the measured long-row workload (4,096 rows x 32,768
+    keys, budgets 2,048 / 4,096 / 8,192, E = 32, at most 64 swaps), as timed;
+    four rows re-run by the oracle, properties on every row."""
+    b = workloads.long_rows(seed=0, backend="torch", device="cuda")
+    rows = fw.rows_from_batch(b)
+    g = fw.dense_and_topk_gap(rows, b.k)
+    sw = fw.swap_refine(rows, b.k, g, E=32, max_swaps=64)
+    torch.cuda.synchronize()
+    pick = _Pick(b, np.sort(np.random.default_rng(1).choice(rows.num_rows, 4, replace=False)))
+    o = oracle.swap_refine(pick.H, E=32, max_swaps=64)
+    on = row_onorm(oracle.dense_and_topk_gap(pick.H)["o"])
+    _compare_swap(sw, o, pick.rows_index, on)
+    # on every row: finite, never worse than the top-k set, never capped
+    rg, tg = np_(sw["refined_gap"]), np_(sw["topk_gap"])
+    assert np.all(np.isfinite(rg)) and np.all(rg <= tg * (1 + 1e-6))
+    assert np.all(np_(sw["capped"]) == 0)
+
+
+def test_mixed_profiles_full_scale_sampled(fw):
+    """The mixed-profile sweep at full size (168,192 rows in GQA groups of 4,
+    n from 1,024 to 16,384, bf16 V), profile by profile: gap and swap rule on
+    every row, three rows of each profile re-run by the oracle, properties on
+    every row."""
+    rng = np.random.default_rng(5)
+    # one profile at a time keeps the device footprint of generation below
+    # ~100 GB (profile E: 18,432 rows x 16,384 keys, 19 GB of bf16 values)
+    for prof in workloads.MIXED_PROFILES:
+        b = workloads.mixed_profiles(seed=0, backend="torch", device="cuda", profiles=(prof,))[0]
+        rows = fw.rows_from_batch(b)
+        g = fw.dense_and_topk_gap(rows, b.k)
+        sw = fw.swap_refine(rows, b.k, g, E=32, max_swaps=64)
+        torch.cuda.synchronize()
+        assert np.all(np_(g["row_status"]) == 0)
+        gap, dr = np_(g["gap"]), np_(g["dropped"])
+        assert np.all(np.isfinite(gap)) and np.all((dr >= 0) & (dr <= 1 + 1e-6))
+        rg, tg = np_(sw["refined_gap"]), np_(sw["topk_gap"])
+        assert np.all(np.isfinite(rg)) and np.all(rg <= tg * (1 + 1e-6))
+        # one row from the first, a middle and the last group
+        G = rows.num_rows // b.rows_per_group
+        groups = [0, G // 2, G - 1]
+        sel = np.array([gi * b.rows_per_group + int(rng.integers(b.rows_per_group)) for gi in groups])
+        pick = _PickRagged(b, sel)
+        og = oracle.dense_and_topk_gap(pick.H)
+        on = row_onorm(og["o"])
+        assert_close(gap[sel], og["gap"], on, "gap")
+        assert_close(dr[sel], og["dropped"], np.ones_like(on), "dropped")
+        assert_close(np_(g["o"])[sel], og["o"], on, "o")
+        o = oracle.swap_refine(pick.H, E=32, max_swaps=64)
+        _compare_swap(sw, o, sel, on)
+        del rows, g, sw, b
+        torch.cuda.empty_cache()
