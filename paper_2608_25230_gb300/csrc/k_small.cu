@@ -20,7 +20,8 @@ struct SmallGapArgs {
 };
 
 // Definition 2.1 / Sec. 2.1 / Lemma 2.1 for one row and up to four budgets.
-template <int DPL, typename VT>
+// NBM: budgets held in registers (1, or up to 4)
+template <int DPL, typename VT, int NBM>
 __global__ void __launch_bounds__(256) k_small_gap(const SmallGapArgs a)
 {
     const int lane = threadIdx.x & 31;
@@ -54,10 +55,10 @@ __global__ void __launch_bounds__(256) k_small_gap(const SmallGapArgs a)
         rank += (ls > l) || (ls == l && s < lane);
     }
     const int nb = a.nb;
-    uint32_t mask[4];
+    uint32_t mask[NBM];
     int status = FW_OK;
 #pragma unroll
-    for (int b = 0; b < 4; ++b) {
+    for (int b = 0; b < NBM; ++b) {
         mask[b] = 0u;
         if (b >= nb) continue;
         const int kb = a.k[row * nb + b];
@@ -87,9 +88,9 @@ __global__ void __launch_bounds__(256) k_small_gap(const SmallGapArgs a)
             mu[t] = df_add(mu[t], df_mul_f(pj, load_v(V, (int64_t)j * d + lane + 32 * t)));
     }
     // g_A = sum_{j in A} p_j (v_j - mu) for each budget (Lemma 2.1)
-    df gA[4][DPL];
+    df gA[NBM][DPL];
 #pragma unroll
-    for (int b = 0; b < 4; ++b)
+    for (int b = 0; b < NBM; ++b)
 #pragma unroll
         for (int t = 0; t < DPL; ++t) gA[b][t] = df_zero();
     for (int j = 0; j < n; ++j) {
@@ -98,7 +99,7 @@ __global__ void __launch_bounds__(256) k_small_gap(const SmallGapArgs a)
         for (int t = 0; t < DPL; ++t) {
             const df tj = df_mul(pj, df_rsub_f(load_v(V, (int64_t)j * d + lane + 32 * t), mu[t]));
 #pragma unroll
-            for (int b = 0; b < 4; ++b)
+            for (int b = 0; b < NBM; ++b)
                 if ((mask[b] >> j) & 1u) gA[b][t] = df_add(gA[b][t], tj);
         }
     }
@@ -107,7 +108,7 @@ __global__ void __launch_bounds__(256) k_small_gap(const SmallGapArgs a)
         for (int t = 0; t < DPL; ++t) a.out.o[row * d + lane + 32 * t] = mu[t].hi + mu[t].lo;  // rounded once
     }
 #pragma unroll
-    for (int b = 0; b < 4; ++b) {
+    for (int b = 0; b < NBM; ++b) {
         if (mask[b] == 0u) continue;
         const bool in = (mask[b] >> lane) & 1u;
         const double PA = warp_sum_d(in ? p : 0.0);
@@ -425,7 +426,11 @@ fw_status small_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out
     const SmallGapArgs a{R, k, nb, out};
     const int warps = 8;
     const unsigned grid = (unsigned)((R.rows + warps - 1) / warps);
-    FW_DISPATCH(R.d, R.v_dtype, FW_LAUNCH((k_small_gap<DPL, VT>), grid, warps * 32, 0, s, a));
+    if (nb == 1) {
+        FW_DISPATCH(R.d, R.v_dtype, FW_LAUNCH((k_small_gap<DPL, VT, 1>), grid, warps * 32, 0, s, a));
+    } else {
+        FW_DISPATCH(R.d, R.v_dtype, FW_LAUNCH((k_small_gap<DPL, VT, 4>), grid, warps * 32, 0, s, a));
+    }
     return FW_OK;
 }
 
