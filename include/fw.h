@@ -29,9 +29,11 @@
  *     once the stream has reached that point.
  *   - Arguments are validated on the host before any launch; on any error the
  *     call returns a status other than FW_OK and enqueues nothing.
- *   - Conditions only the device can see (non-finite logits) are reported per
- *     row in `row_status`.  The library never traps, asserts or spins on the
- *     device.
+ *   - Conditions only the device can see (non-finite logits, an out-of-range
+ *     budget, a bounded wait that gave up) are reported per row in
+ *     `row_status`.  The library never traps or asserts on the device, and
+ *     every device-side wait (an mbarrier of a bulk copy or of the tensor
+ *     core) gives up after a fixed number of polls instead of spinning.
  *   - Kept sets are stated by threshold: key j of a row is in the top-k set iff
  *     key(l_j) > thr_key or (key(l_j) == thr_key and j <= thr_idx), where key()
  *     maps a float to an unsigned integer of the same order after folding -0
@@ -52,7 +54,7 @@ typedef enum {
     FW_ERR_INVALID_ARG = 1,   /* a size, budget or pointer is out of range     */
     FW_ERR_UNSUPPORTED = 2,   /* valid but not implemented (e.g. d not in 32k) */
     FW_ERR_CUDA = 3,          /* a CUDA launch or query failed                */
-    FW_ERR_TIMEOUT = 4,       /* reserved: no entry point waits on the device */
+    FW_ERR_TIMEOUT = 4,       /* per-row: a bounded device-side wait gave up  */
     FW_ERR_WORKSPACE = 5,     /* workspace missing, too small or misaligned   */
     FW_ERR_NONFINITE = 6      /* per-row: a logit is NaN or infinite          */
 } fw_status;
@@ -94,7 +96,8 @@ typedef struct {
     int32_t *thr_idx;    /* [rows][nb]     largest kept index carrying thr_key     */
     uint32_t *kept_bits; /* [rows][nb][kept_words] bit j%32 of word j/32 = (j in A) */
     int32_t kept_words;  /* words per (row, budget); >= ceil(max_n/32) if kept_bits */
-    int32_t *row_status; /* [rows]         FW_OK or FW_ERR_NONFINITE               */
+    int32_t *row_status; /* [rows]         FW_OK, FW_ERR_NONFINITE, FW_ERR_INVALID_ARG
+                                           (budget out of range) or FW_ERR_TIMEOUT */
 } fw_gap_out;
 
 /* Dense output, top-k kept sets, forced-weight outputs, gaps and dropped mass
@@ -111,6 +114,9 @@ typedef struct {
 fw_status fw_dense_and_topk_gap(const fw_rows *rows, const int32_t *k, int32_t nb,
                                 const fw_gap_out *out, void *workspace, size_t workspace_bytes,
                                 void *stream);
+/* Workspace bytes (0 for max_n <= 32): per-row softmax statistics, thresholds
+ * and status, and a list of the rows whose threshold search falls back to the
+ * radix select (rows with heavy ties). */
 size_t fw_dense_and_topk_gap_workspace(const fw_rows *rows, int32_t nb);
 
 /* Parameters of the balancing selector. */
@@ -137,6 +143,10 @@ fw_status fw_swap_refine(const fw_rows *rows, const int32_t *k, int32_t nb, cons
                          const fw_swap_params *prm, int32_t *n_swaps, int32_t *swap_out,
                          int32_t *swap_in, float *refined_gap, float *topk_gap, int32_t *capped,
                          void *workspace, size_t workspace_bytes, void *stream);
+/* Workspace bytes (0 for max_n <= 32): for up to 3 x 152 persistent blocks,
+ * per-key arrays of max_n entries and a table of kept x pool cross products
+ * (fp32, max_n x round_up(E, 32) entries per block: 1.9 GB for max_n = 32,768
+ * and E = 32). */
 size_t fw_swap_refine_workspace(const fw_rows *rows, int32_t nb, const fw_swap_params *prm);
 
 /* Exact ES(k) (Sec. 2.1) by exhaustive search over all C(n, k) subsets, for
