@@ -71,9 +71,9 @@ struct LSArgs {
     int32_t *kbuf;   // key at each position of the current kept list
     float *pbuf;     // its mass
     float *xbuf;     // its |w|^2
-    // per-block cross-product table, [gridDim.x][Ep][cstride]
+    // per-block cross-product table, [gridDim.x][cstride][Ep] (position-major)
     float *cbuf;
-    int cstride;     // positions per slot row (max_n rounded up to a multiple of 4)
+    int cstride;     // positions per block table (max_n rounded up to a multiple of 4)
 };
 
 __device__ __forceinline__ float block_sum(float v, float *red)
@@ -205,11 +205,12 @@ __device__ __forceinline__ void cross_table(const int *kb, int nk, const VT *V, 
 #pragma unroll
                 for (int u = 0; u < TK; ++u) cur[u] = nxt[u];
             }
-            static_assert(TK == 2, "the tile stores TK consecutive positions as one float2");
-#pragma unroll
-            for (int s = 0; s < TS; ++s)
-                __stcs(reinterpret_cast<float2 *>(cb + (size_t)(q0 + sub * TS + s) * cstride + t0),
-                       make_float2(acc[0][s], acc[1][s]));
+            #pragma unroll
+            for (int u = 0; u < TK; ++u) {
+                float4 *dst = reinterpret_cast<float4 *>(cb + (size_t)(t0 + u) * Ep + q0 + sub * TS);
+                __stcs(dst, make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]));
+                __stcs(dst + 1, make_float4(acc[u][4], acc[u][5], acc[u][6], acc[u][7]));
+            }
         }
     }
 }
@@ -335,8 +336,9 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
     float *wdep = g + d;               // [d]   w of the key that left A last (its pool slot's column)
     float *wtmp = wdep + d;            // [d]   w of the key that entered A last
     float *Wt = wtmp + d;              // [d][Ep] pool vectors w_j, slot-major inner
-    float4 *slot4 = reinterpret_cast<float4 *>(Wt + d * Ep);  // [Ep] per-round slot terms
-    float *pj = reinterpret_cast<float *>(slot4 + Ep);         // [Ep] masses of the pool slots
+    // per-round slot terms of the regrouped score: B_j, k_j, h_j, p_j ([Ep] each)
+    float *sB = Wt + d * Ep, *sK = sB + Ep, *sH = sK + Ep, *sP = sH + Ep;
+    float *pj = sP + Ep;               // [Ep] masses of the pool slots
     float *betaj = pj + Ep;            // [Ep]
     int *idxj = reinterpret_cast<int *>(betaj + Ep);  // [Ep] keys in the slots
     float *red = reinterpret_cast<float *>(idxj + Ep);  // [32]
@@ -354,7 +356,7 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
     float *pk = a.pbuf + boff;
     float *xk = a.xbuf + boff;
     const int cs = a.cstride;
-    float *cb = a.cbuf + (size_t)blockIdx.x * Ep * cs;
+    float *cb = a.cbuf + (size_t)blockIdx.x * Ep * cs;  // [cs][Ep]
     const int nb = a.nb, MS = a.max_swaps;
 
     for (int64_t row = blockIdx.x; row < a.R.rows; row += gridDim.x) {
@@ -611,7 +613,10 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
                         const float beta = p * p * s2 + 2.f * p * sg;
                         betaj[q] = beta;
                         // D_ij = A_i + B_j + p_i (h_j + k_j C_ij) (the file comment's D regrouped)
-                        slot4[q] = make_float4(beta * P2 - N * p * fmaf(2.f, P, p), -2.f * P2 * p, 2.f * N * p, p);
+                        sB[q] = beta * P2 - N * p * fmaf(2.f, P, p);
+                        sK[q] = -2.f * P2 * p;
+                        sH[q] = 2.f * N * p;
+                        sP[q] = p;
                     }
                 }
                 if (wid == SWT / 32 - 1) {  // mu.g and mu.(changed slot's vector) for the folded products
@@ -649,7 +654,7 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
                         if (wid == 0 && q < nadd) {
                             float c3 = 0.f;
                             for (int w = 0; w < SWT / 32; ++w) c3 += part[w * 32 + lane];
-                            __stcs(cb + (size_t)q * cs + tprev, c3);
+                            __stcs(cb + (size_t)tprev * Ep + q, c3);
                         }
                         __syncthreads();
                     }
@@ -678,28 +683,45 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
                     const bool fast = 16.f * (Pm + pmin) * (Pm + pmin) >= P2;
                     float kmin = INFINITY;
                     for (int q0 = 0; q0 < nadd; q0 += 32) {
+                        const int qb = q0 + 8 * sub;  // this lane's 8 consecutive slots
                         float cq[8];
+                        if (q0 == 0) {
 #pragma unroll
-                        for (int m = 0; m < 8; ++m)
-                            cq[m] = q0 == 0 ? cq0[m] : __ldcs(cb + (size_t)(q0 + 4 * m + sub) * cs + t);
-                        if (col && qprev >= q0 && qprev < q0 + 32 && ((qprev - q0) & 3) == sub) {
-                            const int mm = (qprev - q0) >> 2;
+                            for (int m = 0; m < 8; ++m) cq[m] = cq0[m];
+                        } else {
+                            const float4 *src = reinterpret_cast<const float4 *>(cb + (size_t)t * Ep + qb);
+                            const float4 c0 = __ldcs(src), c1 = __ldcs(src + 1);
+                            cq[0] = c0.x, cq[1] = c0.y, cq[2] = c0.z, cq[3] = c0.w;
+                            cq[4] = c1.x, cq[5] = c1.y, cq[6] = c1.z, cq[7] = c1.w;
+                        }
+                        if (col && qprev >= qb && qprev < qb + 8) {
+                            const int mm = qprev - qb;
 #pragma unroll
                             for (int m = 0; m < 8; ++m)
                                 if (m == mm) cq[m] = sn;
-                            __stcs(cb + (size_t)qprev * cs + t, sn);
+                            __stcs(cb + (size_t)t * Ep + qprev, sn);
                         }
-                        const int nq = nadd - q0;  // slot q0 + 4m + sub exists iff 4m + sub < nq
-                        if (fast && nq >= 32) {
+                        const int nq = nadd - qb;  // slot qb + m exists iff m < nq
+                        if (fast && nq >= 8) {
 #pragma unroll
-                            for (int m = 0; m < 8; ++m)
-                                kmin = fminf(kmin, fast_score(slot4[q0 + 4 * m + sub], cq[m], p_i, Ai, Pm));
+                            for (int h = 0; h < 8; h += 4) {
+                                const float4 B4 = *reinterpret_cast<const float4 *>(sB + qb + h);
+                                const float4 K4 = *reinterpret_cast<const float4 *>(sK + qb + h);
+                                const float4 H4 = *reinterpret_cast<const float4 *>(sH + qb + h);
+                                const float4 P4 = *reinterpret_cast<const float4 *>(sP + qb + h);
+                                kmin = fminf(kmin, fast_score(make_float4(B4.x, K4.x, H4.x, P4.x), cq[h], p_i, Ai, Pm));
+                                kmin = fminf(kmin, fast_score(make_float4(B4.y, K4.y, H4.y, P4.y), cq[h + 1], p_i, Ai, Pm));
+                                kmin = fminf(kmin, fast_score(make_float4(B4.z, K4.z, H4.z, P4.z), cq[h + 2], p_i, Ai, Pm));
+                                kmin = fminf(kmin, fast_score(make_float4(B4.w, K4.w, H4.w, P4.w), cq[h + 3], p_i, Ai, Pm));
+                            }
                         } else {
 #pragma unroll
                             for (int m = 0; m < 8; ++m)
-                                if (4 * m + sub < nq)
-                                    kmin = fminf(kmin, any_score<DPL, VT>(slot4[q0 + 4 * m + sub], cq[m], p_i, Ai, Pm, P,
-                                                                          P2, N, vr, mu, g, Wt, Ep, q0 + 4 * m + sub));
+                                if (m < nq) {
+                                    const int q = qb + m;
+                                    kmin = fminf(kmin, any_score<DPL, VT>(make_float4(sB[q], sK[q], sH[q], sP[q]), cq[m],
+                                                                          p_i, Ai, Pm, P, P2, N, vr, mu, g, Wt, Ep, q));
+                                }
                         }
                     }
                     if (kmin < lmin) {  // first position of the lane's least score
@@ -710,9 +732,11 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
                         lA = Ai;
                     }
                 };
-                auto load_cq0 = [&](int t, float (&cq0)[8]) {
-#pragma unroll
-                    for (int m = 0; m < 8; ++m) cq0[m] = __ldcs(cb + (size_t)(4 * m + sub) * cs + t);
+                auto load_cq0 = [&](int t, float (&cq0)[8]) {  // slots 8 sub .. 8 sub + 7
+                    const float4 *src = reinterpret_cast<const float4 *>(cb + (size_t)t * Ep + 8 * sub);
+                    const float4 c0 = __ldcs(src), c1 = __ldcs(src + 1);
+                    cq0[0] = c0.x, cq0[1] = c0.y, cq0[2] = c0.z, cq0[3] = c0.w;
+                    cq0[4] = c1.x, cq0[5] = c1.y, cq0[6] = c1.z, cq0[7] = c1.w;
                 };
                 if (first) {
                     for (int t0 = 0; t0 < nk; t0 += KPI) {
@@ -786,9 +810,11 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
                 if (bmin < 0.f && lt >= 0 && lmin == bmin) {
                     const float Pm = P - lp;
                     const VT *vr = V + (int64_t)li * d;
-                    for (int q = sub; q < nadd; q += QL) {
-                        const float sc = any_score<DPL, VT>(slot4[q], __ldcs(cb + (size_t)q * cs + lt), lp, lA, Pm, P, P2,
-                                                            N, vr, mu, g, Wt, Ep, q);
+                    for (int q = 0; q < nadd; ++q) {
+                        if (((q >> 3) & (QL - 1)) != sub) continue;  // this lane's slots
+                        const float sc = any_score<DPL, VT>(make_float4(sB[q], sK[q], sH[q], sP[q]),
+                                                            __ldcs(cb + (size_t)lt * Ep + q), lp, lA, Pm, P, P2, N,
+                                                            vr, mu, g, Wt, Ep, q);
                         if (sc == bmin) {
                             const unsigned long long key = ((unsigned long long)(uint32_t)li << 32) | (uint32_t)idxj[q];
                             if (key < mykey) {
