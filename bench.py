@@ -169,6 +169,16 @@ class EnumE2E:
         for rows in wl.rows:
             # per row: topk gap, dropped, refined gap, best gap, best rank (8 B), best idx (k * 4 B)
             self.d2h += rows.num_rows * (4 * 4 + 8 + 4 * K_SEL)
+        # pinned host buffers for the results, so every download is asynchronous
+        self.out_host = []
+        for rows in wl.rows:
+            R = rows.num_rows
+            self.out_host.append([torch.empty(R, 1, dtype=torch.float32).pin_memory(),
+                                  torch.empty(R, 1, dtype=torch.float32).pin_memory(),
+                                  torch.empty(R, 1, dtype=torch.float32).pin_memory(),
+                                  torch.empty(R, dtype=torch.float32).pin_memory(),
+                                  torch.empty(R, dtype=torch.int64).pin_memory(),
+                                  torch.empty(R, K_SEL, dtype=torch.int32).pin_memory()])
 
     def step(self):
         wl, fw = self.wl, self.wl.fw
@@ -182,16 +192,15 @@ class EnumE2E:
                 ev = torch.cuda.Event()
                 ev.record(cs)
                 ready.append(ev)
-        res = []
-        for ev, rows, k2, k1 in zip(ready, wl.rows, wl.k2, wl.k1):
+        for ev, rows, k2, k1, hout in zip(ready, wl.rows, wl.k2, wl.k1, self.out_host):
             main.wait_event(ev)
             top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
             sw = fw.swap_refine(rows, k2, top, E=N_KEYS, max_swaps=32)
             bs = fw.best_subset(rows, k1, k_max=K_SEL)
-            res.append([t.to("cpu", non_blocking=True) for t in
-                        (top["gap"], top["dropped"], sw["refined_gap"], bs["best_gap"], bs["best_rank"],
-                         bs["best_idx"][:, :K_SEL])])
-        return res
+            for h, t in zip(hout, (top["gap"], top["dropped"], sw["refined_gap"], bs["best_gap"], bs["best_rank"],
+                                   bs["best_idx"][:, :K_SEL])):
+                h.copy_(t.reshape(h.shape), non_blocking=True)
+        return self.out_host
 
 
 def combine_ranks(ms, units_per_rank, dist=None, device=None):
