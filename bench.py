@@ -161,6 +161,7 @@ class EnumE2E:
         self.h2d = 0
         self.d2h = 0
         self.copy_stream = torch.cuda.Stream()
+        self.upload_ev = []  # (start, end) of each step's uploads on the copy stream
         for rows in wl.rows:
             hl = rows.logits.cpu().pin_memory()
             hv = rows.v.cpu().pin_memory()
@@ -186,12 +187,15 @@ class EnumE2E:
         cs.wait_stream(main)
         ready = []
         with torch.cuda.stream(cs):
+            u0 = torch.cuda.Event(enable_timing=True)
+            u0.record(cs)
             for (hl, hv), rows in zip(self.host, wl.rows):
                 rows.logits.copy_(hl, non_blocking=True)
                 rows.v.copy_(hv, non_blocking=True)
-                ev = torch.cuda.Event()
+                ev = torch.cuda.Event(enable_timing=True)
                 ev.record(cs)
                 ready.append(ev)
+        self.upload_ev.append((u0, ready[-1]))
         for ev, rows, k2, k1, hout in zip(ready, wl.rows, wl.k2, wl.k1, self.out_host):
             main.wait_event(ev)
             top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
@@ -201,6 +205,13 @@ class EnumE2E:
                                    bs["best_idx"][:, :K_SEL])):
                 h.copy_(t.reshape(h.shape), non_blocking=True)
         return self.out_host
+
+    def upload_ms(self, last):
+        """Copy-stream time of the uploads of the last `last` steps (ms each)."""
+        torch.cuda.synchronize()
+        r = [a.elapsed_time(b) for a, b in self.upload_ev[-last:]]
+        self.upload_ev = []
+        return r
 
 
 def combine_ranks(ms, units_per_rank, dist=None, device=None):
@@ -435,8 +446,10 @@ def main():
 
     # end to end through the public API with host buffers
     e2e = EnumE2E(wl)
-    e2e_total, _ = time_steps(e2e.step, max(3, K // 2), W, flush, barrier)
-    e2e_value, e2e_ms = combine_ranks(e2e_total / max(3, K // 2), wl.subsets, dist, device)
+    K2 = max(3, K // 2)
+    e2e_total, e2e_times = time_steps(e2e.step, K2, W, flush, barrier)
+    e2e_value, e2e_ms = combine_ranks(e2e_total / K2, wl.subsets, dist, device)
+    up_ms = e2e.upload_ms(K2)
 
     sections = {}
     if not args.no_sections and rank == 0:
@@ -468,7 +481,13 @@ def main():
                                             "scaled to the average call by input bytes (the rescore and exhaustive "
                                             "kernels of the call are not included)"),
                 e2e=dict(value=e2e_value, unit="subsets/s",
-                         h2d_bytes_per_step=e2e.h2d, d2h_bytes_per_step=e2e.d2h),
+                         h2d_bytes_per_step=e2e.h2d, d2h_bytes_per_step=e2e.d2h,
+                         step_ms=[round(t, 2) for t in e2e_times],
+                         upload_ms=[round(t, 2) for t in up_ms],
+                         upload_gbs=e2e.h2d / (statistics.median(up_ms) * 1e-3) / 1e9 if up_ms else None,
+                         note="uploads overlap compute within a step (group g + 1 uploads while group g "
+                              "computes); upload_ms is the copy stream's time from the first to the last "
+                              "upload of a step"),
                 gpu_launches=int(launches_timed), clocks=clocks, peaks_source=peaks["source"])
     if cpu:
         line["cpu_baseline"] = cpu
