@@ -57,6 +57,8 @@ def lib():
             L.orc_contour_alloc.argtypes = [vp, C.c_int, C.c_int, C.c_int, C.c_int64, C.c_int,
                                             vp, vp, vp, vp, vp, vp]
             L.orc_ragged_compact.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, C.c_int, vp, vp, vp, vp]
+            L.orc_group_vote.argtypes = [C.POINTER(_Rows), C.c_int, vp, C.c_int, vp, vp, vp, vp, C.c_int,
+                                         vp, vp, vp]
             L.orc_num_threads.restype = C.c_int
             _lib = L
     return _lib
@@ -170,6 +172,28 @@ def best_subset(batch):
                topk_gap=np.zeros(rows))
     st = lib().orc_best_subset(C.byref(H.c), _p(kk), _p(out["best_rank"]), _p(out["best_gap"]),
                                _p(out["best_idx"]), kmax, _p(out["second_gap"]), _p(out["topk_gap"]))
+    assert st == 0, st
+    return out
+
+
+def group_vote(batch, s, eval_rows=None, words=None):
+    """f1, the group vote: one kept set per group of rows (the s keys of
+    largest summed mass G), every row scored against it.  s: [groups][nb]
+    budgets.  eval_rows: optional boolean [rows]; rows left out are not scored
+    (their gap / dropped stay 0).  Returns dict of numpy arrays."""
+    H = batch if isinstance(batch, HostRows) else HostRows(batch)
+    s = np.ascontiguousarray(_host(s), np.int32)
+    if s.ndim == 1:
+        s = s[:, None].copy()
+    G, nb = s.shape
+    assert G == len(H.n)
+    words = words or (H.max_n + 31) // 32
+    ev = None if eval_rows is None else np.ascontiguousarray(eval_rows, np.uint8)
+    out = dict(mass=np.zeros((G, H.max_n)), margin=np.zeros((G, nb)),
+               bits=np.zeros((G, nb, words), np.uint32), gap=np.zeros((H.num_rows, nb)),
+               dropped=np.zeros((H.num_rows, nb)), status=np.zeros(H.num_rows, np.int32))
+    st = lib().orc_group_vote(C.byref(H.c), nb, _p(s), H.max_n, _p(ev), _p(out["mass"]), _p(out["margin"]),
+                              _p(out["bits"]), words, _p(out["gap"]), _p(out["dropped"]), _p(out["status"]))
     assert st == 0, st
     return out
 

@@ -16,6 +16,9 @@
  *                   none decreases it
  *   Definition 2.2  candidate set = top-mass set + keys of largest single-key
  *                   error p_j ||v_j - mu||
+ *   Sec. 2.1        group vote: one kept set per KV head, the s keys of
+ *                   largest mass summed over the head's query rows, scored
+ *                   for every row of the group
  *   Sec. 4          ContourKV: one score r, one global threshold tau, a
  *                   recency floor of the last 32 positions per cell, tau set
  *                   so that the cache averages s entries per cell; ragged
@@ -30,6 +33,7 @@
  *     stay in the pool; the most-decreasing pair wins, ties -> smallest
  *     (i, j) lexicographically; a swap is taken only on a strict decrease;
  *   - best subset: exact ties -> smallest colex rank sum_i C(c_i, i);
+ *   - group vote: equal summed mass -> lower index first;
  *   - ContourKV: ties at tau are broken by (score desc, cell asc, pos asc);
  *     floor = last min(32, T) positions; the per-cell dropped mass is that of
  *     the cell's normalised scores, for the allocated set and for the cell's
@@ -708,6 +712,113 @@ int orc_ragged_compact(const void *K, const void *V, int cells, int T, int d, in
             memcpy((char *)K_out + (size_t)q * row, (const char *)K + src, row);
             memcpy((char *)V_out + (size_t)q * row, (const char *)V + src, row);
         }
+    return ORC_OK;
+}
+
+/* ---------------------------------------------------------- group vote */
+
+/* f1: the group vote (Sec. 2.1, shared kept sets).  Deployment keeps one set
+ * per KV head for all the query rows that share it; the vote keeps the s keys
+ * of largest mass summed over the group's rows,
+ *     G_j = sum_{rows i of the group} p_ij,
+ * equal G -> lower index first (the same tie reading as the top-mass set).
+ * Every row of the group is then scored against that one set with the
+ * Definition 2.1 / Sec. 2.1 quantities (es and dropped mass of the row's own
+ * masses).  With one row per group the vote is the row's own top-mass set.
+ * s: [groups][nb], 1 <= s <= n[g].
+ * Outputs (any may be NULL except status):
+ *   mass [groups][max_n]      G (entries past n[g] untouched),
+ *   margin [groups][nb]       (G_(s) - G_(s+1)) / G_(s) of the order, the
+ *                             relative gap between the last kept and the first
+ *                             dropped key (1 when s = n, 0 when G_(s) = 0),
+ *   bits [groups][nb][words]  bit j%32 of word j/32 = (j in the vote set),
+ *   gap, dropped [rows][nb]   es(A) and sum_{j not in A} p_j of each row,
+ *   status [rows]             0, ORC_ERR_ARG (a budget of its group is out of
+ *                             range) or ORC_ERR_NONFINITE (a logit of its group
+ *                             is not finite).
+ * eval: [rows] or NULL; rows with eval[r] == 0 skip the per-row scoring (the
+ * group's G and set still use every row). */
+int orc_group_vote(const orc_rows *R, int nb, const int32_t *s, int max_n, const unsigned char *eval,
+                   double *mass, double *margin, uint32_t *bits, int words, double *gap,
+                   double *dropped, int32_t *status)
+{
+    const int64_t G = R->num_groups, RPG = R->rows_per_group;
+    unsigned char *sets = (unsigned char *)calloc((size_t)(G * nb * (int64_t)max_n) + 1, 1);
+    int32_t *gst = (int32_t *)calloc((size_t)G + 1, sizeof(int32_t));
+    /* the vote set of every group and budget */
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t g = 0; g < G; ++g) {
+        const int n = R->n[g];
+        double *Gm = (double *)calloc((size_t)n + 1, sizeof(double));
+        double *p = (double *)malloc(sizeof(double) * ((size_t)n + 1));
+        for (int64_t i = 0; i < RPG && !gst[g]; ++i) {
+            const float *l = R->logits + R->logit_off[g] + i * (int64_t)n;
+            if (softmax_f64(n, l, p))
+                gst[g] = ORC_ERR_NONFINITE;
+            else
+                for (int j = 0; j < n; ++j)
+                    Gm[j] += p[j];
+        }
+        if (mass)
+            for (int j = 0; j < n; ++j)
+                mass[g * (int64_t)max_n + j] = Gm[j];
+        keyed *o = (keyed *)malloc(sizeof(keyed) * ((size_t)n + 1));
+        for (int j = 0; j < n; ++j) {
+            o[j].key = Gm[j];
+            o[j].idx = j;
+        }
+        qsort(o, (size_t)n, sizeof(keyed), cmp_desc_key_asc_idx);
+        for (int b = 0; b < nb; ++b) {
+            const int sb = s[g * nb + b];
+            const int64_t gb = g * nb + b;
+            if (sb < 1 || sb > n) {
+                if (!gst[g])
+                    gst[g] = ORC_ERR_ARG;
+                continue;
+            }
+            unsigned char *in_A = sets + gb * (int64_t)max_n;
+            for (int t = 0; t < sb; ++t)
+                in_A[o[t].idx] = 1;
+            if (margin) {
+                const double last = o[sb - 1].key;
+                margin[gb] = sb == n ? 1.0 : (last > 0 ? (last - o[sb].key) / last : 0.0);
+            }
+            if (bits) {
+                uint32_t *w = bits + gb * (int64_t)words;
+                for (int t = 0; t < words; ++t)
+                    w[t] = 0u;
+                for (int j = 0; j < n; ++j)
+                    if (in_A[j])
+                        w[j >> 5] |= 1u << (j & 31);
+            }
+        }
+        free(o);
+        free(p);
+        free(Gm);
+    }
+    /* every row against its group's sets */
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < G * RPG; ++r) {
+        const int64_t g = r / RPG;
+        status[r] = gst[g];
+        if (gst[g] || (eval && !eval[r]))
+            continue;
+        instance I;
+        int st = load_row(R, r, &I);
+        if (st) {
+            status[r] = st;
+            instance_free(&I);
+            continue;
+        }
+        for (int b = 0; b < nb; ++b) {
+            set_eval e = eval_set(&I, sets + (g * nb + b) * (int64_t)max_n, NULL);
+            if (gap) gap[r * nb + b] = e.gap;
+            if (dropped) dropped[r * nb + b] = e.dropped;
+        }
+        instance_free(&I);
+    }
+    free(gst);
+    free(sets);
     return ORC_OK;
 }
 
