@@ -14,6 +14,8 @@
  *     Phi = ||g_{A*_s}|| is the one-pass certificate.
  *   - Definition 2.2: the candidate set (top-mass set plus the keys of largest
  *     single-key error p_j ||v_j - mu||).
+ *   - Sec. 2.1: the group vote (one kept set per KV head, by the mass summed
+ *     over the head's query rows).
  *   - Sec. 4: ContourKV (one score, one global threshold, a recency floor of
  *     the last 32 positions per cell) and ragged per-head storage.
  *
@@ -161,6 +163,33 @@ fw_status fw_best_subset(const fw_rows *rows, const int32_t *k, uint64_t *best_r
                          int32_t *row_status, void *workspace, size_t workspace_bytes,
                          void *stream);
 size_t fw_best_subset_workspace(const fw_rows *rows);
+
+/* The group vote (Sec. 2.1).  Deployment keeps one set per KV head and
+ * applies it to every query row that shares the head.  For each group of
+ * rows_per_group rows (one value block) the vote keeps the s keys of largest
+ * summed mass G_j = sum over the group's rows of p_j (equal G: the lower index
+ * is kept first), and every row of the group is scored against that set with
+ * its own masses.  With rows_per_group = 1 the vote is each row's own top-mass
+ * set.  The sets of one group for its nb budgets are nested (prefixes of one
+ * order).
+ *   s    : device [num_groups][nb] int32 budgets, 1 <= s <= n[g] (checked on
+ *          the device: a group with an out-of-range budget gets row_status
+ *          FW_ERR_INVALID_ARG on all its rows, its outputs unspecified).
+ *   nb   : 1..4.
+ *   topk : a fw_gap_out filled by fw_dense_and_topk_gap for the same rows; its
+ *          o, row_max and row_sum must be non-NULL.
+ * Outputs (device): vote_gap [rows][nb] es of the group's set for the row;
+ * vote_dropped [rows][nb] the row's mass outside the set, summed over those
+ * keys (may be NULL); vote_bits [num_groups][nb][kept_words] bit j%32 of word
+ * j/32 = (j in the set) (may be NULL; kept_words >= ceil(max_n/32));
+ * row_status [rows] FW_OK, FW_ERR_INVALID_ARG, or FW_ERR_NONFINITE when a logit
+ * of the row's group is not finite (may be NULL). */
+fw_status fw_group_vote(const fw_rows *rows, const int32_t *s, int32_t nb, const fw_gap_out *topk,
+                        float *vote_gap, float *vote_dropped, uint32_t *vote_bits, int32_t kept_words,
+                        int32_t *row_status, void *workspace, size_t workspace_bytes, void *stream);
+/* Workspace bytes: the summed mass of every group (num_groups x max_n fp32)
+ * and the threshold of every (group, budget). */
+size_t fw_group_vote_workspace(const fw_rows *rows, int32_t nb);
 
 /* ContourKV allocation (Sec. 4).  scores: device [cells][T] fp32, finite and
  * >= 0.  Every cell keeps its recency floor (the last min(floor, T) positions)

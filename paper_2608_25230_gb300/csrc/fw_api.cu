@@ -111,6 +111,30 @@ fw_status fw_swap_refine(const fw_rows *rows, const int32_t *k, int32_t nb, cons
                      topk_gap, capped, workspace, workspace_bytes, s);
 }
 
+size_t fw_group_vote_workspace(const fw_rows *rows, int32_t nb)
+{
+    RowsDev R;
+    if (check_rows(rows, R) != FW_OK || nb < 1 || nb > 4) return 0;
+    return group_vote_workspace(R, nb);
+}
+
+fw_status fw_group_vote(const fw_rows *rows, const int32_t *s, int32_t nb, const fw_gap_out *topk, float *vote_gap,
+                        float *vote_dropped, uint32_t *vote_bits, int32_t kept_words, int32_t *row_status,
+                        void *workspace, size_t workspace_bytes, void *stream)
+{
+    RowsDev R;
+    fw_status st = check_rows(rows, R);
+    if (st != FW_OK) return st;
+    if (nb < 1 || nb > 4 || !s || !topk || !vote_gap) return FW_ERR_INVALID_ARG;
+    if (!topk->o || !topk->row_max || !topk->row_sum) return FW_ERR_INVALID_ARG;
+    if (vote_bits && kept_words < (R.max_n + 31) / 32) return FW_ERR_INVALID_ARG;
+    if (R.rows == 0) return FW_OK;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < group_vote_workspace(R, nb))
+        return FW_ERR_WORKSPACE;
+    return group_vote(R, s, nb, *topk, vote_gap, vote_dropped, vote_bits, kept_words, row_status, workspace,
+                      workspace_bytes, (cudaStream_t)stream);
+}
+
 size_t fw_best_subset_workspace(const fw_rows *rows)
 {
     RowsDev R;

@@ -53,6 +53,12 @@ fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out
                     float *refined_gap, float *topk_gap, int32_t *capped, void *ws,
                     size_t ws_bytes, cudaStream_t s);
 
+// The group vote: one kept set per group of rows by summed mass, every row scored.
+size_t group_vote_workspace(const RowsDev &R, int nb);
+fw_status group_vote(const RowsDev &R, const int32_t *s, int nb, const fw_gap_out &topk, float *gap,
+                     float *dropped, uint32_t *bits, int words, int32_t *row_status, void *ws, size_t ws_bytes,
+                     cudaStream_t st);
+
 // ContourKV allocation and ragged compaction.
 size_t contour_workspace(int cells, int T);
 fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64_t total_budget,

@@ -58,10 +58,15 @@ _lib.fw_contour_alloc.argtypes = [vp, C.c_int32, C.c_int32, C.c_int32, C.c_int64
 _lib.fw_contour_alloc_workspace.argtypes = [C.c_int32, C.c_int32]
 _lib.fw_contour_alloc_workspace.restype = C.c_size_t
 _lib.fw_ragged_compact.argtypes = [vp, vp, C.c_int32, C.c_int32, C.c_int32, vp, vp, C.c_int64, vp, vp, vp]
+_lib.fw_group_vote.argtypes = [C.POINTER(FwRows), vp, C.c_int32, C.POINTER(FwGapOut), vp, vp, vp, C.c_int32, vp,
+                               vp, C.c_size_t, vp]
+_lib.fw_group_vote_workspace.argtypes = [C.POINTER(FwRows), C.c_int32]
+_lib.fw_group_vote_workspace.restype = C.c_size_t
 _lib.fw_status_string.argtypes = [C.c_int]
 _lib.fw_status_string.restype = C.c_char_p
 _lib.fw_launch_count.restype = C.c_uint64
-for _f in ("fw_dense_and_topk_gap", "fw_swap_refine", "fw_best_subset", "fw_contour_alloc", "fw_ragged_compact"):
+for _f in ("fw_dense_and_topk_gap", "fw_swap_refine", "fw_best_subset", "fw_contour_alloc", "fw_ragged_compact",
+           "fw_group_vote"):
     getattr(_lib, _f).restype = C.c_int
 
 
@@ -193,6 +198,28 @@ def swap_refine(rows: Rows, k: torch.Tensor, topk: dict, *, E: int, max_swaps: i
                              _ptr(out["refined_gap"]), _ptr(out["topk_gap"]), _ptr(out["capped"]), _ptr(ws),
                              ws.numel(), _stream(stream))
     _check(st, "fw_swap_refine")
+    out["_ws"] = ws
+    return out
+
+
+def group_vote(rows: Rows, s: torch.Tensor, topk: dict, *, bits=True, stream=None):
+    """fw_group_vote.  s: int32 [groups][nb] budgets on the device; topk: the
+    dict dense_and_topk_gap returned for the same rows.  Returns gap, dropped,
+    row_status ([rows][nb] / [rows]) and bits ([groups][nb][words])."""
+    dev = rows.device
+    R, nb = rows.num_rows, int(s.shape[1])
+    words = (rows.max_n + 31) // 32
+    out = dict(gap=torch.empty(R, nb, dtype=torch.float32, device=dev),
+               dropped=torch.empty(R, nb, dtype=torch.float32, device=dev),
+               row_status=torch.empty(R, dtype=torch.int32, device=dev))
+    if bits:
+        out["bits"] = torch.empty(rows.num_groups, nb, words, dtype=torch.int32, device=dev)
+    nbytes = _lib.fw_group_vote_workspace(C.byref(rows.c), nb)
+    ws = _ws(nbytes, dev)
+    st = _lib.fw_group_vote(C.byref(rows.c), _ptr(s), nb, C.byref(topk["_c"]), _ptr(out["gap"]),
+                            _ptr(out["dropped"]), _ptr(out.get("bits")), words, _ptr(out["row_status"]), _ptr(ws),
+                            ws.numel(), _stream(stream))
+    _check(st, "fw_group_vote")
     out["_ws"] = ws
     return out
 

@@ -27,7 +27,7 @@ def lib():
 def test_header_declares_the_five_calls():
     syms = declared_symbols()
     for name in ("fw_dense_and_topk_gap", "fw_swap_refine", "fw_best_subset", "fw_contour_alloc",
-                 "fw_ragged_compact"):
+                 "fw_ragged_compact", "fw_group_vote"):
         assert name in syms
 
 
@@ -72,4 +72,18 @@ def test_host_validation_rejects_bad_arguments(lib):
     prm = fw.FwSwapParams(97, 4)
     assert fw._lib.fw_swap_refine(C.byref(rows), C.c_void_p(256), 1, C.byref(top), C.byref(prm),
                                   *([C.c_void_p(256)] * 6), C.c_void_p(256), 1 << 40, None) == fw.FW_ERR_UNSUPPORTED
+    # group vote: budgets per call, the gap call's outputs, the bit-mask width and the workspace
+    P = C.c_void_p(256)
+    assert fw._lib.fw_group_vote(C.byref(rows), P, 5, C.byref(top), P, P, P, 2, P, P, 1 << 30,
+                                 None) == fw.FW_ERR_INVALID_ARG
+    nosum = fw.FwGapOut()
+    nosum.o = nosum.row_max = 256
+    assert fw._lib.fw_group_vote(C.byref(rows), P, 1, C.byref(nosum), P, P, P, 2, P, P, 1 << 30,
+                                 None) == fw.FW_ERR_INVALID_ARG
+    assert fw._lib.fw_group_vote(C.byref(rows), P, 1, C.byref(top), P, P, P, 1, P, P, 1 << 30,
+                                 None) == fw.FW_ERR_INVALID_ARG
+    need = fw._lib.fw_group_vote_workspace(C.byref(rows), 2)
+    assert need >= 64 * 4
+    assert fw._lib.fw_group_vote(C.byref(rows), P, 2, C.byref(top), P, P, None, 0, None, P, need - 1,
+                                 None) == fw.FW_ERR_WORKSPACE
     assert fw.launch_count() == before  # nothing was launched
