@@ -305,6 +305,23 @@ def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
     ms_swap = total / ks
     ns = holder["sw"]["n_swaps"].float()
     R, n, d, nb = rows.num_rows, int(b.n_host[0]), b.d, rows_k.shape[1]
+
+    # the group vote: one set per KV head (its rows_per_head query rows) at the
+    # same three budgets, every row scored against it
+    s_vote = rows_k[::rows.rows_per_group].contiguous()
+
+    def vote_step():
+        holder["vote"] = fw.group_vote(rows, s_vote, top)
+
+    total, _ = time_steps(vote_step, K, W, flush, lambda: None)
+    ms_vote = total / K
+    G = rows.num_groups
+    # algorithmic bytes: the logits twice (the set needs every row's logits, each
+    # row's score needs the set), the value blocks once, the summed masses
+    # written and read, outputs (gap, dropped, status, bits)
+    vbytes = (2 * rows.logits.numel() * 4 + rows.v.numel() * 2 + 2 * G * n * 4
+              + R * (nb * 8 + 4) + G * nb * (n // 8))
+    vach = vbytes / (ms_vote * 1e-3) / 1e9
     # algorithmic bytes of the gap call: logits once, the value blocks once,
     # outputs (o, three o_A, gap / dropped / phi, thresholds, kept bits)
     nbytes = (rows.logits.numel() * 4 + rows.v.numel() * 2
@@ -324,7 +341,13 @@ def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
                               tensor_flops_executed=2 * 3 * (nb + 1) * n * d * R,
                               tensor_tflops=2 * 3 * (nb + 1) * n * d * R / (ms_gap * 1e-3) / 1e12,
                               tensor_basis="P.V as a bf16 GEMM: 3 bf16 terms per probability, nb + 1 band rows; "
-                                           "time of the whole gap call (the select kernel included)"))
+                                           "time of the whole gap call (the select kernel included)"),
+                group_vote=dict(path="fw_group_vote: one set per KV head by summed mass, all rows scored",
+                                ms_per_call=ms_vote, rows_per_s=R / (ms_vote * 1e-3),
+                                roofline=dict(bound="hbm", kernel="k_vote_mass + k_vote_select + k_vote_eval",
+                                              achieved=vach, peak=peaks["hbm_gbs"], unit="GB/s",
+                                              frac=vach / peaks["hbm_gbs"], traffic=None,
+                                              algorithmic_bytes=vbytes)))
 
 
 def section_contour(fw, device, K, W, flush, peaks):
