@@ -16,6 +16,8 @@
  *                   none decreases it
  *   Definition 2.2  candidate set = top-mass set + keys of largest single-key
  *                   error p_j ||v_j - mu||
+ *   Definition 2.2  ES_pool: exact minimum of es over the size-s subsets of
+ *                   the candidate set
  *   Sec. 2.1        group vote: one kept set per KV head, the s keys of
  *                   largest mass summed over the head's query rows, scored
  *                   for every row of the group
@@ -713,6 +715,141 @@ int orc_ragged_compact(const void *K, const void *V, int cells, int T, int d, in
             memcpy((char *)V_out + (size_t)q * row, (const char *)V + src, row);
         }
     return ORC_OK;
+}
+
+/* ------------------------------------------------- candidate-set search */
+
+/* The candidate set of Definition 2.2 for budget k: the top-mass set plus the
+ * E dropped keys of largest single-key error p_j ||v_j - mu|| (ties -> lower
+ * index).  pool receives the members in ascending key order; returns their
+ * number. */
+static int candidate_set(const instance *I, int k, int E, unsigned char *in_A, int *pool)
+{
+    const int n = I->n, d = I->d;
+    topk_by_logit(n, I->logit, k, in_A);
+    keyed *err = (keyed *)malloc(sizeof(keyed) * ((size_t)n + 1));
+    int nd = 0;
+    for (int j = 0; j < n; ++j) {
+        if (in_A[j])
+            continue;
+        double s2 = 0.0;
+        for (int c = 0; c < d; ++c) {
+            double t = I->v[(int64_t)j * d + c] - I->mu[c];
+            s2 += t * t;
+        }
+        err[nd].key = I->p[j] * sqrt(s2);
+        err[nd].idx = j;
+        ++nd;
+    }
+    qsort(err, (size_t)nd, sizeof(keyed), cmp_desc_key_asc_idx);
+    unsigned char *in_pool = (unsigned char *)malloc((size_t)n + 1);
+    memcpy(in_pool, in_A, (size_t)n);
+    for (int t = 0; t < E && t < nd; ++t)
+        in_pool[err[t].idx] = 1;
+    int P = 0;
+    for (int j = 0; j < n; ++j)
+        if (in_pool[j])
+            pool[P++] = j;
+    free(in_pool);
+    free(err);
+    return P;
+}
+
+/* f2: ES_pool(k) (Definition 2.2), the exact minimum of es over the size-k
+ * subsets of the candidate set, by exhaustive enumeration in lexicographic
+ * order with es of every subset from its definition (m_A = N_A / p(A) with the
+ * row's own masses and mu).  Exact ties -> the smallest colex rank of the
+ * members' positions in the candidate set (sorted by key index).
+ * k: [rows][nb]; E: [nb] extras of budget slot b.
+ * Outputs: best_gap [rows][nb] = ES_pool; best_idx [rows][nb][k_max]
+ * ascending key indices (-1 past k); topk_gap [rows][nb] = es(A*_k);
+ * second_gap [rows][nb] the second-smallest es over the enumerated subsets
+ * (+inf if there is one subset); n_subsets [rows][nb] = C(|pool|, k); status
+ * [rows].  Returns ORC_ERR_ARG for a budget out of range, k > k_max, or more
+ * than max_subsets subsets in a pool. */
+int orc_pool_best_subset(const orc_rows *R, int nb, const int32_t *k, const int32_t *E, int k_max,
+                         int64_t max_subsets, double *best_gap, int32_t *best_idx, double *topk_gap,
+                         double *second_gap, int64_t *n_subsets, int32_t *status)
+{
+    int64_t rows = R->num_groups * R->rows_per_group;
+    int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : bad)
+    for (int64_t r = 0; r < rows; ++r) {
+        instance I;
+        int st = load_row(R, r, &I);
+        status[r] = st;
+        if (st) {
+            instance_free(&I);
+            continue;
+        }
+        const int n = I.n;
+        unsigned char *in_A = (unsigned char *)malloc((size_t)n + 1);
+        int *pool = (int *)malloc(sizeof(int) * ((size_t)n + 1));
+        int *c = (int *)malloc(sizeof(int) * ((size_t)n + 1));
+        int *mem = (int *)malloc(sizeof(int) * ((size_t)n + 1));
+        double *NA = (double *)malloc(sizeof(double) * (size_t)I.d);
+        for (int b = 0; b < nb; ++b) {
+            const int64_t rb = r * nb + b;
+            const int kb = k[rb];
+            if (kb < 1 || kb > n || kb > k_max || E[b] < 0) {
+                bad |= 1;
+                continue;
+            }
+            const int P = candidate_set(&I, kb, E[b], in_A, pool);
+            const uint64_t cnt = binom(P, kb);
+            if (n_subsets)
+                n_subsets[rb] = (int64_t)cnt;
+            if (cnt > (uint64_t)max_subsets) {
+                bad |= 1;
+                continue;
+            }
+            if (topk_gap)
+                topk_gap[rb] = eval_set(&I, in_A, NULL).gap;
+            double best = INFINITY, second = INFINITY;
+            uint64_t best_rank = 0;
+            int32_t *bi = best_idx + rb * (int64_t)k_max;
+            for (int t = 0; t < kb; ++t)
+                c[t] = t;
+            for (;;) {
+                for (int t = 0; t < kb; ++t)
+                    mem[t] = pool[c[t]];
+                const double es = es_of_members(&I, mem, kb, NA);
+                uint64_t rank = 0;
+                for (int t = 0; t < kb; ++t)
+                    rank += binom(c[t], t + 1);
+                if (es < best || (es == best && rank < best_rank)) {
+                    second = best < second ? best : second;
+                    best = es;
+                    best_rank = rank;
+                    for (int t = 0; t < kb; ++t)
+                        bi[t] = mem[t];
+                } else if (es < second) {
+                    second = es;
+                }
+                /* next combination in lexicographic order */
+                int t = kb - 1;
+                while (t >= 0 && c[t] == P - kb + t)
+                    --t;
+                if (t < 0)
+                    break;
+                ++c[t];
+                for (int u = t + 1; u < kb; ++u)
+                    c[u] = c[u - 1] + 1;
+            }
+            for (int t = kb; t < k_max; ++t)
+                bi[t] = -1;
+            best_gap[rb] = best;
+            if (second_gap)
+                second_gap[rb] = second;
+        }
+        free(NA);
+        free(mem);
+        free(c);
+        free(pool);
+        free(in_A);
+        instance_free(&I);
+    }
+    return bad ? ORC_ERR_ARG : ORC_OK;
 }
 
 /* ---------------------------------------------------------- group vote */
