@@ -8,6 +8,9 @@
 // mass of the row's own masses).  Three launches, each one pass over HBM:
 //   k_vote_mass    G of every group: one thread per key walks the group's rows
 //                  in order (loads coalesced over keys); flags non-finite logits.
+//                  Each mass is the fast exponential times 1/Z of its row (a few
+//                  ulp): an accurate exp and a divide per (row, key) would make
+//                  this pass and the scoring pass instruction-bound.
 //   k_vote_select  per group and budget, the order key T of the s-th largest G
 //                  (three-pass radix select over G staged in shared memory) and
 //                  the index L of the last tied key taken; the set is
@@ -53,7 +56,7 @@ struct VoteArgs {
 
 __global__ void __launch_bounds__(VM_T) k_vote_mass(VoteArgs a)
 {
-    __shared__ float sM[VM_T], sZ[VM_T];
+    __shared__ float sM[VM_T], sZ[VM_T];  // M and 1 / Z of the rows in the chunk
     const int tid = threadIdx.x;
     const int Rg = a.R.R;
     for (int64_t g = blockIdx.y; g < a.R.num_groups; g += gridDim.y) {
@@ -70,7 +73,7 @@ __global__ void __launch_bounds__(VM_T) k_vote_mass(VoteArgs a)
                 if (tid < cnt) {
                     const int64_t r = g * Rg + i0 + tid;
                     sM[tid] = a.M[r];
-                    sZ[tid] = a.Z[r];
+                    sZ[tid] = 1.f / a.Z[r];
                 }
                 __syncthreads();
                 if (j < n) {
@@ -79,7 +82,7 @@ __global__ void __launch_bounds__(VM_T) k_vote_mass(VoteArgs a)
                     for (int i = 0; i < cnt; ++i) {
                         const float l = __ldg(col + (int64_t)i * n);
                         bad |= !isfinite(l);
-                        acc += expf(l - sM[i]) / sZ[i];
+                        acc = fmaf(__expf(l - sM[i]), sZ[i], acc);
                     }
                 }
             }
@@ -270,7 +273,7 @@ __global__ void __launch_bounds__(VE_W * 32) k_vote_eval(VoteArgs a)
         const float *l = a.R.logits + a.R.logit_off[g] + i * n;
         const VT *V = static_cast<const VT *>(a.R.v) + a.R.v_off[g];
         const float *G = a.mass + g * (int64_t)a.R.max_n;
-        const float M = a.M[r], Z = a.Z[r];
+        const float M = a.M[r], Zi = 1.f / a.Z[r];
 
         // the group's budgets in ascending order of s: the sets are nested along it
         int sv[V_NBMAX], ord[V_NBMAX];
@@ -323,7 +326,7 @@ __global__ void __launch_bounds__(VE_W * 32) k_vote_eval(VoteArgs a)
             float p = 0.f;
             int band = nb;  // number of (ascending) budgets whose set leaves key j out
             if (j < n) {
-                p = expf(lc - M) / Z;
+                p = __expf(lc - M) * Zi;
                 const uint32_t u = order_key(gc);
                 band = 0;
 #pragma unroll
