@@ -26,7 +26,7 @@
  *                   so that the cache averages s entries per cell; ragged
  *                   per-head storage that frees the evicted bytes
  *
- * Readings where the paper is silent (all listed in the design doc):
+ * Readings taken where the paper is silent:
  *   - p is the softmax of the fp32 logits computed in fp64 (std exp);
  *   - top-mass ranks by logit, equal logits -> lower index first; -0 == +0;
  *   - dropped mass is summed over the dropped keys, not formed as 1 - p(A);
