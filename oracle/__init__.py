@@ -60,7 +60,7 @@ def lib():
             L.orc_group_vote.argtypes = [C.POINTER(_Rows), C.c_int, vp, C.c_int, vp, vp, vp, vp, C.c_int,
                                          vp, vp, vp]
             L.orc_pool_best_subset.argtypes = [C.POINTER(_Rows), C.c_int, vp, vp, C.c_int, C.c_int64,
-                                               vp, vp, vp, vp, vp, vp]
+                                               vp, vp, vp, vp, vp, vp, vp]
             L.orc_num_threads.restype = C.c_int
             _lib = L
     return _lib
@@ -183,17 +183,19 @@ def pool_best_subset(batch, E, max_subsets=1 << 24):
     candidate set (top-mass set + E extras of largest single-key error) for
     every row and budget slot.  E: extras per budget slot (length nb).
     Returns dict of numpy arrays (best_gap, best_idx, topk_gap, second_gap,
-    n_subsets, status) and the call status."""
+    n_subsets, pool_margin, status) and the call status."""
     H = batch if isinstance(batch, HostRows) else HostRows(batch)
     rows, nb = H.num_rows, H.nb
     E = np.ascontiguousarray(np.broadcast_to(np.asarray(E, np.int32), (nb,)), np.int32)
     kmax = int(H.k.max())
     out = dict(best_gap=np.zeros((rows, nb)), best_idx=np.full((rows, nb, kmax), -1, np.int32),
                topk_gap=np.zeros((rows, nb)), second_gap=np.zeros((rows, nb)),
-               n_subsets=np.zeros((rows, nb), np.int64), status=np.zeros(rows, np.int32))
+               n_subsets=np.zeros((rows, nb), np.int64), pool_margin=np.zeros((rows, nb)),
+               status=np.zeros(rows, np.int32))
     st = lib().orc_pool_best_subset(C.byref(H.c), nb, _p(H.k), _p(E), kmax, int(max_subsets),
                                     _p(out["best_gap"]), _p(out["best_idx"]), _p(out["topk_gap"]),
-                                    _p(out["second_gap"]), _p(out["n_subsets"]), _p(out["status"]))
+                                    _p(out["second_gap"]), _p(out["n_subsets"]), _p(out["pool_margin"]),
+                                    _p(out["status"]))
     out["call_status"] = st
     return out
 

@@ -722,8 +722,9 @@ int orc_ragged_compact(const void *K, const void *V, int cells, int T, int d, in
 /* The candidate set of Definition 2.2 for budget k: the top-mass set plus the
  * E dropped keys of largest single-key error p_j ||v_j - mu|| (ties -> lower
  * index).  pool receives the members in ascending key order; returns their
- * number. */
-static int candidate_set(const instance *I, int k, int E, unsigned char *in_A, int *pool)
+ * number.  *margin = (e_E - e_{E+1}) / e_E at the pool boundary (+inf when
+ * every dropped key joins the pool or E = 0). */
+static int candidate_set(const instance *I, int k, int E, unsigned char *in_A, int *pool, double *margin)
 {
     const int n = I->n, d = I->d;
     topk_by_logit(n, I->logit, k, in_A);
@@ -742,6 +743,8 @@ static int candidate_set(const instance *I, int k, int E, unsigned char *in_A, i
         ++nd;
     }
     qsort(err, (size_t)nd, sizeof(keyed), cmp_desc_key_asc_idx);
+    *margin = (E > 0 && E < nd) ? (err[E - 1].key > 0 ? (err[E - 1].key - err[E].key) / err[E - 1].key : 0.0)
+                                : INFINITY;
     unsigned char *in_pool = (unsigned char *)malloc((size_t)n + 1);
     memcpy(in_pool, in_A, (size_t)n);
     for (int t = 0; t < E && t < nd; ++t)
@@ -764,12 +767,13 @@ static int candidate_set(const instance *I, int k, int E, unsigned char *in_A, i
  * Outputs: best_gap [rows][nb] = ES_pool; best_idx [rows][nb][k_max]
  * ascending key indices (-1 past k); topk_gap [rows][nb] = es(A*_k);
  * second_gap [rows][nb] the second-smallest es over the enumerated subsets
- * (+inf if there is one subset); n_subsets [rows][nb] = C(|pool|, k); status
- * [rows].  Returns ORC_ERR_ARG for a budget out of range, k > k_max, or more
+ * (+inf if there is one subset); n_subsets [rows][nb] = C(|pool|, k);
+ * pool_margin [rows][nb] the relative gap between the E-th and the (E+1)-th
+ * single-key error of the dropped keys (+inf if all join); status [rows].  Returns ORC_ERR_ARG for a budget out of range, k > k_max, or more
  * than max_subsets subsets in a pool. */
 int orc_pool_best_subset(const orc_rows *R, int nb, const int32_t *k, const int32_t *E, int k_max,
                          int64_t max_subsets, double *best_gap, int32_t *best_idx, double *topk_gap,
-                         double *second_gap, int64_t *n_subsets, int32_t *status)
+                         double *second_gap, int64_t *n_subsets, double *pool_margin, int32_t *status)
 {
     int64_t rows = R->num_groups * R->rows_per_group;
     int bad = 0;
@@ -795,7 +799,10 @@ int orc_pool_best_subset(const orc_rows *R, int nb, const int32_t *k, const int3
                 bad |= 1;
                 continue;
             }
-            const int P = candidate_set(&I, kb, E[b], in_A, pool);
+            double pm;
+            const int P = candidate_set(&I, kb, E[b], in_A, pool, &pm);
+            if (pool_margin)
+                pool_margin[rb] = pm;
             const uint64_t cnt = binom(P, kb);
             if (n_subsets)
                 n_subsets[rb] = (int64_t)cnt;

@@ -48,6 +48,7 @@ def test_full_pool_equals_exhaustive_search(seed):
     k = rng.integers(1, n, size=(rows, 1))
     b = many_rows_batch(L, V, k)
     o = oracle.pool_best_subset(b, E=[n])
+    assert np.all(np.isinf(o["pool_margin"]))  # every dropped key joins: no pool boundary
     es = oracle.best_subset(b)
     np.testing.assert_allclose(o["best_gap"][:, 0], es["best_gap"], rtol=1e-12, atol=1e-15)
     for r in range(rows):
@@ -57,7 +58,8 @@ def test_full_pool_equals_exhaustive_search(seed):
 
 def _brute_pool(L, V, s, E):
     """Build the candidate set in numpy and score every size-s subset of it by
-    es = ||g_A|| / p(A) (Lemma 2.1).  Returns (best es, best set, es(top-mass))."""
+    es = ||g_A|| / p(A) (Lemma 2.1).  Returns (best es, best set, es(top-mass),
+    relative margin between the E-th and (E+1)-th single-key errors)."""
     l = L.astype(np.float32).astype(np.float64)
     p = np.exp(l - l.max())
     p /= p.sum()
@@ -76,7 +78,9 @@ def _brute_pool(L, V, s, E):
         return np.linalg.norm(g) / p[A].sum()
 
     best = min((es(A), A) for A in itertools.combinations(pool, s))
-    return best[0], list(best[1]), es(top)
+    e_sorted = np.sort(err)[::-1]
+    margin = (e_sorted[E - 1] - e_sorted[E]) / e_sorted[E - 1] if 0 < E < len(rest) else np.inf
+    return best[0], list(best[1]), es(top), margin
 
 
 @pytest.mark.parametrize("s,E", [(3, 4), (5, 6), (2, 9)])
@@ -88,8 +92,9 @@ def test_brute_force_over_the_pool(s, E):
     b = many_rows_batch(L, V, s)
     o = oracle.pool_best_subset(b, E=[E])
     for r in range(rows):
-        best, A, top = _brute_pool(L[r], V[r], s, E)
+        best, A, top, margin = _brute_pool(L[r], V[r], s, E)
         assert o["best_gap"][r, 0] == pytest.approx(best, rel=1e-10, abs=1e-14)
+        assert o["pool_margin"][r, 0] == pytest.approx(margin, rel=1e-9, abs=1e-15)
         assert o["topk_gap"][r, 0] == pytest.approx(top, rel=1e-10, abs=1e-14)
         if o["second_gap"][r, 0] - best > 1e-9 * best:
             assert list(o["best_idx"][r, 0]) == A
