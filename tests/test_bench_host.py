@@ -49,3 +49,25 @@ def test_unreadable_values_and_short_lines_are_skipped():
 def test_no_samples_and_no_sampler_are_flagged():
     assert summarise([])["reasons"] == ["no samples"]
     assert bench.ClockSampler(0).summary()["reasons"] == ["nvidia-smi unavailable"]
+
+
+def test_reference_arm_prints_one_contract_line():
+    # the reference arm is the fp64 oracle on the host cores (no GPU needed)
+    import json
+    import os
+    import subprocess
+    import sys
+
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--steps", "1", "--warmup", "1"],
+                       cwd=root, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [x for x in r.stdout.splitlines() if x.strip().startswith("{")]
+    assert len(lines) == 1
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["metric"] == "subsets/s" and line["unit"] == "subsets/s"
+    assert line["higher_is_better"] is True and line["value"] > 0 and line["warmup"] >= 3
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
