@@ -70,7 +70,10 @@ typedef enum { FW_F32 = 0, FW_BF16 = 1 } fw_dtype;
  * r = g * rows_per_group + i has its n[g] fp32 logits at
  * logits + logit_off[g] + i * n[g]; the group's values are the n[g] x d
  * row-major block at v + v_off[g] (elements of type v_dtype).  The softmax of
- * a row's logits is its mass vector p. */
+ * a row's logits is its mass vector p.
+ * One batch has one value width d and one value dtype: a cache whose heads
+ * differ in width (say d = 64 and d = 128 layers) is issued as one call per
+ * width, each call a ragged batch over n. */
 typedef struct {
     int64_t num_groups;
     int32_t rows_per_group;
@@ -191,6 +194,33 @@ fw_status fw_group_vote(const fw_rows *rows, const int32_t *s, int32_t nb, const
  * and the threshold of every (group, budget). */
 size_t fw_group_vote_workspace(const fw_rows *rows, int32_t nb);
 
+/* ES_pool (Definition 2.2): the exact minimum of es over the size-s subsets
+ * of the candidate set -- the top-mass set A*_s plus the E[b] dropped keys of
+ * largest single-key error p_j ||v_j - mu|| (equal errors: lower index first)
+ * -- by exhaustive search of the pool, for every row and budget slot b.
+ *   k    : device [rows][nb] budgets, 1 <= s <= min(n, 32, k_max); a slot with
+ *          s + min(E[b], n - s) > 64 pool keys, or more than 2^32 subsets on
+ *          the pool's smaller side, is refused (row_status FW_ERR_UNSUPPORTED,
+ *          its gap NaN); an out-of-range s gives FW_ERR_INVALID_ARG.
+ *   E    : HOST [nb] extras per budget slot, >= 0 (the paper's schedule is
+ *          24/12/6/4 at s = 4/8/16/32).
+ *   topk : a fw_gap_out filled by fw_dense_and_topk_gap for the same rows, k
+ *          and nb; its thr_key, thr_idx, o, row_max and row_sum must be
+ *          non-NULL.  mu is taken as its dense output o.
+ * Outputs (device): best_gap [rows][nb] = ES_pool; best_idx [rows][nb][k_max]
+ * the minimising set's keys ascending (entries past s are -1; exact ties go
+ * to the smallest colex rank of the members' positions in the pool, the pool
+ * in ascending key order); topk_gap [rows][nb] es(A*_s) (may be NULL); n_cand
+ * [rows][nb] the subsets re-scored in fp64 after the fp32 screen (may be
+ * NULL); row_status [rows] (may be NULL).  Rows up to 49,152 keys
+ * (FW_ERR_UNSUPPORTED above). */
+fw_status fw_pool_best_subset(const fw_rows *rows, const int32_t *k, int32_t nb, const int32_t *E,
+                              const fw_gap_out *topk, float *best_gap, int32_t *best_idx, int32_t k_max,
+                              float *topk_gap, int64_t *n_cand, int32_t *row_status, void *workspace,
+                              size_t workspace_bytes, void *stream);
+/* Workspace bytes: the pool of every (row, budget), 64 int32 each, and its size. */
+size_t fw_pool_best_subset_workspace(const fw_rows *rows, int32_t nb);
+
 /* ContourKV allocation (Sec. 4).  scores: device [cells][T] fp32, finite and
  * >= 0.  Every cell keeps its recency floor (the last min(floor, T) positions)
  * plus the non-floor positions among the K = total_budget - cells*min(floor,T)
@@ -246,6 +276,15 @@ fw_status fw_contour_alloc_noalloc(const float *scores, int32_t cells, int32_t T
                                    int64_t total_budget, int32_t uniform_s, int32_t *counts,
                                    int64_t *offsets, int32_t *kept_pos, float *tau,
                                    float *dropped_uniform, float *dropped_alloc, void *stream);
+
+/* Waits for `stream` and reports the device-side outcome of the work queued
+ * on it: FW_ERR_CUDA if the stream holds a failed launch or a device fault,
+ * otherwise the first status other than FW_OK in row_status[0 .. rows) (a
+ * per-row status array that an entry point above filled on that stream),
+ * with its row in *first_row (-1, and FW_OK, when every row is fine;
+ * first_row may be NULL).  row_status is device memory; it is read through
+ * a host buffer on the stack, so the call allocates nothing. */
+fw_status fw_sync_status(const int32_t *row_status, int64_t rows, int64_t *first_row, void *stream);
 
 /* Human-readable name of a status. */
 const char *fw_status_string(fw_status s);

@@ -8,6 +8,25 @@ std::atomic<uint64_t> g_launches{0};
 
 static bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
+fw_status device_sms(int *sms)
+{
+    static std::atomic<int> cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return FW_ERR_CUDA;
+    if (dev >= 0 && dev < 64) {
+        const int c = cache[dev].load(std::memory_order_relaxed);
+        if (c > 0) {
+            *sms = c;
+            return FW_OK;
+        }
+    }
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) return FW_ERR_CUDA;
+    if (dev >= 0 && dev < 64) cache[dev].store(n, std::memory_order_relaxed);
+    *sms = n;
+    return FW_OK;
+}
+
 static fw_status check_rows(const fw_rows *r, RowsDev &R)
 {
     if (!r) return FW_ERR_INVALID_ARG;
@@ -155,6 +174,54 @@ fw_status fw_best_subset(const fw_rows *rows, const int32_t *k, uint64_t *best_r
     if (!workspace || !aligned(workspace, 256) || workspace_bytes < enum_workspace(R)) return FW_ERR_WORKSPACE;
     return best_subset(R, k, best_rank, best_gap, best_idx, k_max, topk_gap, row_status, workspace,
                        workspace_bytes, (cudaStream_t)stream);
+}
+
+size_t fw_pool_best_subset_workspace(const fw_rows *rows, int32_t nb)
+{
+    RowsDev R;
+    if (check_rows(rows, R) != FW_OK || nb < 1 || nb > 4) return 0;
+    return pool_best_subset_workspace(R, nb);
+}
+
+fw_status fw_pool_best_subset(const fw_rows *rows, const int32_t *k, int32_t nb, const int32_t *E,
+                              const fw_gap_out *topk, float *best_gap, int32_t *best_idx, int32_t k_max,
+                              float *topk_gap, int64_t *n_cand, int32_t *row_status, void *workspace,
+                              size_t workspace_bytes, void *stream)
+{
+    RowsDev R;
+    fw_status st = check_rows(rows, R);
+    if (st != FW_OK) return st;
+    if (nb < 1 || nb > 4 || !k || !E || !topk || !best_gap || !best_idx || k_max < 1 || k_max > 32)
+        return FW_ERR_INVALID_ARG;
+    for (int b = 0; b < nb; ++b)
+        if (E[b] < 0) return FW_ERR_INVALID_ARG;
+    if (!topk->thr_key || !topk->thr_idx || !topk->o || !topk->row_max || !topk->row_sum) return FW_ERR_INVALID_ARG;
+    if (R.rows == 0) return FW_OK;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < pool_best_subset_workspace(R, nb))
+        return FW_ERR_WORKSPACE;
+    return pool_best_subset(R, k, nb, E, *topk, best_gap, best_idx, k_max, topk_gap, n_cand, row_status, workspace,
+                            (cudaStream_t)stream);
+}
+
+fw_status fw_sync_status(const int32_t *row_status, int64_t rows, int64_t *first_row, void *stream)
+{
+    if (first_row) *first_row = -1;
+    if (rows < 0 || (rows > 0 && !row_status)) return FW_ERR_INVALID_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FW_ERR_CUDA;
+    int32_t buf[4096];
+    for (int64_t r0 = 0; r0 < rows; r0 += 4096) {
+        const int64_t cnt = rows - r0 < 4096 ? rows - r0 : 4096;
+        if (cudaMemcpyAsync(buf, row_status + r0, (size_t)cnt * 4, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+            cudaStreamSynchronize(s) != cudaSuccess)
+            return FW_ERR_CUDA;
+        for (int64_t i = 0; i < cnt; ++i)
+            if (buf[i] != FW_OK) {
+                if (first_row) *first_row = r0 + i;
+                return (fw_status)buf[i];
+            }
+    }
+    return FW_OK;
 }
 
 size_t fw_contour_alloc_workspace(int32_t cells, int32_t T)

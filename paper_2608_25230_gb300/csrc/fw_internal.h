@@ -69,6 +69,15 @@ fw_status ragged_compact(const void *K, const void *V, int cells, int T, int row
                          const int64_t *offsets, const int32_t *kept_pos, int64_t total,
                          void *K_out, void *V_out, cudaStream_t s);
 
+// ES_pool (Definition 2.2): exact best subset of the candidate set, any row length.
+size_t pool_best_subset_workspace(const RowsDev &R, int nb);
+fw_status pool_best_subset(const RowsDev &R, const int32_t *k, int nb, const int32_t *E, const fw_gap_out &topk,
+                           float *best_gap, int32_t *best_idx, int k_max, float *topk_gap, int64_t *n_cand,
+                           int32_t *row_status, void *ws, cudaStream_t st);
+
+// Number of SMs of the current device (queried once per device).
+fw_status device_sms(int *sms);
+
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 }  // namespace fw

@@ -62,11 +62,16 @@ _lib.fw_group_vote.argtypes = [C.POINTER(FwRows), vp, C.c_int32, C.POINTER(FwGap
                                vp, C.c_size_t, vp]
 _lib.fw_group_vote_workspace.argtypes = [C.POINTER(FwRows), C.c_int32]
 _lib.fw_group_vote_workspace.restype = C.c_size_t
+_lib.fw_pool_best_subset.argtypes = [C.POINTER(FwRows), vp, C.c_int32, vp, C.POINTER(FwGapOut), vp, vp, C.c_int32,
+                                     vp, vp, vp, vp, C.c_size_t, vp]
+_lib.fw_pool_best_subset_workspace.argtypes = [C.POINTER(FwRows), C.c_int32]
+_lib.fw_pool_best_subset_workspace.restype = C.c_size_t
+_lib.fw_sync_status.argtypes = [vp, C.c_int64, C.POINTER(C.c_int64), vp]
 _lib.fw_status_string.argtypes = [C.c_int]
 _lib.fw_status_string.restype = C.c_char_p
 _lib.fw_launch_count.restype = C.c_uint64
 for _f in ("fw_dense_and_topk_gap", "fw_swap_refine", "fw_best_subset", "fw_contour_alloc", "fw_ragged_compact",
-           "fw_group_vote"):
+           "fw_group_vote", "fw_pool_best_subset", "fw_sync_status"):
     getattr(_lib, _f).restype = C.c_int
 
 
@@ -246,6 +251,38 @@ def best_subset(rows: Rows, k: torch.Tensor, *, k_max=None, stream=None, ws=None
     _check(st, "fw_best_subset")
     out["_ws"] = ws
     return out
+
+
+def pool_best_subset(rows: Rows, k: torch.Tensor, topk: dict, *, E, k_max: int = 32, stream=None):
+    """fw_pool_best_subset (ES_pool, Definition 2.2).  k: int32 [rows][nb] on
+    the device (the budgets of the gap call `topk`); E: extras per budget slot
+    (host sequence of nb ints).  Returns best_gap, best_idx, topk_gap, n_cand,
+    row_status."""
+    dev, R, nb = rows.device, rows.num_rows, int(k.shape[1])
+    E = [int(e) for e in E]
+    if len(E) != nb:
+        raise ValueError("E needs one entry per budget slot")
+    Eh = (C.c_int32 * nb)(*E)
+    out = dict(best_gap=torch.empty(R, nb, dtype=torch.float32, device=dev),
+               best_idx=torch.empty(R, nb, int(k_max), dtype=torch.int32, device=dev),
+               topk_gap=torch.empty(R, nb, dtype=torch.float32, device=dev),
+               n_cand=torch.empty(R, nb, dtype=torch.int64, device=dev),
+               row_status=torch.empty(R, dtype=torch.int32, device=dev))
+    ws = _ws(_lib.fw_pool_best_subset_workspace(C.byref(rows.c), nb), dev)
+    st = _lib.fw_pool_best_subset(C.byref(rows.c), _ptr(k), nb, Eh, C.byref(topk["_c"]), _ptr(out["best_gap"]),
+                                  _ptr(out["best_idx"]), int(k_max), _ptr(out["topk_gap"]), _ptr(out["n_cand"]),
+                                  _ptr(out["row_status"]), _ptr(ws), ws.numel(), _stream(stream))
+    _check(st, "fw_pool_best_subset")
+    out["_ws"] = ws
+    return out
+
+
+def sync_status(row_status: torch.Tensor, stream=None):
+    """fw_sync_status: wait for the stream, then (status, first bad row) of a
+    per-row status array (FW_OK, -1 when every row is fine)."""
+    first = C.c_int64(-1)
+    st = _lib.fw_sync_status(_ptr(row_status), int(row_status.numel()), C.byref(first), _stream(stream))
+    return int(st), int(first.value)
 
 
 def contour_alloc(scores: torch.Tensor, *, floor: int, total_budget: int, uniform_s: int, stream=None):

@@ -27,7 +27,7 @@ def lib():
 def test_header_declares_the_five_calls():
     syms = declared_symbols()
     for name in ("fw_dense_and_topk_gap", "fw_swap_refine", "fw_best_subset", "fw_contour_alloc",
-                 "fw_ragged_compact", "fw_group_vote"):
+                 "fw_ragged_compact", "fw_group_vote", "fw_pool_best_subset", "fw_sync_status"):
         assert name in syms
 
 
@@ -86,4 +86,22 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert need >= 64 * 4
     assert fw._lib.fw_group_vote(C.byref(rows), P, 2, C.byref(top), P, P, None, 0, None, P, need - 1,
                                  None) == fw.FW_ERR_WORKSPACE
+    # ES_pool: budget slots, extras, the gap call's thresholds, k_max and the workspace
+    E2 = (C.c_int32 * 2)(4, 4)
+    assert fw._lib.fw_pool_best_subset(C.byref(rows), P, 5, E2, C.byref(top), P, P, 32, None, None, None, P, 1 << 30,
+                                       None) == fw.FW_ERR_INVALID_ARG
+    Eneg = (C.c_int32 * 2)(4, -1)
+    assert fw._lib.fw_pool_best_subset(C.byref(rows), P, 2, Eneg, C.byref(top), P, P, 32, None, None, None, P, 1 << 30,
+                                       None) == fw.FW_ERR_INVALID_ARG
+    assert fw._lib.fw_pool_best_subset(C.byref(rows), P, 2, E2, C.byref(nosum), P, P, 32, None, None, None, P, 1 << 30,
+                                       None) == fw.FW_ERR_INVALID_ARG
+    assert fw._lib.fw_pool_best_subset(C.byref(rows), P, 2, E2, C.byref(top), P, P, 33, None, None, None, P, 1 << 30,
+                                       None) == fw.FW_ERR_INVALID_ARG
+    need = fw._lib.fw_pool_best_subset_workspace(C.byref(rows), 2)
+    assert need >= 2 * 64 * 4
+    assert fw._lib.fw_pool_best_subset(C.byref(rows), P, 2, E2, C.byref(top), P, P, 32, None, None, None, P, need - 1,
+                                       None) == fw.FW_ERR_WORKSPACE
+    # the status read-back rejects a negative row count before it touches the device
+    first = C.c_int64(7)
+    assert fw._lib.fw_sync_status(P, -1, C.byref(first), None) == fw.FW_ERR_INVALID_ARG and first.value == -1
     assert fw.launch_count() == before  # nothing was launched
