@@ -167,6 +167,23 @@ fw_status fw_best_subset(const fw_rows *rows, const int32_t *k, uint64_t *best_r
                          void *stream);
 size_t fw_best_subset_workspace(const fw_rows *rows);
 
+/* What the last fw_best_subset call made with `workspace` spent: the search
+ * covers all C(n, k) subsets, but evaluates only those no bound excludes.
+ * The paper has no counterpart; these are the search's own work counters. */
+typedef struct {
+    int64_t rows_exhaustive;  /* rows whose candidates overflowed and that went to the
+                                 exhaustive fp64 path (every subset screened in fp32) */
+    int64_t candidates;       /* subsets re-scored in double-float after the walk     */
+    uint64_t inner_nodes;     /* inner-set enumerations the walk ran                  */
+    uint64_t inner_leaves;    /* subsets those enumerations visited                   */
+    uint64_t inner_ops;       /* fp32 add/min operations of those enumerations        */
+    uint64_t skipped;         /* walk nodes and removal classes excluded by a bound   */
+} fw_best_subset_stats;
+/* Waits for `stream` (on which that call ran) and fills *stats.  rows must
+ * describe the same batch.  Returns FW_ERR_UNSUPPORTED for max_n > 32. */
+fw_status fw_best_subset_read_stats(const fw_rows *rows, const void *workspace, fw_best_subset_stats *stats,
+                                    void *stream);
+
 /* The group vote (Sec. 2.1).  Deployment keeps one set per KV head and
  * applies it to every query row that shares the head.  For each group of
  * rows_per_group rows (one value block) the vote keeps the s keys of largest
@@ -259,15 +276,18 @@ fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t
  * cudaMalloc would synchronise the device -- and cannot provide the
  * workspace fw_contour_alloc asks for.  This variant takes the same
  * arguments minus the workspace and uses a scratch area compiled into the
- * library instead (about 83 KB, held by every GPU that loads the library
- * until the process exits).
+ * library instead: 87,552 bytes (20 bytes per cell of the maximum plus
+ * 5,632 bytes of histograms and alignment), held by every GPU that loads
+ * the library until the process exits.
  *   - cells must be <= FW_CONTOUR_NOALLOC_MAX_CELLS, otherwise the call
  *     returns FW_ERR_WORKSPACE and launches nothing; the other argument
  *     rules and all outputs are exactly those of fw_contour_alloc.
  *   - It never allocates or frees device memory.
- *   - The first call on each device looks up the scratch area's device
- *     address (with that device current); make that first call before any
- *     stream capture on the device.
+ *   - Every call looks up the scratch area's address in the current
+ *     device's context (a host-side query), so the address stays right after
+ *     a device reset.  The first call on a device may load the library's
+ *     module there; make that first call before any stream capture on the
+ *     device.
  *   - All calls share the one scratch area and every call re-initialises
  *     what it reads, so consecutive calls are independent; calls that
  *     overlap on the GPU (concurrent streams, several host threads) race on

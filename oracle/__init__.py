@@ -61,6 +61,8 @@ def lib():
                                          vp, vp, vp]
             L.orc_pool_best_subset.argtypes = [C.POINTER(_Rows), C.c_int, vp, vp, C.c_int, C.c_int64,
                                                vp, vp, vp, vp, vp, vp, vp]
+            L.orc_candidate_set.argtypes = [C.POINTER(_Rows), C.c_int64, C.c_int, C.c_int, vp, vp]
+            L.orc_swap_scores.argtypes = [C.POINTER(_Rows), C.c_int64, vp, vp, C.c_int, vp, vp]
             L.orc_num_threads.restype = C.c_int
             _lib = L
     return _lib
@@ -198,6 +200,33 @@ def pool_best_subset(batch, E, max_subsets=1 << 24):
                                     _p(out["status"]))
     out["call_status"] = st
     return out
+
+
+def candidate_set(batch, row, k, E):
+    """Definition 2.2's candidate set of one row at budget k: (pool key indices
+    ascending, pool-boundary margin)."""
+    H = batch if isinstance(batch, HostRows) else HostRows(batch)
+    g = int(row) // H.R
+    pool = np.zeros(int(H.n[g]) + 1, np.int32)
+    margin = np.zeros(1)
+    P = lib().orc_candidate_set(C.byref(H.c), int(row), int(k), int(E), _p(pool), _p(margin))
+    assert P >= 0, P
+    return pool[:P].copy(), float(margin[0])
+
+
+def swap_scores(batch, row, in_A, add):
+    """One balancing round scored in full: es(A - i + j) for every kept key i
+    (ascending; rows of the result) and every j in `add` (columns), and es(A).
+    in_A: boolean mask over the row's keys."""
+    H = batch if isinstance(batch, HostRows) else HostRows(batch)
+    m = np.ascontiguousarray(in_A, np.uint8)
+    add = np.ascontiguousarray(add, np.int32)
+    na = int(m.sum())
+    out = np.zeros((na, len(add)))
+    cur = np.zeros(1)
+    got = lib().orc_swap_scores(C.byref(H.c), int(row), _p(m), _p(add), len(add), _p(out), _p(cur))
+    assert got == na, got
+    return out, float(cur[0])
 
 
 def group_vote(batch, s, eval_rows=None, words=None):

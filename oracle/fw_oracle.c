@@ -859,6 +859,88 @@ int orc_pool_best_subset(const orc_rows *R, int nb, const int32_t *k, const int3
     return bad ? ORC_ERR_ARG : ORC_OK;
 }
 
+/* The candidate set of Definition 2.2 for row r at budget k (the helper
+ * above, exposed for the tests): pool (capacity n of the row) receives the
+ * members in ascending key order, the return value is their number (negative
+ * on a bad row or budget), *margin the pool-boundary margin. */
+int orc_candidate_set(const orc_rows *R, int64_t r, int k, int E, int32_t *pool, double *margin)
+{
+    instance I;
+    if (load_row(R, r, &I)) {
+        instance_free(&I);
+        return -1;
+    }
+    if (k < 1 || k > I.n || E < 0) {
+        instance_free(&I);
+        return -1;
+    }
+    unsigned char *in_A = (unsigned char *)malloc((size_t)I.n + 1);
+    int *pl = (int *)malloc(sizeof(int) * ((size_t)I.n + 1));
+    const int P = candidate_set(&I, k, E, in_A, pl, margin);
+    for (int t = 0; t < P; ++t)
+        pool[t] = pl[t];
+    free(pl);
+    free(in_A);
+    instance_free(&I);
+    return P;
+}
+
+/* One round of the balancing selector (Sec. 2.1), every option scored: for
+ * row r and the kept set in_A (n bytes of the row), es(A - i + j) for every
+ * kept key i (ascending) and every j in add[0..nadd), from the definition
+ * m_A' = N_A' / p(A') with N_A' = N_A - p_i v_i + p_j v_j.  Writes
+ * es_out[a * nadd + q] for the a-th kept key and add[q], and *cur = es(A).
+ * Keys of add that are already in A are scored as given (the tests pass keys
+ * outside A).  Returns the number of kept keys, or -1 on a bad row. */
+int orc_swap_scores(const orc_rows *R, int64_t r, const unsigned char *in_A, const int32_t *add, int nadd,
+                    double *es_out, double *cur)
+{
+    instance I;
+    if (load_row(R, r, &I)) {
+        instance_free(&I);
+        return -1;
+    }
+    const int n = I.n, d = I.d;
+    double *NA = (double *)calloc((size_t)d, sizeof(double));
+    int *kept = (int *)malloc(sizeof(int) * ((size_t)n + 1));
+    double PA = 0.0;
+    int na = 0;
+    for (int j = 0; j < n; ++j)
+        if (in_A[j]) {
+            kept[na++] = j;
+            PA += I.p[j];
+            for (int c = 0; c < d; ++c)
+                NA[c] += I.p[j] * I.v[(int64_t)j * d + c];
+        }
+    if (cur) {
+        double g2 = 0.0;
+        for (int c = 0; c < d; ++c) {
+            const double diff = NA[c] / PA - I.mu[c];
+            g2 += diff * diff;
+        }
+        *cur = sqrt(g2);
+    }
+#pragma omp parallel for schedule(static)
+    for (int a = 0; a < na; ++a) {
+        const int i = kept[a];
+        for (int q = 0; q < nadd; ++q) {
+            const int j = add[q];
+            const double P2 = PA - I.p[i] + I.p[j];
+            double g2 = 0.0;
+            for (int c = 0; c < d; ++c) {
+                const double Nc = NA[c] - I.p[i] * I.v[(int64_t)i * d + c] + I.p[j] * I.v[(int64_t)j * d + c];
+                const double diff = Nc / P2 - I.mu[c];
+                g2 += diff * diff;
+            }
+            es_out[(int64_t)a * nadd + q] = sqrt(g2);
+        }
+    }
+    free(kept);
+    free(NA);
+    instance_free(&I);
+    return na;
+}
+
 /* ---------------------------------------------------------- group vote */
 
 /* f1: the group vote (Sec. 2.1, shared kept sets).  Deployment keeps one set

@@ -224,6 +224,17 @@ fw_status fw_sync_status(const int32_t *row_status, int64_t rows, int64_t *first
     return FW_OK;
 }
 
+fw_status fw_best_subset_read_stats(const fw_rows *rows, const void *workspace, fw_best_subset_stats *stats,
+                                    void *stream)
+{
+    RowsDev R;
+    fw_status st = check_rows(rows, R);
+    if (st != FW_OK) return st;
+    if (!stats || !workspace || !aligned(workspace, 256)) return FW_ERR_INVALID_ARG;
+    if (R.max_n > 32) return FW_ERR_UNSUPPORTED;
+    return best_subset_stats(R, workspace, stats, (cudaStream_t)stream);
+}
+
 size_t fw_contour_alloc_workspace(int32_t cells, int32_t T)
 {
     if (cells < 1 || T < 1) return 0;

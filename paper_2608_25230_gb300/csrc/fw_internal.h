@@ -31,6 +31,7 @@ size_t enum_workspace(const RowsDev &R);
 fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, float *best_gap,
                       int32_t *best_idx, int k_max, float *topk_gap, int32_t *row_status,
                       void *ws, size_t ws_bytes, cudaStream_t s);
+fw_status best_subset_stats(const RowsDev &R, const void *ws, fw_best_subset_stats *out, cudaStream_t s);
 
 // Long rows (any n): row statistics + radix top-k, then the P.V products.
 // Per-row results of the select kernel that the P.V kernels read.

@@ -15,7 +15,6 @@
 // prefix sum into ragged offsets, and per-cell ordered compaction of the kept
 // positions.  The compaction copy moves 16-byte vectors, a row per 16 lanes.
 #include <algorithm>
-#include <mutex>
 
 #include "fw_internal.h"
 
@@ -480,22 +479,15 @@ namespace {
 constexpr size_t kNoallocBytes = 4 * 256 * 4 + 256 + 5 * (size_t)FW_CONTOUR_NOALLOC_MAX_CELLS * 4;  // >= contour_workspace
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocBytes + 5 * 256];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_noalloc_mu;
-void *g_noalloc_ptr[kMaxDevices] = {};
-
-// Device address of the scratch array for the current device (looked up once per device).
+// Device address of the scratch array in the current device's context.  It is
+// looked up on every call (a host-side query, no launch): after a device reset
+// or a re-created primary context the module is loaded anew and the array may
+// sit elsewhere, so no address is kept between calls.
 fw_status noalloc_scratch(void **ptr)
 {
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FW_ERR_CUDA;
-    std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return FW_ERR_CUDA;
-        g_noalloc_ptr[dev] = p;
-    }
-    *ptr = g_noalloc_ptr[dev];
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return FW_ERR_CUDA;
+    *ptr = p;
     return FW_OK;
 }
 

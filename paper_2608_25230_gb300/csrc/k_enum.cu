@@ -1,8 +1,12 @@
 // k_enum.cu -- exact ES(k) (Sec. 2.1) by exhaustive search, rows with n <= 32.
 //
-// Every size-k subset A of the row's keys is examined; the one of smallest
-// es(A) is reported (exact ties: smallest colex rank).  Instead of O(k d)
-// work per subset, the walk below spends ~4 fp32 instructions per subset:
+// Every size-k subset A of the row's keys is covered -- either evaluated, or
+// excluded together with a whole group of subsets by a rigorous bound -- and
+// the one of smallest es(A) is reported (exact ties: smallest colex rank).
+// Instead of O(k d) work per subset, the walk below spends a few fp32
+// instructions per subset it visits, and on the measured rows the bounds
+// exclude most subsets without visiting them; the walk counts the nodes,
+// subsets (leaves) and fp32 operations it spends (fw_best_subset_read_stats).
 //
 // (1) With u_j = p_j (v_j - mu), Lemma 2.1 gives es(A)^2 = Q(A) / P(A)^2,
 //     Q(A) = ||sum_{j in A} u_j||^2, P(A) = sum_{j in A} p_j.  With
@@ -60,6 +64,8 @@ struct EnumArgs {
     uint8_t *perms;       // [rows][PERM] local key order
     float2 *kg;           // [rows] kappa, |g0| (rounded up)
     int stride;           // floats per row slot (odd)
+    unsigned long long *stats;  // [4] walk counters: inner enumerations, their leaves,
+                                // their fp32 operations, nodes / classes skipped by a bound
 };
 
 // Per-row slot (floats).  Local key order: L (EM inner keys, padded), A0 (k),
@@ -126,7 +132,35 @@ struct Walk {
     float kappa, g0n;
     uint32_t *cand;
     int32_t *ccount;
+    unsigned long long *stats;
 };
+
+// Leaves (C(EM, c)) and fp32 add/min operations of one inner<c> enumeration
+// (the dfs below: one add per visited key, the running sums of the remaining
+// keys at every internal node, one min per leaf, three to merge the minima).
+__host__ __device__ constexpr unsigned long long dfs_ops(int C, int E)
+{
+    return (C >= 1 && E <= EM - C)
+               ? 1ull + (C == 1 ? 1ull : (unsigned long long)(EM - E - 1) + dfs_ops(C - 1, E + 1)) + dfs_ops(C, E + 1)
+               : 0ull;
+}
+__host__ __device__ constexpr unsigned long long dfs_leaves(int C, int E)
+{
+    return (C >= 1 && E <= EM - C) ? (C == 1 ? 1ull : dfs_leaves(C - 1, E + 1)) + dfs_leaves(C, E + 1) : 0ull;
+}
+struct InnerCost {
+    unsigned long long leaves[EM + 1], ops[EM + 1];
+};
+constexpr InnerCost make_inner_cost()
+{
+    InnerCost t{};
+    for (int c = 0; c <= EM; ++c) {
+        t.leaves[c] = c == 0 ? 1ull : dfs_leaves(c, 0);
+        t.ops[c] = c == 0 ? 0ull : dfs_ops(c, 0) + 3ull;
+    }
+    return t;
+}
+static __constant__ InnerCost c_inner_cost = make_inner_cost();
 
 // ---- slow path: list every inner set C (size c) of a node whose folded value is <= 0
 __device__ __noinline__ void collect(const Walk W, uint32_t keep0, uint32_t hmask, const float *w, float q, int c)
@@ -235,6 +269,7 @@ __device__ __noinline__ void walk_row(const Walk W)
     float qst[MAXD];
     int path[MAXD];
     const uint32_t nR = 1u << k;
+    unsigned long long n_inner = 0, n_leaf = 0, n_ops = 0, n_skip = 0;
     // Removal sets R of A0 by size class; the row's two lanes take alternate
     // members of the same class at the same time, so they run the same code.
     for (int r = 0; r <= k; ++r) {
@@ -323,6 +358,7 @@ __device__ __noinline__ void walk_row(const Walk W)
             skip_r = lb > root_slack(r) * (fabsf(q) + aw + pabs);
         }
         if (skip_r) {
+            ++n_skip;
             R = next_same_size(R);
             if (R < nR) R = next_same_size(R);
             valid = R < nR;
@@ -359,8 +395,13 @@ __device__ __noinline__ void walk_row(const Walk W)
                     skip = lb > kInnerSlack * (fabsf(q) + aw + g2abs);
                 }
                 if (!skip) {
+                    ++n_inner;
+                    n_leaf += c_inner_cost.leaves[c];
+                    n_ops += c_inner_cost.ops[c];
                     const float mval = inner_dispatch(c, w, q, G2);
                     if (mval <= 0.f) collect(W, keep0, imask, w, q, c);
+                } else {
+                    ++n_skip;
                 }
             }
             if (!(depth < r && e < nHp && depth < MAXD)) {
@@ -405,6 +446,10 @@ __device__ __noinline__ void walk_row(const Walk W)
         // hence runs this loop the same number of times.
         if (W.sync_mask) __syncwarp(W.sync_mask);
     }
+    atomicAdd(W.stats + 0, n_inner);
+    atomicAdd(W.stats + 1, n_leaf);
+    atomicAdd(W.stats + 2, n_ops);
+    atomicAdd(W.stats + 3, n_skip);
 }
 
 // Write one Gram entry (or a_x / l_x) into the walk tables of a row slot.
@@ -827,6 +872,7 @@ __global__ void __launch_bounds__(32, 1) k_enum_walk(const EnumArgs a)
         my.g0n = kg.y;
         my.cand = a.cand + row * ECAP;
         my.ccount = a.cand_count + row;
+        my.stats = a.stats;
     }
     {
         const uint32_t wmask = __ballot_sync(FW_FULL, my_walk);
@@ -1288,6 +1334,7 @@ fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, f
     a.fb_list = (int32_t *)w;
     w += align256((size_t)R.rows * 4);
     a.fb_count = (int32_t *)w;
+    a.stats = (unsigned long long *)(w + 64);  // the same 256-byte block, zeroed below
     w += 256;
     a.fb_e = (double *)w;
     w += align256((size_t)R.rows * FBS * 8);
@@ -1299,7 +1346,9 @@ fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, f
     w += align256((size_t)R.rows * PERM);
     a.kg = (float2 *)w;
     a.stride = enum_stride(R.max_n, k_max);
-    FW_CUDA_CHECK(cudaMemsetAsync(a.fb_count, 0, sizeof(int32_t), s));
+    FW_CUDA_CHECK(cudaMemsetAsync(a.fb_count, 0, 256, s));
+    int sms = 0;
+    if (device_sms(&sms) != FW_OK) return FW_ERR_CUDA;
     FW_DISPATCH(R.d, R.v_dtype, {
         constexpr int DCH = DPL * 32 < 64 ? DPL * 32 : 64;
         const int ust = (((R.max_n + 1) * (DCH + 1)) + 1) & ~1;
@@ -1317,9 +1366,39 @@ fw_status best_subset(const RowsDev &R, const int32_t *k, uint64_t *best_rank, f
         const size_t smem2 = (size_t)33 * (2 * DPL * 32 + 1) * sizeof(float);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_enum_exhaustive<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)smem2));
-        FW_LAUNCH((k_enum_exhaustive<DPL, VT>), 152 * 4, 256, smem2, s, a);
+        FW_LAUNCH((k_enum_exhaustive<DPL, VT>), (unsigned)sms * 4, 256, smem2, s, a);
         FW_LAUNCH(k_enum_exhaustive_merge, 8, 128, 0, s, a);
     });
+    return FW_OK;
+}
+
+fw_status best_subset_stats(const RowsDev &R, const void *ws, fw_best_subset_stats *out, cudaStream_t s)
+{
+    const char *w = (const char *)ws;
+    const int32_t *cand_count = (const int32_t *)(w + align256((size_t)R.rows * ECAP * 4));
+    const char *blk = w + align256((size_t)R.rows * ECAP * 4) + 2 * align256((size_t)R.rows * 4);
+    int32_t fb = 0;
+    unsigned long long st[4] = {0, 0, 0, 0};
+    if (cudaMemcpyAsync(&fb, blk, 4, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaMemcpyAsync(st, blk + 64, sizeof(st), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return FW_ERR_CUDA;
+    int64_t cands = 0;
+    int32_t buf[4096];
+    for (int64_t r0 = 0; r0 < R.rows; r0 += 4096) {
+        const int64_t cnt = R.rows - r0 < 4096 ? R.rows - r0 : 4096;
+        if (cudaMemcpyAsync(buf, cand_count + r0, (size_t)cnt * 4, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+            cudaStreamSynchronize(s) != cudaSuccess)
+            return FW_ERR_CUDA;
+        for (int64_t i = 0; i < cnt; ++i)
+            if (buf[i] > 0 && buf[i] <= ECAP) cands += buf[i];
+    }
+    out->rows_exhaustive = fb;
+    out->candidates = cands;
+    out->inner_nodes = st[0];
+    out->inner_leaves = st[1];
+    out->inner_ops = st[2];
+    out->skipped = st[3];
     return FW_OK;
 }
 

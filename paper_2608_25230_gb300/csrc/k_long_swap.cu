@@ -897,8 +897,14 @@ template <int DPL> size_t ls_smem(int Ep)
 
 }  // namespace
 
-// LS_BPS resident blocks per SM (the launch bounds guarantee the registers for it)
-static unsigned ls_grid(const RowsDev &R) { return (unsigned)std::min<int64_t>(R.rows, 152 * LS_BPS); }
+// LS_BPS resident blocks per SM (the launch bounds guarantee the registers for
+// it); the workspace is sized by the same count, queried from the current device
+static unsigned ls_grid(const RowsDev &R)
+{
+    int sms = 0;
+    if (device_sms(&sms) != FW_OK) sms = 152;  // no device: the size query still answers
+    return (unsigned)std::min<int64_t>(R.rows, (int64_t)sms * LS_BPS);
+}
 
 static size_t ls_array_bytes(const RowsDev &R) { return align256((size_t)ls_grid(R) * R.max_n * 4); }
 

@@ -7,7 +7,8 @@
 // set with Definition 2.1's quantities (es(A) = ||m_A - mu|| and the dropped
 // mass of the row's own masses).  Three launches, each one pass over HBM:
 //   k_vote_mass    G of every group: one thread per key walks the group's rows
-//                  in order (loads coalesced over keys); flags non-finite logits.
+//                  in order (loads coalesced over keys) with a compensated sum;
+//                  flags non-finite logits.
 //                  Each mass is the fast exponential times 1/Z of its row (a few
 //                  ulp): an accurate exp and a divide per (row, key) would make
 //                  this pass and the scoring pass instruction-bound.
@@ -66,7 +67,9 @@ __global__ void __launch_bounds__(VM_T) k_vote_mass(VoteArgs a)
         bool bad = false;
         for (int j0 = blockIdx.x * VM_T; j0 < n; j0 += gridDim.x * VM_T) {
             const int j = j0 + tid;
-            float acc = 0.f;
+            // compensated sum (TwoSum, errors carried in lo): the rounding of the
+            // sum stays at about one ulp of G whatever the group size
+            float hi = 0.f, lo = 0.f;
             for (int i0 = 0; i0 < Rg; i0 += VM_T) {
                 const int cnt = min(VM_T, Rg - i0);
                 __syncthreads();
@@ -82,11 +85,14 @@ __global__ void __launch_bounds__(VM_T) k_vote_mass(VoteArgs a)
                     for (int i = 0; i < cnt; ++i) {
                         const float l = __ldg(col + (int64_t)i * n);
                         bad |= !isfinite(l);
-                        acc = fmaf(__expf(l - sM[i]), sZ[i], acc);
+                        const float p = __expf(l - sM[i]) * sZ[i];
+                        const float t = hi + p, bb = t - hi;
+                        lo += (hi - (t - bb)) + (p - bb);
+                        hi = t;
                     }
                 }
             }
-            if (j < n) G[j] = acc;
+            if (j < n) G[j] = hi + lo;
         }
         if (__syncthreads_or(bad) && tid == 0) a.gflag[g] = FW_ERR_NONFINITE;
     }
@@ -456,8 +462,10 @@ fw_status group_vote(const RowsDev &R, const int32_t *s, int nb, const fw_gap_ou
     a.staged = R.max_n <= VS_STAGE_MAX;
     FW_CUDA_CHECK(cudaMemsetAsync(a.gflag, 0, (size_t)R.num_groups * 4, st));
 
+    int sms = 0;
+    if (device_sms(&sms) != FW_OK) return FW_ERR_CUDA;
     const int64_t chunks = (R.max_n + VM_T - 1) / VM_T;
-    const int64_t per_group = std::max<int64_t>(1, (152 * 8 + R.num_groups - 1) / R.num_groups);
+    const int64_t per_group = std::max<int64_t>(1, ((int64_t)sms * 8 + R.num_groups - 1) / R.num_groups);
     const dim3 gm((unsigned)std::min(chunks, per_group), (unsigned)std::min<int64_t>(R.num_groups, 65535));
     FW_LAUNCH(k_vote_mass, gm, VM_T, 0, st, a);
 

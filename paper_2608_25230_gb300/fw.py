@@ -39,6 +39,11 @@ class FwGapOut(C.Structure):
                 ("kept_words", C.c_int32), ("row_status", vp)]
 
 
+class FwBestSubsetStats(C.Structure):
+    _fields_ = [("rows_exhaustive", C.c_int64), ("candidates", C.c_int64), ("inner_nodes", C.c_uint64),
+                ("inner_leaves", C.c_uint64), ("inner_ops", C.c_uint64), ("skipped", C.c_uint64)]
+
+
 class FwSwapParams(C.Structure):
     _fields_ = [("E", C.c_int32), ("max_swaps", C.c_int32)]
 
@@ -53,6 +58,8 @@ _lib.fw_swap_refine_workspace.restype = C.c_size_t
 _lib.fw_best_subset.argtypes = [C.POINTER(FwRows), vp, vp, vp, vp, C.c_int32, vp, vp, vp, C.c_size_t, vp]
 _lib.fw_best_subset_workspace.argtypes = [C.POINTER(FwRows)]
 _lib.fw_best_subset_workspace.restype = C.c_size_t
+_lib.fw_best_subset_read_stats.argtypes = [C.POINTER(FwRows), vp, C.POINTER(FwBestSubsetStats), vp]
+_lib.fw_best_subset_read_stats.restype = C.c_int
 _lib.fw_contour_alloc.argtypes = [vp, C.c_int32, C.c_int32, C.c_int32, C.c_int64, C.c_int32, vp, vp, vp, vp, vp,
                                   vp, vp, C.c_size_t, vp]
 _lib.fw_contour_alloc_workspace.argtypes = [C.c_int32, C.c_int32]
@@ -251,6 +258,16 @@ def best_subset(rows: Rows, k: torch.Tensor, *, k_max=None, stream=None, ws=None
     _check(st, "fw_best_subset")
     out["_ws"] = ws
     return out
+
+
+def best_subset_stats(rows: Rows, out: dict, stream=None) -> dict:
+    """fw_best_subset_read_stats for the call that returned `out` (waits for
+    the stream): rows sent to the exhaustive path, re-scored candidates, and
+    the walk's inner enumerations, leaves, fp32 operations and skipped nodes."""
+    st = FwBestSubsetStats()
+    _check(_lib.fw_best_subset_read_stats(C.byref(rows.c), _ptr(out["_ws"]), C.byref(st), _stream(stream)),
+           "fw_best_subset_read_stats")
+    return {name: int(getattr(st, name)) for name, _ in FwBestSubsetStats._fields_}
 
 
 def pool_best_subset(rows: Rows, k: torch.Tensor, topk: dict, *, E, k_max: int = 32, stream=None):

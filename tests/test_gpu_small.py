@@ -250,9 +250,32 @@ def test_best_hardness_instance(fw):
     assert np_(bs["best_gap"])[0] >= 2.0 / m ** 2 * (1 - 1e-5)
 
 
+@pytest.mark.parametrize("kind", workloads.ADVERSARIAL_KINDS)
+def test_best_adversarial_rows(fw, kind):
+    """512 rows of each adversarial kind (flat rows, near-duplicate values,
+    planted ES = 0 rows with exact ties) against the oracle, every row.  Where
+    the oracle's best gap is exactly 0 (a planted row: every quantity is a short
+    binary fraction, so the ties are exact on both sides) the rank must be the
+    smallest colex rank among the tied subsets, the oracle's, with no near-tie
+    exemption."""
+    b = workloads.exact_adversarial(kind, rows=512, seed=0)
+    bs, o = check_best(fw, b)
+    zero = o["best_gap"] == 0.0
+    if kind.startswith("planted"):
+        assert zero.all()
+        np.testing.assert_array_equal(np_(bs["best_rank"]).astype(np.uint64)[zero], o["best_rank"][zero])
+        assert np.all(np_(bs["best_gap"])[zero] == 0.0)
+    rows = fw.rows_from_batch(b)
+    st = fw.best_subset_stats(rows, bs)
+    print(f"{kind}: {st['rows_exhaustive']} of {rows.num_rows} rows on the exhaustive path, "
+          f"{st['candidates']} candidates re-scored, {st['inner_leaves']} leaves visited")
+    assert 0 <= st["rows_exhaustive"] <= rows.num_rows
+
+
 def test_best_full_scale_sampled(fw):
-    """The measured workload (168,192 rows, n=24, k=6) in one call per group;
-    sampled rows checked against the oracle, properties on every row."""
+    """The measured workload (168,192 rows, n=24, k=6) in one call per group:
+    2,000 rows of every group (10,000 in all) against the oracle, properties on
+    every row."""
     rng = np.random.default_rng(5)
     for b in workloads.exact_enum(seed=0, backend="torch", device="cuda"):
         rows = fw.rows_from_batch(b)
@@ -265,13 +288,22 @@ def test_best_full_scale_sampled(fw):
         assert np.all(best <= tg * (1 + 1e-6))
         np.testing.assert_allclose(tg, np_(top["gap"])[:, 0], rtol=1e-5)
         assert np.all(np_(bs["best_rank"]) < math.comb(24, 6))
-        pick = np.sort(rng.choice(rows.num_rows, 6, replace=False))
+        pick = np.sort(rng.choice(rows.num_rows, 2000, replace=False))
         sub = _subset_rows(b, pick)
         o = oracle.best_subset(sub)
         on = row_onorm(oracle.dense_and_topk_gap(sub)["o"])
         assert_close(best[pick], o["best_gap"], on, "best_gap (sampled)")
+        assert_close(tg[pick], o["topk_gap"], on, "topk_gap (sampled)")
         tie = (o["second_gap"] - o["best_gap"]) < NEAR_TIE * o["best_gap"]
+        assert tie.mean() < 0.01
         np.testing.assert_array_equal(np_(bs["best_rank"])[pick][~tie].astype(np.uint64), o["best_rank"][~tie])
+        idx = np_(bs["best_idx"])[pick]
+        np.testing.assert_array_equal(idx[~tie], o["best_idx"][~tie])
+        st = fw.best_subset_stats(rows, bs)
+        print(f"group d={b.d}: {rows.num_rows} rows, {st['rows_exhaustive']} on the exhaustive path, "
+              f"{st['candidates']} candidates, {st['inner_leaves']} leaves, {st['skipped']} skipped")
+        del rows, top, bs, b
+        torch.cuda.empty_cache()
 
 
 def _subset_rows(b, pick):

@@ -31,15 +31,19 @@ def fw():
     return _fw
 
 
-def call_noalloc(fw, scores, floor, budget, s):
-    dev = scores.device
+def new_outputs(cells, budget, dev):
+    return dict(counts=torch.full((cells,), -7, dtype=torch.int32, device=dev),
+                offsets=torch.full((cells + 1,), -7, dtype=torch.int64, device=dev),
+                kept_pos=torch.full((budget,), -7, dtype=torch.int32, device=dev),
+                tau=torch.zeros(1, dtype=torch.float32, device=dev),
+                dropped_uniform=torch.zeros(cells, dtype=torch.float32, device=dev),
+                dropped_alloc=torch.zeros(cells, dtype=torch.float32, device=dev))
+
+
+def call_noalloc(fw, scores, floor, budget, s, out=None):
     cells, T = scores.shape
-    out = dict(counts=torch.full((cells,), -7, dtype=torch.int32, device=dev),
-               offsets=torch.full((cells + 1,), -7, dtype=torch.int64, device=dev),
-               kept_pos=torch.full((budget,), -7, dtype=torch.int32, device=dev),
-               tau=torch.zeros(1, dtype=torch.float32, device=dev),
-               dropped_uniform=torch.zeros(cells, dtype=torch.float32, device=dev),
-               dropped_alloc=torch.zeros(cells, dtype=torch.float32, device=dev))
+    if out is None:
+        out = new_outputs(cells, budget, scores.device)
     p = lambda t: C.c_void_p(t.data_ptr())  # noqa: E731
     st = fw.raw().fw_contour_alloc_noalloc(p(scores), cells, T, floor, budget, s, p(out["counts"]),
                                            p(out["offsets"]), p(out["kept_pos"]), p(out["tau"]),
@@ -66,6 +70,31 @@ def test_noalloc_matches_the_workspace_entry_point_on_consecutive_calls(fw):
         one = np.ones(sc.shape[0])
         assert_close(np_(got["dropped_alloc"]), np_(ref["dropped_alloc"]), one, "dropped_alloc")
         assert_close(np_(got["dropped_uniform"]), np_(ref["dropped_uniform"]), one, "dropped_uniform")
+
+
+def test_noalloc_at_its_largest_size_allocates_nothing(fw):
+    # exactly FW_CONTOUR_NOALLOC_MAX_CELLS cells (the shared array filled to its
+    # limit), bit for bit against the workspace entry point; the device's free
+    # memory is the same before and after the call
+    cells = 4096
+    cb = workloads.contour_cache(seed=77, cells=cells, T=96, with_kv=False, budget_frac=1 / 2)
+    sc = torch.as_tensor(cb.scores).cuda()
+    ref = fw.contour_alloc(sc, floor=cb.floor, total_budget=cb.total_budget, uniform_s=cb.uniform_s)
+    st, _ = call_noalloc(fw, sc, cb.floor, cb.total_budget, cb.uniform_s)  # the module is loaded after this
+    assert st == 0, st
+    got = new_outputs(cells, cb.total_budget, sc.device)  # outputs allocated before the measured call
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    st, got = call_noalloc(fw, sc, cb.floor, cb.total_budget, cb.uniform_s, out=got)
+    torch.cuda.synchronize()
+    free1 = torch.cuda.mem_get_info()[0]
+    assert st == 0, st
+    assert free1 == free0
+    for key in ("counts", "offsets", "kept_pos", "tau"):
+        np.testing.assert_array_equal(np_(got[key]), np_(ref[key]), err_msg=key)
+    one = np.ones(cells)
+    assert_close(np_(got["dropped_alloc"]), np_(ref["dropped_alloc"]), one, "dropped_alloc")
+    assert_close(np_(got["dropped_uniform"]), np_(ref["dropped_uniform"]), one, "dropped_uniform")
 
 
 def test_noalloc_rejects_more_cells_than_its_scratch_holds(fw):

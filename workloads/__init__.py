@@ -257,6 +257,56 @@ def exact_enum(seed: int = 0, rows_scale: float = 1.0, n: int = 24, k: int = 6,
     return out
 
 
+# Adversarial inputs for the exact search (n <= 32), each a stress on a
+# different part of it:
+#   flat      n=24, k=6, d=64: logits Gumbel*0.3 and no sink, so many subsets
+#             have es close to the best and few bounds exclude anything;
+#   near_dup  n=24, k=6, d=64: values = one point + eps*N(0,1) (eps cycling
+#             through 1e-2, 1e-3, 1e-4), logits as in exact_enum: es of every
+#             subset within a few eps of the others;
+#   planted   n=32, k=4, d=32: uniform logits and integer points in the first
+#             dimension (the rest 0), with one random 4-subset planted so that
+#             its mean equals the mean of all 32 points -- es = 0 exactly, and
+#             every other 4-subset with that mean ties with it (App. A.2 builds
+#             its hardness instances the same way);
+#   planted_half  n=16, k=8, d=32: App. A.2's construction itself, uniform
+#             masses and a planted split of the points into two halves of
+#             equal sum (es = 0 exactly for the planted half, usually many
+#             more).
+# Uniform masses over 16 or 32 keys and integer points keep every quantity a
+# short binary fraction, so es = 0 holds exactly in floating point too.
+ADVERSARIAL_KINDS = ("flat", "near_dup", "planted", "planted_half")
+
+
+def exact_adversarial(kind: str, rows: int = 512, seed: int = 0) -> RowBatch:
+    rng = _NumpyRng(seed * 1000 + 300 + ADVERSARIAL_KINDS.index(kind))
+    if kind == "flat":
+        n, k, d = 24, 6, 64
+        l = rng.gumbel((rows, n)) * np.float32(0.3)
+        v = rng.normal((rows, n, d))
+    elif kind == "near_dup":
+        n, k, d = 24, 6, 64
+        tau = rng.uniform((rows, 1), 0.5, 3.0)
+        l = rng.gumbel((rows, n)) * tau
+        l[:, 0] += 6.0
+        eps = np.array([1e-2, 1e-3, 1e-4], np.float32)[np.arange(rows) % 3][:, None, None]
+        v = (rng.normal((rows, 1, d)) + eps * rng.normal((rows, n, d))).astype(np.float32)
+    elif kind in ("planted", "planted_half"):
+        n, k, d = (32, 4, 32) if kind == "planted" else (16, 8, 32)
+        l = np.zeros((rows, n), np.float32)
+        w = np.floor(rng.uniform((rows, n), -8.0, 9.0)).astype(np.int64)
+        v = np.zeros((rows, n, d), np.float32)
+        for r in range(rows):
+            perm = rng.g.permutation(n)
+            A, out = perm[:k], perm[k:]
+            # make sum(all) = (n / k) * sum(A) by moving one point outside A
+            w[r, out[0]] += (n // k) * w[r, A].sum() - w[r].sum()
+            v[r, :, 0] = w[r]
+    else:
+        raise ValueError(kind)
+    return _batch_rows_own_v(rng, l.astype(np.float32), v.astype(np.float32), n, d, k, f"adversarial_{kind}")
+
+
 def _batch_rows_own_v(rng, l, v, n, d, k, name):
     """Each row is its own group (R = 1): rows are contiguous, V blocks too."""
     rows = l.shape[0]
