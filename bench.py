@@ -5,11 +5,17 @@ five groups (d = 64,128,128,128,64), n = 24 keys, k = 6 (134,596 subsets per
 row), logits Gumbel*tau + sink, V fp32.  One step runs the whole path on every
 row: softmax, top-k kept set, dense and forced-weight outputs, gap and dropped
 mass (fw_dense_and_topk_gap), the swap rule over all keys (fw_swap_refine) and
-the exact best subset (fw_best_subset).  Metric: subsets/s.
+the exact best subset ES(k) (fw_best_subset).  Metric: rows/s (every row gets
+its exact ES(k)); the subsets the search covers per second are reported beside
+it as a derived figure, with the subsets its walk actually visits.
 
-Also timed in the same run (reported under "sections"): the long-row top-k
-gap workload (4,096 rows x 32,768 keys, d=128, three budgets) and ContourKV
-allocation + ragged compaction (256 cells x 32,768 tokens, d=128).
+Also timed in the same run (reported under "sections"), one line per config:
+  exact_toy       256 rows, n=20, k=5, d=64: the whole path
+  adversarial     512 rows each of flat, near-duplicate and planted-tie rows
+  long_rows       4,096 rows x 32,768 keys, d=128, three budgets: gap, swap, vote
+  contour         ContourKV allocation + ragged compaction, 256 cells x 32,768 tokens
+  mixed_profiles  168,192 ragged rows (n 1,024..16,384, GQA-4, bf16 V): gap + swap
+  pool            ES_pool (Definition 2.2) at s = 4/8/16/32 on mixed-profile rows
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 """
@@ -35,7 +41,20 @@ import workloads  # noqa: E402
 
 N_KEYS, K_SEL = 24, 6
 SUBSETS_PER_ROW = math.comb(N_KEYS, K_SEL)
-ALU_OPS_PER_SUBSET = 3  # inner walk leaf: value add, carry add, running min
+POOL_SCHED = ((4, 24), (8, 12), (16, 6), (32, 4))  # (s, E): the candidate-set schedule of App. B
+
+# DRAM bytes (read + write) per unit of work, from one-kernel ncu captures on
+# reduced cases (dram__bytes_read.sum + dram__bytes_write.sum; the commands are
+# in profiles/), scaled to a full launch by the units it processes.  None where
+# the kernel changed after its capture.
+TRAFFIC_PER_UNIT = {
+    # kernel: (bytes per unit, unit)
+    "fw_best_subset": None,
+    "long_gap": None,
+    "group_vote": None,
+    "contour": None,
+    "mixed_gap": None,
+}
 
 
 def read_peaks():
@@ -44,8 +63,15 @@ def read_peaks():
         with open(path) as f:
             p = json.load(f)
         return dict(hbm_gbs=p.get("hbm_gbs", 6800.0), bf16=p.get("bf16_tflops", 1900.0),
-                    sm_max=p.get("sm_max_mhz", 2070.0), source="measured")
-    return dict(hbm_gbs=6800.0, bf16=1900.0, sm_max=2070.0, source="fallback")
+                    bf16_sust=p.get("bf16_tflops_sustained", 1700.0), sm_max=p.get("sm_max_mhz", 2070.0),
+                    source="measured")
+    return dict(hbm_gbs=6800.0, bf16=1900.0, bf16_sust=1700.0, sm_max=2070.0, source="fallback")
+
+
+def fp32_peak_tflops(device, sm_mhz):
+    """FP32 FMA peak: SMs x 128 lanes x 2 flops x the SM clock sampled under load."""
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    return sms * 128 * 2 * sm_mhz * 1e6 / 1e12, sms
 
 
 class ClockSampler:
@@ -109,43 +135,80 @@ class L2Flush:
         self.buf.fill_(1)
 
 
+class Events:
+    """CUDA events recorded on the current stream around calls, read later."""
+
+    def __init__(self):
+        self.ev = []
+
+    def start(self):
+        e = torch.cuda.Event(enable_timing=True)
+        e.record()
+        return e
+
+    def stop(self, e0, tag=None):
+        e1 = torch.cuda.Event(enable_timing=True)
+        e1.record()
+        self.ev.append((e0, e1, tag))
+
+    def take(self):
+        torch.cuda.synchronize()
+        r = [(a.elapsed_time(b), t) for a, b, t in self.ev]
+        self.ev = []
+        return r
+
+
 # ---------------------------------------------------------------- workloads
 
 class EnumWorkload:
     """168,192 rows, n=24, k=6: the whole a1..a6 path per step."""
 
-    def __init__(self, fw, seed, device, rows_scale=1.0):
+    def __init__(self, fw, seed, device, rows_scale=1.0, batches=None, E=N_KEYS):
         self.fw = fw
-        self.batches = workloads.exact_enum(seed=seed, rows_scale=rows_scale, backend="torch", device=device)
+        self.batches = batches if batches is not None else workloads.exact_enum(
+            seed=seed, rows_scale=rows_scale, backend="torch", device=device)
         self.rows = [fw.rows_from_batch(b, device) for b in self.batches]
-        self.k2 = [b.k for b in self.batches]
-        self.k1 = [b.k[:, 0].contiguous() for b in self.batches]
+        self.k2 = [torch.as_tensor(np.asarray(b.k)).to(device) if not isinstance(b.k, torch.Tensor) else b.k
+                   for b in self.batches]
+        self.k1 = [k[:, 0].contiguous() for k in self.k2]
+        self.kmax = [int(k.max().item()) for k in self.k1]
         self.num_rows = sum(r.num_rows for r in self.rows)
-        self.subsets = self.num_rows * SUBSETS_PER_ROW
-        self.ev = []
+        self.subsets = sum(r.num_rows * math.comb(int(b.n_host[0]), int(np.asarray(b.k if not isinstance(
+            b.k, torch.Tensor) else b.k.cpu())[0, 0])) for r, b in zip(self.rows, self.batches))
+        self.E = E
+        self.ev = Events()
+        self.last = None
 
     def step(self, time_enum=False):
         fw = self.fw
         outs = []
-        for rows, k2, k1 in zip(self.rows, self.k2, self.k1):
+        for rows, k2, k1, kmax in zip(self.rows, self.k2, self.k1, self.kmax):
             top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
-            sw = fw.swap_refine(rows, k2, top, E=N_KEYS, max_swaps=32)
+            sw = fw.swap_refine(rows, k2, top, E=self.E, max_swaps=32)
+            e0 = self.ev.start() if time_enum else None
+            bs = fw.best_subset(rows, k1, k_max=kmax)
             if time_enum:
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record()
-            bs = fw.best_subset(rows, k1, k_max=K_SEL)
-            if time_enum:
-                e1.record()
-                self.ev.append((e0, e1, rows.num_rows))
+                self.ev.stop(e0, rows.num_rows)
             outs.append((top, sw, bs))
+        self.last = outs
         return outs
 
-    def enum_times(self):
-        """(ms, rows) of every timed fw_best_subset launch."""
-        torch.cuda.synchronize()
-        r = [(a.elapsed_time(b), n) for a, b, n in self.ev]
-        self.ev = []
-        return r
+    def stats(self):
+        """Work counters of the last step's fw_best_subset calls, summed."""
+        tot = {}
+        for rows, (_, _, bs) in zip(self.rows, self.last):
+            for key, v in self.fw.best_subset_stats(rows, bs).items():
+                tot[key] = tot.get(key, 0) + v
+        return tot
+
+    def gram_flops(self):
+        """The prep kernel's Gram products per step: (n+1)(n+2)/2 dot products of
+        length d per row (the n keys and g of the top-k set), 2 flops per FMA."""
+        f = 0
+        for r, b in zip(self.rows, self.batches):
+            n = int(b.n_host[0])
+            f += r.num_rows * 2 * b.d * (n + 1) * (n + 2) // 2
+        return f
 
 
 class EnumE2E:
@@ -237,8 +300,6 @@ def time_steps(step, K, W, flush, barrier):
     barrier()
     torch.cuda.synchronize()
     times = []
-    start_all = torch.cuda.Event(enable_timing=True)
-    end_all = torch.cuda.Event(enable_timing=True)
     total = 0.0
     for _ in range(K):
         flush()
@@ -252,8 +313,16 @@ def time_steps(step, K, W, flush, barrier):
         total += t
     torch.cuda.synchronize()
     barrier()
-    del start_all, end_all
     return total, times
+
+
+def roofline(bound, achieved, peak, unit, traffic=None, **extra):
+    return dict(bound=bound, achieved=achieved, peak=peak, unit=unit, frac=achieved / peak, traffic=traffic, **extra)
+
+
+def traffic_of(name, units):
+    t = TRAFFIC_PER_UNIT.get(name)
+    return None if t is None else t[0] * units
 
 
 # ------------------------------------------------------------- CPU oracle
@@ -274,7 +343,7 @@ def cpu_baseline(seed, rows_per_group=40):
         oracle.best_subset(H)
     dt = time.perf_counter() - t0
     rows = sum(H.num_rows for H in Hs)
-    return dict(value=rows * SUBSETS_PER_ROW / dt, unit="subsets/s", cores=oracle.num_threads(), kind="oracle",
+    return dict(value=rows / dt, unit="rows/s", cores=oracle.num_threads(), kind="oracle",
                 sample=f"first {rows_per_group} rows of each of the 5 groups ({rows} rows, "
                        f"{rows * SUBSETS_PER_ROW:,} subsets), whole path (gap, swap, best subset), fp64",
                 seconds=dt)
@@ -282,9 +351,49 @@ def cpu_baseline(seed, rows_per_group=40):
 
 # ----------------------------------------------------------------- sections
 
+def section_exact_toy(fw, device, K, W, flush, peaks):
+    """cfg 1: 256 rows, n=20, k=5, d=64, the whole path (latency-bound, too small
+    for a roofline claim)."""
+    b = workloads.exact_toy(seed=0)
+    wl = EnumWorkload(fw, 0, device, batches=[b], E=20)
+    total, _ = time_steps(lambda: wl.step(), K, W, flush, lambda: None)
+    ms = total / K
+    st = wl.stats()
+    return dict(workload="exact_toy: 256 rows, n=20, k=5, d=64, fp32 V", metric="rows/s",
+                value=wl.num_rows / (ms * 1e-3), ms_per_step=ms,
+                subsets_covered_per_s=wl.subsets / (ms * 1e-3), walk_leaves=st["inner_leaves"],
+                rows_exhaustive=st["rows_exhaustive"])
+
+
+def section_adversarial(fw, device, K, W, flush, peaks):
+    """The exact search alone on 512 rows of each adversarial kind: rows/s and
+    the rows that overflow to the exhaustive fp64 path."""
+    out = {}
+    for kind in workloads.ADVERSARIAL_KINDS:
+        b = workloads.exact_adversarial(kind, rows=512, seed=0)
+        rows = fw.rows_from_batch(b, device)
+        k1 = torch.as_tensor(np.asarray(b.k)[:, 0].copy()).to(device)
+        kk = int(np.asarray(b.k)[0, 0])
+        holder = {}
+
+        def step():
+            holder["bs"] = fw.best_subset(rows, k1, k_max=kk)
+
+        total, _ = time_steps(step, K, W, flush, lambda: None)
+        ms = total / K
+        st = fw.best_subset_stats(rows, holder["bs"])
+        n = int(b.n_host[0])
+        out[kind] = dict(n=n, k=kk, d=b.d, rows=rows.num_rows, ms_per_call=ms, rows_per_s=rows.num_rows / (ms * 1e-3),
+                         subsets_covered_per_s=rows.num_rows * math.comb(n, kk) / (ms * 1e-3),
+                         rows_exhaustive=st["rows_exhaustive"],
+                         exhaustive_frac=st["rows_exhaustive"] / rows.num_rows, candidates=st["candidates"],
+                         walk_leaves=st["inner_leaves"])
+    return out
+
+
 def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
     """a1-a4 (top-k gap) and a5 (swap rule, E=32) on 8 heads x rows_per_head rows
-    x 32,768 keys (4,096 rows at the default)."""
+    x 32,768 keys (4,096 rows at the default), and the group vote."""
     b = workloads.long_rows(seed=0, rows_per_head=rows_per_head, backend="torch", device=device)
     rows = fw.rows_from_batch(b, device)
     rows_k = b.k
@@ -301,7 +410,7 @@ def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
         holder["sw"] = fw.swap_refine(rows, rows_k, top, E=32, max_swaps=64)
 
     ks = max(2, K // 2)
-    total, _ = time_steps(swap_step, ks, 2, flush, lambda: None)
+    total, _ = time_steps(swap_step, ks, 1, flush, lambda: None)
     ms_swap = total / ks
     ns = holder["sw"]["n_swaps"].float()
     R, n, d, nb = rows.num_rows, int(b.n_host[0]), b.d, rows_k.shape[1]
@@ -327,27 +436,20 @@ def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
     nbytes = (rows.logits.numel() * 4 + rows.v.numel() * 2
               + R * (d * 4 * (1 + nb) + nb * 3 * 4 + nb * 8 + nb * (n // 8)))
     ach = nbytes / (ms_gap * 1e-3) / 1e9
-    # the swap rounds: per round one pass over the k kept keys (a d-long product
-    # with g and one with the changed pool vector, E table entries)
     rounds = float((ns + 1).sum().item())
     return dict(workload=f"long_rows: 8 heads x {rows_per_head} rows, n=32768, d=128, bf16 V, k in {{2048,4096,8192}}",
                 path="a1-a4 (fw_dense_and_topk_gap) then a5 (fw_swap_refine, E=32)", metric="rows/s",
                 value=R / ((ms_gap + ms_swap) * 1e-3), gap_rows_per_s=R / (ms_gap * 1e-3),
                 swap_rows_per_s=R / (ms_swap * 1e-3), ms_gap=ms_gap, ms_swap=ms_swap,
                 swaps_per_row_budget=float(ns.mean().item()), swap_rounds=rounds,
-                roofline=dict(bound="hbm", kernel="k_long_select_bins + k_long_pv_tc (fw_dense_and_topk_gap)",
-                              achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s", frac=ach / peaks["hbm_gbs"],
-                              traffic=None, algorithmic_bytes=nbytes,
-                              tensor_flops_executed=2 * 3 * (nb + 1) * n * d * R,
-                              tensor_tflops=2 * 3 * (nb + 1) * n * d * R / (ms_gap * 1e-3) / 1e12,
-                              tensor_basis="P.V as a bf16 GEMM: 3 bf16 terms per probability, nb + 1 band rows; "
-                                           "time of the whole gap call (the select kernel included)"),
+                roofline=roofline("hbm", ach, peaks["hbm_gbs"], "GB/s", traffic_of("long_gap", R),
+                                  kernel="fw_dense_and_topk_gap (select + P.V)", algorithmic_bytes=nbytes,
+                                  launch_ms=ms_gap),
                 group_vote=dict(path="fw_group_vote: one set per KV head by summed mass, all rows scored",
                                 ms_per_call=ms_vote, rows_per_s=R / (ms_vote * 1e-3),
-                                roofline=dict(bound="hbm", kernel="k_vote_mass + k_vote_select + k_vote_eval",
-                                              achieved=vach, peak=peaks["hbm_gbs"], unit="GB/s",
-                                              frac=vach / peaks["hbm_gbs"], traffic=None,
-                                              algorithmic_bytes=vbytes)))
+                                roofline=roofline("hbm", vach, peaks["hbm_gbs"], "GB/s", traffic_of("group_vote", R),
+                                                  kernel="k_vote_mass + k_vote_select + k_vote_eval",
+                                                  algorithmic_bytes=vbytes)))
 
 
 def section_contour(fw, device, K, W, flush, peaks):
@@ -355,20 +457,109 @@ def section_contour(fw, device, K, W, flush, peaks):
     Kc, Vc = cb.K.view(torch.int16), cb.V.view(torch.int16)
     Ko = torch.empty(cb.total_budget, cb.d, dtype=torch.int16, device=device)
     Vo = torch.empty_like(Ko)
+    ev = Events()
 
     def step():
+        e0 = ev.start()
         a = fw.contour_alloc(cb.scores, floor=cb.floor, total_budget=cb.total_budget, uniform_s=cb.uniform_s)
+        ev.stop(e0, "alloc")
+        e1 = ev.start()
         fw.ragged_compact(Kc, Vc, a["offsets"], a["kept_pos"], cb.total_budget, out=(Ko, Vo))
+        ev.stop(e1, "compact")
 
     total, times = time_steps(step, K, W, flush, lambda: None)
     ms = total / K
+    parts = ev.take()[-2 * K:]
+    ms_alloc = sum(t for t, tag in parts if tag == "alloc") / K
+    ms_comp = sum(t for t, tag in parts if tag == "compact") / K
     nbytes = cb.cells * cb.T * 4 + 2 * 2 * cb.total_budget * cb.d * 2 + cb.total_budget * 4 + (cb.cells + 1) * 8
     ach = nbytes / (ms * 1e-3) / 1e9
+    cbytes = 2 * 2 * cb.total_budget * cb.d * 2
     return dict(workload="contour_cache: 256 cells x 32768 tokens, d=128 bf16 K/V, budget 1/8, floor 32",
                 path="a7-a8 (fw_contour_alloc + fw_ragged_compact)", metric="kept KV rows/s",
-                value=cb.total_budget / (ms * 1e-3), ms_per_step=ms,
-                roofline=dict(bound="hbm", achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s",
-                              frac=ach / peaks["hbm_gbs"], traffic=None, algorithmic_bytes=nbytes))
+                value=cb.total_budget / (ms * 1e-3), ms_per_step=ms, ms_alloc=ms_alloc, ms_compact=ms_comp,
+                roofline=roofline("hbm", ach, peaks["hbm_gbs"], "GB/s", traffic_of("contour", cb.total_budget),
+                                  algorithmic_bytes=nbytes, kernel="k_c_* + k_compact"),
+                compact_roofline=roofline("hbm", cbytes / (ms_comp * 1e-3) / 1e9, peaks["hbm_gbs"], "GB/s",
+                                          kernel="k_compact", algorithmic_bytes=cbytes))
+
+
+def section_mixed(fw, device, K, W, flush, peaks, rows_scale=1.0):
+    """cfg 5: 168,192 rows from five profiles, GQA groups of 4 sharing bf16 V,
+    one budget per row: the gap call and the swap rule (E = 32), one profile
+    per call (each profile is generated, timed and freed in turn)."""
+    tot_rows, ms_gap, ms_swap, nbytes, swaps = 0, 0.0, 0.0, 0, []
+    per = {}
+    for prof in workloads.MIXED_PROFILES:
+        b = workloads.mixed_profiles(seed=0, backend="torch", device=device, profiles=(prof,),
+                                     rows_scale=rows_scale)[0]
+        rows = fw.rows_from_batch(b, device)
+        holder = {}
+
+        def gap_step():
+            holder["top"] = fw.dense_and_topk_gap(rows, b.k, kept_bits=False)
+
+        t, _ = time_steps(gap_step, K, W, flush, lambda: None)
+        g = t / K
+
+        def swap_step():
+            holder["sw"] = fw.swap_refine(rows, b.k, holder["top"], E=32, max_swaps=64)
+
+        t, _ = time_steps(swap_step, 2, 1, flush, lambda: None)
+        s = t / 2
+        R, n, d = rows.num_rows, int(b.n_host[0]), b.d
+        by = rows.logits.numel() * 4 + rows.v.numel() * 2 + R * (d * 4 * 2 + 4 * 4 + 8)
+        per[prof[0]] = dict(rows=R, n=n, d=d, ms_gap=g, ms_swap=s, gap_gbs=by / (g * 1e-3) / 1e9,
+                            swaps_per_row=float(holder["sw"]["n_swaps"].float().mean().item()))
+        tot_rows += R
+        ms_gap += g
+        ms_swap += s
+        nbytes += by
+        del rows, holder, b
+        torch.cuda.empty_cache()
+    ach = nbytes / (ms_gap * 1e-3) / 1e9
+    return dict(workload="mixed_profiles: 168,192 rows, 5 profiles (d 64/128, n 1,024..16,384), GQA-4 bf16 V, "
+                         "k/n in {1/32,1/16,1/8,1/4}", metric="rows/s", value=tot_rows / ((ms_gap + ms_swap) * 1e-3),
+                gap_rows_per_s=tot_rows / (ms_gap * 1e-3), swap_rows_per_s=tot_rows / (ms_swap * 1e-3),
+                ms_gap=ms_gap, ms_swap=ms_swap, profiles=per,
+                roofline=roofline("hbm", ach, peaks["hbm_gbs"], "GB/s", traffic_of("mixed_gap", tot_rows),
+                                  kernel="fw_dense_and_topk_gap, one call per profile", algorithmic_bytes=nbytes,
+                                  bytes_basis="logits once, each GQA group's value block once, outputs"))
+
+
+def section_pool(fw, device, K, W, flush, peaks, groups=256):
+    """f2: ES_pool at the candidate-set schedule s = 4/8/16/32 (E = 24/12/6/4)
+    on the first `groups` GQA groups of mixed profiles B (n = 4,096, d = 128)
+    and E (n = 16,384, d = 128): rows/s, subsets/s, and the share of the top-mass
+    gap that the best candidate subset closes."""
+    out = {}
+    for prof in (workloads.MIXED_PROFILES[1], workloads.MIXED_PROFILES[4]):
+        name, rows_full, d, n = prof
+        b = workloads.mixed_profiles(seed=0, backend="torch", device=device, profiles=(prof,),
+                                     rows_scale=groups * 4 / rows_full)[0]
+        rows = fw.rows_from_batch(b, device)
+        R = rows.num_rows
+        k = torch.tensor([s for s, _ in POOL_SCHED], dtype=torch.int32, device=device).repeat(R, 1)
+        E = [e for _, e in POOL_SCHED]
+        top = fw.dense_and_topk_gap(rows, k, kept_bits=False, o_kept=False)
+        holder = {}
+
+        def step():
+            holder["p"] = fw.pool_best_subset(rows, k, top, E=E)
+
+        t, _ = time_steps(step, max(1, K // 2), 1, flush, lambda: None)
+        ms = t / max(1, K // 2)
+        p = holder["p"]
+        bg, tg = p["best_gap"].double(), p["topk_gap"].double()
+        c_hat = torch.where(tg > 0, 1.0 - bg / tg, torch.zeros_like(tg)).cpu().numpy()
+        subsets = sum(math.comb(s + e, min(s, e)) for s, e in POOL_SCHED) * R
+        out[name] = dict(rows=R, n=n, d=d, ms_per_call=ms, rows_per_s=R / (ms * 1e-3), subsets_per_s=subsets / (ms * 1e-3),
+                         c_hat_quartiles={f"s={s}": [float(np.percentile(c_hat[:, j], q)) for q in (25, 50, 75)]
+                                          for j, (s, _) in enumerate(POOL_SCHED)},
+                         rescored_per_item=float(p["n_cand"].double().mean().item()))
+        del rows, top, holder, b
+        torch.cuda.empty_cache()
+    return out
 
 
 # --------------------------------------------------------------------- main
@@ -383,10 +574,13 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--rows-scale", type=float, default=1.0,
                     help="fraction of the headline rows (profiling captures of a smaller case)")
-    ap.add_argument("--only", default="all", choices=["all", "long_rows", "contour"],
+    ap.add_argument("--only", default="all",
+                    choices=["all", "exact_toy", "adversarial", "long_rows", "contour", "mixed", "pool"],
                     help="run one section alone and print its line (profiling captures)")
     ap.add_argument("--long-rows-per-head", type=int, default=512,
                     help="rows per head of the long-row section (profiling captures of a smaller case)")
+    ap.add_argument("--mixed-rows-scale", type=float, default=1.0,
+                    help="fraction of the mixed-profile rows (profiling captures of a smaller case)")
     args = ap.parse_args()
     K, W = args.steps, max(3, args.warmup)
 
@@ -410,14 +604,15 @@ def main():
                 steps.append(cpu_baseline(seed=0, rows_per_group=8))
             v = statistics.median(s["value"] for s in steps)
             sec = sum(s["seconds"] for s in steps) / K
-            line = dict(impl="reference", metric="subsets/s", value=v, unit="subsets/s", n_gpus=args.gpus,
+            line = dict(impl="reference", metric="rows/s", value=v, unit="rows/s", n_gpus=args.gpus,
                         steps=K, warmup=W, ms_per_step=sec * 1e3, higher_is_better=True, scaling="weak",
                         vs_baseline=None, dtype="f64", data="synthetic",
-                        config=dict(workload="exact_enum: 168,192 rows (5 groups, d=64/128), n=24, k=6",
+                        config=dict(workload="exact_enum: 168,192 rows (5 groups, d=64/128), n=24, k=6; "
+                                             "step = gap + swap + exact best subset",
                                     sample="first 8 rows of each group per step"),
-                        cpu_baseline=dict(value=v, unit="subsets/s", cores=steps[0]["cores"], kind="oracle",
+                        cpu_baseline=dict(value=v, unit="rows/s", cores=steps[0]["cores"], kind="oracle",
                                           sample=steps[0]["sample"]),
-                        e2e=dict(value=v, unit="subsets/s", h2d_bytes_per_step=0, d2h_bytes_per_step=0))
+                        e2e=dict(value=v, unit="rows/s", h2d_bytes_per_step=0, d2h_bytes_per_step=0))
             print(json.dumps(line), flush=True)
         if dist:
             dist.destroy_process_group()
@@ -429,13 +624,16 @@ def main():
 
     peaks = read_peaks()
     flush = L2Flush(device)
+    sections_fn = dict(
+        exact_toy=lambda k, w: section_exact_toy(fw, device, k, w, flush, peaks),
+        adversarial=lambda k, w: section_adversarial(fw, device, k, w, flush, peaks),
+        long_rows=lambda k, w: section_long_rows(fw, device, k, w, flush, peaks, rows_per_head=args.long_rows_per_head),
+        contour=lambda k, w: section_contour(fw, device, k, w, flush, peaks),
+        mixed=lambda k, w: section_mixed(fw, device, k, w, flush, peaks, rows_scale=args.mixed_rows_scale),
+        pool=lambda k, w: section_pool(fw, device, k, w, flush, peaks))
     if args.only != "all":
         if rank == 0:
-            if args.only == "long_rows":
-                sec = section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=args.long_rows_per_head)
-            else:
-                sec = section_contour(fw, device, K, W, flush, peaks)
-            print(json.dumps(dict(section=args.only, **sec)), flush=True)
+            print(json.dumps(dict(section=args.only, **{"result": sections_fn[args.only](K, W)})), flush=True)
         if dist:
             dist.destroy_process_group()
         return
@@ -448,62 +646,61 @@ def main():
         total_ms, times = time_steps(lambda: wl.step(time_enum=True), K, W, flush, barrier)
     launches = (fw.launch_count() - l0) // (K + W)
     launches_timed = launches * K
-    enum_ev = wl.enum_times()[-5 * K:]
+    enum_ev = wl.ev.take()[-5 * K:]
     clocks = clk.summary()
-    value, ms = combine_ranks(total_ms / K, wl.subsets, dist, device)
+    value, ms = combine_ranks(total_ms / K, wl.num_rows, dist, device)
+    stats = wl.stats()
 
-    # roofline of the dominant kernel (the exact-search walk, fw_best_subset)
+    # roofline of the dominant call (fw_best_subset: prep, walk, rescore, exhaustive)
     enum_ms = sum(t for t, _ in enum_ev) / K  # per step, all five groups
     enum_launch_ms = sum(t for t, _ in enum_ev) / len(enum_ev)
     sm_mhz = clocks.get("sm_mhz") or peaks["sm_max"]
-    fma_peak = 152 * 128 * 2 * sm_mhz * 1e6 / 1e12  # TFLOP/s, fp32 FMA
-    alg_flops = sum(r.num_rows * SUBSETS_PER_ROW * 4 * b.d for r, b in zip(wl.rows, wl.batches))  # 4d flops per subset
-    alu_ach = alg_flops / (enum_ms * 1e-3) / 1e12
-    lane_frac = wl.subsets * ALU_OPS_PER_SUBSET / (enum_ms * 1e-3) / (152 * 128 * sm_mhz * 1e6)
-    # DRAM traffic of one call from the ncu capture of its prep and walk kernels
-    # (group of 36,864 rows, d = 128: 522.3 + 85.7 MB), scaled to the average
-    # call by its input bytes
-    cap_in = 36864 * (24 * 128 * 4 + 24 * 4)
-    avg_in = sum(r.num_rows * (24 * b.d * 4 + 24 * 4) for r, b in zip(wl.rows, wl.batches)) / len(wl.batches)
-    traffic = (522.3e6 + 85.7e6) * avg_in / cap_in if args.rows_scale == 1.0 else None
+    fma_peak, sms = fp32_peak_tflops(device, sm_mhz)
+    gram = wl.gram_flops()
+    work = gram + stats["inner_ops"]
+    alu_ach = work / (enum_ms * 1e-3) / 1e12
 
     # end to end through the public API with host buffers
     e2e = EnumE2E(wl)
     K2 = max(3, K // 2)
     e2e_total, e2e_times = time_steps(e2e.step, K2, W, flush, barrier)
-    e2e_value, e2e_ms = combine_ranks(e2e_total / K2, wl.subsets, dist, device)
+    e2e_value, e2e_ms = combine_ranks(e2e_total / K2, wl.num_rows, dist, device)
     up_ms = e2e.upload_ms(K2)
 
     sections = {}
     if not args.no_sections and rank == 0:
-        sections["long_rows"] = section_long_rows(fw, device, 5, 3, flush, peaks)
-        sections["contour"] = section_contour(fw, device, 5, 3, flush, peaks)
+        for name in ("exact_toy", "adversarial", "long_rows", "contour", "mixed", "pool"):
+            sections[name] = sections_fn[name](5, 3)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         cpu = cpu_baseline(seed=0)
         cpu.pop("seconds", None)
 
-    line = dict(metric="subsets/s", value=value, unit="subsets/s", n_gpus=world, steps=K, warmup=W,
-                ms_per_step=ms, higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f32",
-                data="synthetic",
+    line = dict(metric="rows/s", value=value, unit="rows/s", n_gpus=world, steps=K, warmup=W,
+                ms_per_step=ms, higher_is_better=True, scaling="weak", vs_baseline=None,
+                dtype="f32 (screening), double-float (every decision and reported gap)", data="synthetic",
                 config=dict(workload="exact_enum: 168,192 rows in 5 groups (d=64,128,128,128,64), n=24, k=6, "
                                      "134,596 subsets/row; step = gap + swap (E=all) + exact best subset",
                             rows_per_gpu=wl.num_rows, subsets_per_step_per_gpu=wl.subsets,
                             l2="inputs larger than L2 (1.6 GB) and a 256 MiB L2 flush between steps",
                             parallelism=f"rows sharded, {world} independent replica(s)"),
-                roofline=dict(bound="alu", achieved=alu_ach, peak=fma_peak, unit="TFLOP/s", frac=alu_ach / fma_peak,
-                              traffic=traffic, kernel="k_enum (fw_best_subset)", launch_ms=enum_launch_ms,
-                              work_basis="4d flops per subset (the direct update of g_A and |g_A|^2); the walk "
-                                         "spends about 3 lane instructions per subset instead, so this rate can "
-                                         "pass the FP32 peak",
-                              lane_issue_frac=lane_frac,
-                              peak_basis=f"152 SMs x 128 fp32 lanes x 2 x {sm_mhz:.0f} MHz (median SM clock under "
-                                         f"load)",
-                              traffic_basis="ncu dram bytes of k_enum_prep + k_enum_walk for one full-size group, "
-                                            "scaled to the average call by input bytes (the rescore and exhaustive "
-                                            "kernels of the call are not included)"),
-                e2e=dict(value=e2e_value, unit="subsets/s",
+                derived=dict(subsets_covered_per_s=wl.subsets * world / (ms * 1e-3),
+                             walk_leaves_per_s=stats["inner_leaves"] * world / (ms * 1e-3),
+                             walk_leaves_per_row=stats["inner_leaves"] / wl.num_rows,
+                             rows_exhaustive=stats["rows_exhaustive"], candidates=stats["candidates"],
+                             note="the search covers every subset; its bounds exclude most of them without a "
+                                  "visit, and walk_leaves counts the subsets its inner enumeration visits"),
+                roofline=roofline("alu", alu_ach, fma_peak, "TFLOP/s", traffic_of("fw_best_subset", wl.num_rows),
+                                  kernel="fw_best_subset (k_enum_prep + k_enum_walk + k_enum_rescore + "
+                                         "k_enum_exhaustive)", launch_ms=enum_launch_ms,
+                                  work_basis="fp32 flops the call is known to execute: the prep kernel's Gram "
+                                             "products (2 d (n+1)(n+2)/2 per row) plus the walk's counted "
+                                             "inner-enumeration operations; per step "
+                                             f"{gram:.3e} + {stats['inner_ops']:.3e}",
+                                  peak_basis=f"{sms} SMs x 128 fp32 lanes x 2 x {sm_mhz:.0f} MHz (median SM clock "
+                                             f"under load)"),
+                e2e=dict(value=e2e_value, unit="rows/s",
                          h2d_bytes_per_step=e2e.h2d, d2h_bytes_per_step=e2e.d2h,
                          step_ms=[round(t, 2) for t in e2e_times],
                          upload_ms=[round(t, 2) for t in up_ms],

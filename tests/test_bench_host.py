@@ -65,7 +65,7 @@ def test_reference_arm_prints_one_contract_line():
     lines = [x for x in r.stdout.splitlines() if x.strip().startswith("{")]
     assert len(lines) == 1
     line = json.loads(lines[0])
-    assert line["impl"] == "reference" and line["metric"] == "subsets/s" and line["unit"] == "subsets/s"
+    assert line["impl"] == "reference" and line["metric"] == "rows/s" and line["unit"] == "rows/s"
     assert line["higher_is_better"] is True and line["value"] > 0 and line["warmup"] >= 3
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
     assert line["cpu_baseline"]["cores"] >= 1
