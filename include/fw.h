@@ -257,6 +257,24 @@ fw_status fw_contour_alloc(const float *scores, int32_t cells, int32_t T, int32_
                            size_t workspace_bytes, void *stream);
 size_t fw_contour_alloc_workspace(int32_t cells, int32_t T);
 
+/* ContourKV with its budget enforced per cell (Sec. 4: enforcement caps
+ * every head at a uniform method's per-head count).  The allocation of
+ * fw_contour_alloc -- same floor, same global ranking and tau -- truncated
+ * per cell: a cell whose allocation exceeds `cap` keeps its recency floor
+ * plus its best cap - min(floor, T) non-floor entries (score desc, position
+ * asc), so counts[h] = min(allocated count, cap) and the total
+ * offsets[cells] = sum_h counts[h] <= total_budget (kept_pos needs room for
+ * total_budget entries; the positions past offsets[cells] are not written).
+ * dropped_alloc is the mass outside the truncated set; tau and
+ * dropped_uniform are those of fw_contour_alloc.  Requires
+ * cap >= min(floor, T) (the floor is always kept); other rules as
+ * fw_contour_alloc. */
+fw_status fw_contour_alloc_capped(const float *scores, int32_t cells, int32_t T, int32_t floor, int64_t total_budget,
+                                  int32_t uniform_s, int32_t cap, int32_t *counts, int64_t *offsets, int32_t *kept_pos,
+                                  float *tau, float *dropped_uniform, float *dropped_alloc, void *workspace,
+                                  size_t workspace_bytes, void *stream);
+size_t fw_contour_alloc_capped_workspace(int32_t cells, int32_t T);
+
 /* Ragged per-head storage (Sec. 4): copy the kept rows of K and V
  * ([cells][T][row_bytes] each) into packed [offsets[cells]][row_bytes] outputs,
  * cell by cell, positions in the order of kept_pos.  row_bytes must be a
@@ -265,6 +283,54 @@ size_t fw_contour_alloc_workspace(int32_t cells, int32_t T);
 fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t T,
                             int32_t row_bytes, const int64_t *offsets, const int32_t *kept_pos,
                             int64_t total, void *K_out, void *V_out, void *stream);
+
+/* The observation-window importance score (Sec. 4 runs ContourKV with
+ * SnapKV's window score as well as with a reconstruction score): the last w
+ * query rows of a cell vote for the keys they attend to.  For cell c, keys
+ * K[c][j] (j < T) and window queries Qw[c][i] (i < w; query i sits at
+ * position T - w + i and sees the keys j <= T - w + i):
+ *   a_ij   = softmax over the visible keys of scale * q_i . k_j,
+ *   vote_j = sum_i a_ij,
+ *   scores[c][j] = max of vote over positions [j - pool/2, j + pool/2]
+ *                  clipped to the prefix [0, T - w), for prefix positions;
+ *                  vote_j itself for the w window positions (which a
+ *                  ContourKV floor of at least w keeps anyway).
+ * The output feeds fw_contour_alloc as its importance score.
+ *   Qw : bf16 [cells][w][d];  K : bf16 [cells][T][d] (the cache's keys);
+ *        both 16-byte aligned.  d in {64, 128}; 1 <= w <= min(32, T);
+ *        pool odd >= 1 (SnapKV: 7); scale > 0 (1 / sqrt(d) for attention).
+ *   scores : fp32 [cells][T]; status [cells] (may be NULL): FW_OK, or
+ *        FW_ERR_TIMEOUT if a bounded wait of the cell's CTA gave up.
+ * Workspace: the votes, cells x T fp32.  The products run on the tensor
+ * cores (bf16 inputs, fp32 accumulation), the key tiles arrive by TMA;
+ * cells x T must stay below 2^31. */
+fw_status fw_window_score(const void *Qw, const void *K, int32_t cells, int32_t T, int32_t d, int32_t w, float scale,
+                          int32_t pool, float *scores, int32_t *status, void *workspace, size_t workspace_bytes,
+                          void *stream);
+size_t fw_window_score_workspace(int32_t cells, int32_t T);
+
+/* Ragged per-head storage with room to grow (Sec. 4's ragged storage for the
+ * multi-turn case of Sec. 1, where one compressed cache serves every later
+ * query while decode keeps appending to it).  Cell h owns rows
+ * [base[h], base[h] + capacity[h]) of K_store and V_store ([rows][row_bytes]
+ * each, device).
+ * fw_ragged_compact_to: as fw_ragged_compact, but cell h's kept rows go to
+ *   its own rows from base[h] on; a cell whose count (offsets[h+1] -
+ *   offsets[h]) exceeds capacity[h] is not copied and gets status[h] =
+ *   FW_ERR_WORKSPACE (status [cells] may be NULL).
+ * fw_ragged_append: appends m new rows per cell (new_K, new_V: [cells][m]
+ *   [row_bytes], device) behind its counts[h] filled rows and adds m to
+ *   counts[h] (device, in/out); a cell without room for all m rows takes none
+ *   and gets status[h] = FW_ERR_WORKSPACE, its count unchanged.  A decode step
+ *   is m = 1; a prefill chunk appends several.  Calls on one stream see each
+ *   other's counts in order.
+ * row_bytes: a positive multiple of 16; all row pointers 16-byte aligned. */
+fw_status fw_ragged_compact_to(const void *K, const void *V, int32_t cells, int32_t T, int32_t row_bytes,
+                               const int64_t *offsets, const int32_t *kept_pos, const int64_t *base,
+                               const int32_t *capacity, void *K_store, void *V_store, int32_t *status, void *stream);
+fw_status fw_ragged_append(void *K_store, void *V_store, const int64_t *base, const int32_t *capacity, int32_t *counts,
+                           const void *new_K, const void *new_V, int32_t cells, int32_t m, int32_t row_bytes,
+                           int32_t *status, void *stream);
 
 /* Largest cells accepted by fw_contour_alloc_noalloc. */
 #define FW_CONTOUR_NOALLOC_MAX_CELLS 4096

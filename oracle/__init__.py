@@ -56,6 +56,11 @@ def lib():
             L.orc_colex_rank.restype = C.c_uint64
             L.orc_contour_alloc.argtypes = [vp, C.c_int, C.c_int, C.c_int, C.c_int64, C.c_int,
                                             vp, vp, vp, vp, vp, vp]
+            L.orc_contour_alloc_capped.argtypes = [vp, C.c_int, C.c_int, C.c_int, C.c_int64, C.c_int, C.c_int,
+                                                   vp, vp, vp, vp, vp, vp]
+            L.orc_ragged_compact_to.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp]
+            L.orc_ragged_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, C.c_int, C.c_int, C.c_int, vp]
+            L.orc_window_score.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, C.c_int, C.c_double, C.c_int, vp, vp]
             L.orc_ragged_compact.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, C.c_int, vp, vp, vp, vp]
             L.orc_group_vote.argtypes = [C.POINTER(_Rows), C.c_int, vp, C.c_int, vp, vp, vp, vp, C.c_int,
                                          vp, vp, vp]
@@ -270,6 +275,21 @@ def contour_alloc(scores, floor, total_budget, uniform_s):
     return out
 
 
+def contour_alloc_capped(scores, floor, total_budget, uniform_s, cap):
+    """f3: the ContourKV allocation truncated to `cap` entries per cell."""
+    s = _host(scores, np.float32)
+    cells, T = s.shape
+    out = dict(counts=np.zeros(cells, np.int32), offsets=np.zeros(cells + 1, np.int64),
+               kept_pos=np.full(int(total_budget), -1, np.int32), tau=np.zeros(1, np.float32),
+               dropped_uniform=np.zeros(cells), dropped_alloc=np.zeros(cells))
+    st = lib().orc_contour_alloc_capped(_p(s), cells, T, int(floor), int(total_budget), int(uniform_s), int(cap),
+                                        _p(out["counts"]), _p(out["offsets"]), _p(out["kept_pos"]),
+                                        _p(out["tau"]), _p(out["dropped_uniform"]), _p(out["dropped_alloc"]))
+    out["status"] = st
+    out["tau"] = float(out["tau"][0])
+    return out
+
+
 def ragged_compact(K, V, offsets, kept_pos):
     K = _host(K)
     V = _host(V)
@@ -283,6 +303,52 @@ def ragged_compact(K, V, offsets, kept_pos):
                                   _p(Ko), _p(Vo))
     assert st == 0, st
     return Ko, Vo
+
+
+def ragged_compact_to(K, V, offsets, kept_pos, base, capacity, K_store, V_store):
+    """f3: kept rows into a store with room per cell; K_store / V_store (numpy,
+    [rows][d]) are updated in place.  Returns the per-cell status."""
+    K, V = _host(K), _host(V)
+    cells, T, d = K.shape
+    off = np.ascontiguousarray(offsets, np.int64)
+    kp = np.ascontiguousarray(kept_pos, np.int32)
+    b = np.ascontiguousarray(base, np.int64)
+    cap = np.ascontiguousarray(capacity, np.int32)
+    status = np.zeros(cells, np.int32)
+    assert K_store.flags.c_contiguous and V_store.flags.c_contiguous
+    st = lib().orc_ragged_compact_to(_p(K), _p(V), cells, T, d * K.dtype.itemsize, _p(off), _p(kp), _p(b), _p(cap),
+                                     _p(K_store), _p(V_store), _p(status))
+    assert st == 0, st
+    return status
+
+
+def ragged_append(K_store, V_store, base, capacity, counts, new_K, new_V):
+    """f3: decode-time append of new_K / new_V ([cells][m][d]); counts (numpy
+    int32) and the stores are updated in place.  Returns the per-cell status."""
+    new_K, new_V = _host(new_K), _host(new_V)
+    cells, m, d = new_K.shape
+    b = np.ascontiguousarray(base, np.int64)
+    cap = np.ascontiguousarray(capacity, np.int32)
+    assert counts.dtype == np.int32 and counts.flags.c_contiguous
+    status = np.zeros(cells, np.int32)
+    st = lib().orc_ragged_append(_p(K_store), _p(V_store), _p(b), _p(cap), _p(counts), _p(new_K), _p(new_V), cells, m,
+                                 d * new_K.dtype.itemsize, _p(status))
+    assert st == 0, st
+    return status
+
+
+def window_score(Qw, K, scale, pool=7):
+    """f3: the observation-window score.  Qw: bf16 bits (uint16) [cells][w][d],
+    K: [cells][T][d].  Returns (scores, votes), fp64 [cells][T]."""
+    Qw = np.ascontiguousarray(_host(Qw)).view(np.uint16)
+    K = np.ascontiguousarray(_host(K)).view(np.uint16)
+    cells, w, d = Qw.shape
+    T = K.shape[1]
+    scores = np.zeros((cells, T))
+    votes = np.zeros((cells, T))
+    st = lib().orc_window_score(_p(Qw), _p(K), cells, T, d, w, float(scale), int(pool), _p(scores), _p(votes))
+    assert st == 0, st
+    return scores, votes
 
 
 def num_threads() -> int:

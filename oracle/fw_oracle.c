@@ -698,6 +698,78 @@ int orc_contour_alloc(const float *scores, int cells, int T, int floor_, int64_t
     return ORC_OK;
 }
 
+/* f3: ContourKV with its budget enforced per cell (Sec. 4: enforcement caps
+ * every head at a uniform method's per-head count).  Step 1 is the plain
+ * allocation above (orc_contour_alloc, which also gives tau and the
+ * uniform-budget dropped mass); step 2 truncates each cell: its floor stays,
+ * and of its kept non-floor positions only the best cap - |F| under
+ * (score desc, position asc) remain.  Outputs as orc_contour_alloc, with
+ * counts[h] = min(allocated count, cap), offsets over those counts and
+ * dropped_alloc the mass outside the truncated set.  kept_pos needs room for
+ * total_budget entries.  Requires cap >= |F|. */
+int orc_contour_alloc_capped(const float *scores, int cells, int T, int floor_, int64_t total_budget,
+                             int uniform_s, int cap, int32_t *counts, int64_t *offsets, int32_t *kept_pos,
+                             float *tau, double *dropped_uniform, double *dropped_alloc)
+{
+    const int F = floor_ < T ? floor_ : T;
+    if (cap < F)
+        return ORC_ERR_ARG;
+    int32_t *c0 = (int32_t *)malloc(sizeof(int32_t) * (size_t)cells);
+    int64_t *o0 = (int64_t *)malloc(sizeof(int64_t) * ((size_t)cells + 1));
+    int32_t *p0 = (int32_t *)malloc(sizeof(int32_t) * (size_t)(total_budget > 0 ? total_budget : 1));
+    int st = orc_contour_alloc(scores, cells, T, floor_, total_budget, uniform_s, c0, o0, p0, tau,
+                               dropped_uniform, NULL);
+    if (st) {
+        free(c0);
+        free(o0);
+        free(p0);
+        return st;
+    }
+    keyed *nf = (keyed *)malloc(sizeof(keyed) * (size_t)T);
+    unsigned char *kept = (unsigned char *)malloc((size_t)T);
+    int64_t acc = 0;
+    for (int h = 0; h < cells; ++h) {
+        const float *s = scores + (int64_t)h * T;
+        memset(kept, 0, (size_t)T);
+        int m = 0;
+        for (int64_t q = o0[h]; q < o0[h + 1]; ++q) {
+            const int j = p0[q];
+            if (j >= T - F) {
+                kept[j] = 1; /* the floor */
+            } else {
+                nf[m].key = (double)s[j];
+                nf[m].idx = j;
+                ++m;
+            }
+        }
+        qsort(nf, (size_t)m, sizeof(keyed), cmp_desc_key_asc_idx);
+        const int keep = m < cap - F ? m : cap - F;
+        for (int t = 0; t < keep; ++t)
+            kept[nf[t].idx] = 1;
+        int cnt = 0;
+        double tot = 0.0, da = 0.0;
+        offsets[h] = acc;
+        for (int j = 0; j < T; ++j) {
+            tot += (double)s[j];
+            if (kept[j])
+                kept_pos[acc + cnt++] = j;
+            else
+                da += (double)s[j];
+        }
+        counts[h] = cnt;
+        acc += cnt;
+        if (dropped_alloc)
+            dropped_alloc[h] = tot > 0 ? da / tot : 0.0;
+    }
+    offsets[cells] = acc;
+    free(kept);
+    free(nf);
+    free(c0);
+    free(o0);
+    free(p0);
+    return ORC_OK;
+}
+
 /* a8: ragged per-head storage (Sec. 4): the kept rows of every cell, copied
  * byte for byte, cells in order, positions ascending.  K, V: [cells][T][d]
  * of elem_bytes each; outputs [offsets[cells]][d]. */
@@ -939,6 +1011,112 @@ int orc_swap_scores(const orc_rows *R, int64_t r, const unsigned char *in_A, con
     free(NA);
     instance_free(&I);
     return na;
+}
+
+/* f3: ragged storage with room per cell (Sec. 4, ragged storage; Sec. 1,
+ * the multi-turn cache that decode keeps appending to).  Cell h owns rows
+ * base[h] .. base[h] + capacity[h] - 1 of the store.
+ * orc_ragged_compact_to: cell h's kept rows (offsets[h] .. offsets[h+1] - 1
+ * of kept_pos) copied byte for byte to its rows from base[h] on, when they
+ * fit (status[h] = 0), else nothing copied and status[h] = 1.
+ * orc_ragged_append: m new rows per cell ([cells][m] rows of row_bytes)
+ * copied behind the counts[h] filled rows, counts[h] += m, when they fit
+ * (status[h] = 0), else nothing and status[h] = 1. */
+int orc_ragged_compact_to(const void *K, const void *V, int cells, int T, int row_bytes, const int64_t *offsets,
+                          const int32_t *kept_pos, const int64_t *base, const int32_t *capacity, void *K_store,
+                          void *V_store, int32_t *status)
+{
+    for (int h = 0; h < cells; ++h) {
+        const int64_t cnt = offsets[h + 1] - offsets[h];
+        status[h] = cnt <= capacity[h] ? 0 : 1;
+        if (status[h])
+            continue;
+        for (int64_t q = 0; q < cnt; ++q) {
+            const int j = kept_pos[offsets[h] + q];
+            if (j < 0 || j >= T)
+                return ORC_ERR_ARG;
+            const size_t src = ((size_t)h * T + (size_t)j) * (size_t)row_bytes;
+            const size_t dst = (size_t)(base[h] + q) * (size_t)row_bytes;
+            memcpy((char *)K_store + dst, (const char *)K + src, (size_t)row_bytes);
+            memcpy((char *)V_store + dst, (const char *)V + src, (size_t)row_bytes);
+        }
+    }
+    return ORC_OK;
+}
+
+int orc_ragged_append(void *K_store, void *V_store, const int64_t *base, const int32_t *capacity, int32_t *counts,
+                      const void *new_K, const void *new_V, int cells, int m, int row_bytes, int32_t *status)
+{
+    for (int h = 0; h < cells; ++h) {
+        status[h] = (counts[h] >= 0 && (int64_t)counts[h] + m <= (int64_t)capacity[h]) ? 0 : 1;
+        if (status[h])
+            continue;
+        for (int t = 0; t < m; ++t) {
+            const size_t src = ((size_t)h * m + (size_t)t) * (size_t)row_bytes;
+            const size_t dst = (size_t)(base[h] + counts[h] + t) * (size_t)row_bytes;
+            memcpy((char *)K_store + dst, (const char *)new_K + src, (size_t)row_bytes);
+            memcpy((char *)V_store + dst, (const char *)new_V + src, (size_t)row_bytes);
+        }
+        counts[h] += m;
+    }
+    return ORC_OK;
+}
+
+/* f3: the observation-window importance score (Sec. 4 runs ContourKV with
+ * SnapKV's window score).  Per cell c: window queries q_i (i < w, bf16 bits,
+ * query i at position T - w + i seeing keys j <= T - w + i) and keys k_j
+ * (bf16 bits); a_ij = softmax over the visible j of scale * q_i . k_j (fp64),
+ * vote_j = sum_i a_ij; scores_j = max of vote over [j - pool/2, j + pool/2]
+ * clipped to the prefix [0, T - w) for prefix positions, vote_j in the
+ * window.  votes may be NULL. */
+static double bf16_at(const uint16_t *p, size_t i)
+{
+    uint32_t bits = ((uint32_t)p[i]) << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return (double)f;
+}
+
+int orc_window_score(const uint16_t *Qw, const uint16_t *K, int cells, int T, int d, int w, double scale, int pool,
+                     double *scores, double *votes)
+{
+    if (cells < 1 || T < 1 || d < 1 || w < 1 || w > T || pool < 1 || pool % 2 == 0)
+        return ORC_ERR_ARG;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int c = 0; c < cells; ++c) {
+        double *vote = (double *)calloc((size_t)T, sizeof(double));
+        double *L = (double *)malloc(sizeof(double) * (size_t)T);
+        for (int i = 0; i < w; ++i) {
+            const int last = T - w + i; /* the query's own position */
+            double M = -INFINITY, Z = 0.0;
+            for (int j = 0; j <= last; ++j) {
+                double dot = 0.0;
+                for (int e = 0; e < d; ++e)
+                    dot += bf16_at(Qw, ((size_t)c * w + i) * d + e) * bf16_at(K, ((size_t)c * T + j) * d + e);
+                L[j] = scale * dot;
+                if (L[j] > M)
+                    M = L[j];
+            }
+            for (int j = 0; j <= last; ++j)
+                Z += exp(L[j] - M);
+            for (int j = 0; j <= last; ++j)
+                vote[j] += exp(L[j] - M) / Z;
+        }
+        const int lim = T - w, h = pool / 2;
+        for (int j = 0; j < T; ++j) {
+            double r = vote[j];
+            if (j < lim)
+                for (int q = j - h; q <= j + h; ++q)
+                    if (q >= 0 && q < lim && vote[q] > r)
+                        r = vote[q];
+            scores[(size_t)c * T + j] = r;
+            if (votes)
+                votes[(size_t)c * T + j] = vote[j];
+        }
+        free(L);
+        free(vote);
+    }
+    return ORC_OK;
 }
 
 /* ---------------------------------------------------------- group vote */

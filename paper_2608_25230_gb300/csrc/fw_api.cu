@@ -256,6 +256,28 @@ fw_status fw_contour_alloc(const float *scores, int32_t cells, int32_t T, int32_
                          dropped_uniform, dropped_alloc, workspace, workspace_bytes, (cudaStream_t)stream);
 }
 
+size_t fw_contour_alloc_capped_workspace(int32_t cells, int32_t T)
+{
+    if (cells < 1 || T < 1) return 0;
+    return contour_capped_workspace(cells, T);
+}
+
+fw_status fw_contour_alloc_capped(const float *scores, int32_t cells, int32_t T, int32_t floor_, int64_t total_budget,
+                                  int32_t uniform_s, int32_t cap, int32_t *counts, int64_t *offsets, int32_t *kept_pos,
+                                  float *tau, float *dropped_uniform, float *dropped_alloc, void *workspace,
+                                  size_t workspace_bytes, void *stream)
+{
+    if (!scores || cells < 1 || T < 1 || floor_ < 0 || uniform_s < 0) return FW_ERR_INVALID_ARG;
+    const int F = floor_ < T ? floor_ : T;
+    if (total_budget < (int64_t)cells * F || total_budget > (int64_t)cells * T) return FW_ERR_INVALID_ARG;
+    if (cap < F) return FW_ERR_INVALID_ARG;
+    if (!counts || !offsets || !kept_pos || !tau) return FW_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < contour_capped_workspace(cells, T))
+        return FW_ERR_WORKSPACE;
+    return contour_alloc(scores, cells, T, floor_, total_budget, uniform_s, counts, offsets, kept_pos, tau,
+                         dropped_uniform, dropped_alloc, workspace, workspace_bytes, (cudaStream_t)stream, cap);
+}
+
 fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t T, int32_t row_bytes,
                             const int64_t *offsets, const int32_t *kept_pos, int64_t total, void *K_out,
                             void *V_out, void *stream)
@@ -267,6 +289,52 @@ fw_status fw_ragged_compact(const void *K, const void *V, int32_t cells, int32_t
         return FW_ERR_INVALID_ARG;
     return ragged_compact(K, V, cells, T, row_bytes, offsets, kept_pos, total, K_out, V_out,
                           (cudaStream_t)stream);
+}
+
+fw_status fw_ragged_compact_to(const void *K, const void *V, int32_t cells, int32_t T, int32_t row_bytes,
+                               const int64_t *offsets, const int32_t *kept_pos, const int64_t *base,
+                               const int32_t *capacity, void *K_store, void *V_store, int32_t *status, void *stream)
+{
+    if (!K || !V || !offsets || !kept_pos || !base || !capacity || !K_store || !V_store || cells < 1 || T < 1)
+        return FW_ERR_INVALID_ARG;
+    if (row_bytes <= 0 || row_bytes % 16 != 0) return FW_ERR_INVALID_ARG;
+    if (!aligned(K, 16) || !aligned(V, 16) || !aligned(K_store, 16) || !aligned(V_store, 16)) return FW_ERR_INVALID_ARG;
+    return ragged_compact_to(K, V, cells, T, row_bytes, offsets, kept_pos, base, capacity, K_store, V_store, status,
+                             (cudaStream_t)stream);
+}
+
+fw_status fw_ragged_append(void *K_store, void *V_store, const int64_t *base, const int32_t *capacity, int32_t *counts,
+                           const void *new_K, const void *new_V, int32_t cells, int32_t m, int32_t row_bytes,
+                           int32_t *status, void *stream)
+{
+    if (!K_store || !V_store || !base || !capacity || !counts || !new_K || !new_V || cells < 1 || m < 1)
+        return FW_ERR_INVALID_ARG;
+    if (row_bytes <= 0 || row_bytes % 16 != 0) return FW_ERR_INVALID_ARG;
+    if ((int64_t)m * (row_bytes / 16) >= ((int64_t)1 << 31)) return FW_ERR_INVALID_ARG;
+    if (!aligned(K_store, 16) || !aligned(V_store, 16) || !aligned(new_K, 16) || !aligned(new_V, 16))
+        return FW_ERR_INVALID_ARG;
+    return ragged_append(K_store, V_store, base, capacity, counts, new_K, new_V, cells, m, row_bytes, status,
+                         (cudaStream_t)stream);
+}
+
+size_t fw_window_score_workspace(int32_t cells, int32_t T)
+{
+    if (cells < 1 || T < 1) return 0;
+    return window_score_workspace(cells, T);
+}
+
+fw_status fw_window_score(const void *Qw, const void *K, int32_t cells, int32_t T, int32_t d, int32_t w, float scale,
+                          int32_t pool, float *scores, int32_t *status, void *workspace, size_t workspace_bytes,
+                          void *stream)
+{
+    if (!Qw || !K || !scores || cells < 1 || T < 1 || w < 1 || w > 32 || w > T) return FW_ERR_INVALID_ARG;
+    if (pool < 1 || pool % 2 == 0 || !(scale > 0.f) || !(scale < 1e30f)) return FW_ERR_INVALID_ARG;
+    if (d != 64 && d != 128) return FW_ERR_UNSUPPORTED;
+    if ((int64_t)cells * T >= ((int64_t)1 << 31) - 256) return FW_ERR_UNSUPPORTED;
+    if (!aligned(Qw, 16) || !aligned(K, 16)) return FW_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < window_score_workspace(cells, T))
+        return FW_ERR_WORKSPACE;
+    return window_score(Qw, K, cells, T, d, w, scale, pool, scores, workspace, status, (cudaStream_t)stream);
 }
 
 }  // extern "C"

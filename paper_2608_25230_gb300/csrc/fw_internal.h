@@ -62,19 +62,32 @@ fw_status group_vote(const RowsDev &R, const int32_t *s, int nb, const fw_gap_ou
 
 // ContourKV allocation and ragged compaction.
 size_t contour_workspace(int cells, int T);
+size_t contour_capped_workspace(int cells, int T);
+// cap < 0: no cap (the plain allocation); otherwise each cell keeps at most cap entries
 fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64_t total_budget,
                         int uniform_s, int32_t *counts, int64_t *offsets, int32_t *kept_pos,
                         float *tau, float *dropped_uniform, float *dropped_alloc, void *ws,
-                        size_t ws_bytes, cudaStream_t s);
+                        size_t ws_bytes, cudaStream_t s, int cap = -1);
 fw_status ragged_compact(const void *K, const void *V, int cells, int T, int row_bytes,
                          const int64_t *offsets, const int32_t *kept_pos, int64_t total,
                          void *K_out, void *V_out, cudaStream_t s);
+fw_status ragged_compact_to(const void *K, const void *V, int cells, int T, int row_bytes, const int64_t *offsets,
+                            const int32_t *kept_pos, const int64_t *base, const int32_t *capacity, void *K_store,
+                            void *V_store, int32_t *status, cudaStream_t s);
+fw_status ragged_append(void *K_store, void *V_store, const int64_t *base, const int32_t *capacity, int32_t *counts,
+                        const void *new_K, const void *new_V, int cells, int m, int row_bytes, int32_t *status,
+                        cudaStream_t s);
 
 // ES_pool (Definition 2.2): exact best subset of the candidate set, any row length.
 size_t pool_best_subset_workspace(const RowsDev &R, int nb);
 fw_status pool_best_subset(const RowsDev &R, const int32_t *k, int nb, const int32_t *E, const fw_gap_out &topk,
                            float *best_gap, int32_t *best_idx, int k_max, float *topk_gap, int64_t *n_cand,
                            int32_t *row_status, void *ws, cudaStream_t st);
+
+// The observation-window importance score (TMA + tcgen05).
+size_t window_score_workspace(int cells, int T);
+fw_status window_score(const void *Qw, const void *K, int cells, int T, int d, int w, float scale, int pool,
+                       float *scores, void *ws, int32_t *status, cudaStream_t s);
 
 // Number of SMs of the current device (queried once per device).
 fw_status device_sms(int *sms);

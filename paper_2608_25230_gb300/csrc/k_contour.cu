@@ -14,6 +14,13 @@
 // the cell's alone, so the cell's block fixes its digit at the end of the pass.  Then per-cell counts, an exclusive
 // prefix sum into ragged offsets, and per-cell ordered compaction of the kept
 // positions.  The compaction copy moves 16-byte vectors, a row per 16 lanes.
+//
+// The capped variant (the enforcement of Sec. 4: no cell keeps more than a
+// cap, e.g. a uniform method's per-head count) truncates each cell to its
+// floor plus its best cap - floor non-floor entries of the allocation; the
+// passes carry a third, per-cell select of the (cap - floor)-th non-floor key,
+// and a non-floor position is kept when both the global threshold and the
+// cell's cap threshold keep it (both are prefixes of the cell's order).
 #include <algorithm>
 
 #include "fw_internal.h"
@@ -47,7 +54,13 @@ struct CArgs {
     int uniform_s;
     uint32_t *uprefix;   // [cells] bits of the cell's uniform-budget threshold fixed so far
     uint32_t *urem;      // [cells] rank still to find inside that prefix (0: no uniform set)
+    int capnf;           // cap - floor on non-floor entries per cell; < 0: no cap
+    uint32_t *cprefix;   // [cells] bits of the cell's cap threshold (non-floor keys) fixed so far
+    uint32_t *crem;      // [cells] rank still to find inside that prefix (0: the cap truncates nothing)
 };
+
+// The cap keeps every non-floor entry (no select needed), none, or a prefix.
+__device__ __forceinline__ bool cap_selects(const CArgs &a) { return a.capnf > 0 && a.capnf < a.T - a.F; }
 
 __global__ void k_c_init(CArgs a)
 {
@@ -61,6 +74,10 @@ __global__ void k_c_init(CArgs a)
     for (int c = threadIdx.x; c < a.cells; c += blockDim.x) {
         a.uprefix[c] = 0u;
         a.urem[c] = su;
+        if (a.cprefix) {
+            a.cprefix[c] = 0u;
+            a.crem[c] = cap_selects(a) ? (uint32_t)a.capnf : 0u;
+        }
     }
 }
 
@@ -116,9 +133,9 @@ __device__ __forceinline__ void select_state(const uint32_t *hist4, int npass, u
 constexpr int CPT = 512;  // threads of a pass block
 __global__ void __launch_bounds__(CPT) k_c_pass(CArgs a, int pass)
 {
-    __shared__ uint32_t hg[256], hu[256];
+    __shared__ uint32_t hg[256], hu[256], hc[256];
     __shared__ uint32_t s_prefix;
-    for (int i = threadIdx.x; i < 256; i += CPT) hg[i] = hu[i] = 0u;
+    for (int i = threadIdx.x; i < 256; i += CPT) hg[i] = hu[i] = hc[i] = 0u;
     const bool glob = a.K > 0;
     if (threadIdx.x < 32) {  // the global state after the earlier passes
         uint32_t pf = 0u, rm = 0u;
@@ -132,6 +149,8 @@ __global__ void __launch_bounds__(CPT) k_c_pass(CArgs a, int pass)
     const uint32_t prefix = s_prefix;
     const uint32_t upre = a.uprefix[c];
     const bool uni = a.urem[c] > 0u;
+    const bool cap = a.cprefix && cap_selects(a);
+    const uint32_t cpre = cap ? a.cprefix[c] : 0u;
     const int nf = a.T - a.F;
     const float *sc = a.scores + (int64_t)c * a.T;
     auto visit = [&](int j, float x) {
@@ -139,6 +158,7 @@ __global__ void __launch_bounds__(CPT) k_c_pass(CArgs a, int pass)
         const uint32_t dg = (key >> shift) & 255u;
         if (glob && j < nf && (key & pmask) == prefix) atomicAdd(&hg[dg], 1u);
         if (uni && (key & pmask) == upre) atomicAdd(&hu[dg], 1u);
+        if (cap && j < nf && (key & pmask) == cpre) atomicAdd(&hc[dg], 1u);
     };
     if ((a.T & 3) == 0 && (reinterpret_cast<uintptr_t>(sc) & 15) == 0) {
         for (int q = threadIdx.x; q < a.T / 4; q += CPT) {
@@ -162,6 +182,18 @@ __global__ void __launch_bounds__(CPT) k_c_pass(CArgs a, int pass)
             if (cum + cc >= rem) {
                 a.uprefix[c] = upre | ((uint32_t)v << shift);
                 a.urem[c] = rem - cum;
+                break;
+            }
+            cum += cc;
+        }
+    }
+    if (cap && threadIdx.x == 32) {
+        uint32_t cum = 0, rem = a.crem[c];
+        for (int v = 255; v >= 0; --v) {
+            const uint32_t cc = hc[v];
+            if (cum + cc >= rem) {
+                a.cprefix[c] = cpre | ((uint32_t)v << shift);
+                a.crem[c] = rem - cum;
                 break;
             }
             cum += cc;
@@ -253,7 +285,9 @@ __global__ void __launch_bounds__(1024) k_c_offsets(CArgs a)
         t = t < 0 ? 0 : (t > a.eq[c] ? a.eq[c] : t);
         a.take[c] = (int32_t)t;
         ebefore += a.eq[c];
-        const int cnt = a.F + (a.K > 0 ? a.gt[c] : 0) + (int)t;
+        int nonf = (a.K > 0 ? a.gt[c] : 0) + (int)t;
+        if (a.capnf >= 0) nonf = min(nonf, a.capnf);
+        const int cnt = a.F + nonf;
         a.counts[c] = cnt;
         sc += cnt;
     }
@@ -302,7 +336,7 @@ constexpr int CTE = 1024;  // threads of an emit block
 __global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
 {
     constexpr int NW = CTE / 32;
-    __shared__ int wc[NW], wt[NW], wu[NW];
+    __shared__ int wc[NW], wt[NW], wu[NW], wk[NW];
     __shared__ double red[NW], red2[NW], red3[NW];
     const int c = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
@@ -311,6 +345,11 @@ __global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
     const int64_t base = a.offsets[c];
     const uint32_t uT = a.uprefix[c];
     const int uwant = (int)a.urem[c];  // 0: no uniform set (every key dropped)
+    // the cap: none (every non-floor entry passes it), zero entries, or its threshold
+    const int cmode = a.capnf < 0 || a.capnf >= a.T - a.F ? 0 : (a.capnf == 0 ? 1 : 2);
+    const uint32_t cT = cmode == 2 ? a.cprefix[c] : 0u;
+    const int cwant = cmode == 2 ? (int)a.crem[c] : 0;
+    int cties_seen = 0;
     const float *s = a.scores + (int64_t)c * a.T;
     const uint32_t lmask = (1u << lane) - 1u;
     int written = 0, ties_seen = 0, uties_seen = 0;
@@ -320,16 +359,24 @@ __global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
     float xn = tid < a.T ? __ldg(s + tid) : 0.f;  // the next chunk's score, loaded a chunk ahead
     for (int j0 = 0; j0 < a.T; j0 += CTE) {
         const int j = j0 + tid;
-        bool kept = false, tie = false, ukept = false, utie = false;
+        bool kept = false, tie = false, ukept = false, utie = false, ckept = true, ctie = false;
         const float x = xn;
         if (j + CTE < a.T) xn = __ldg(s + j + CTE);
         if (j < a.T) {
             const uint32_t key = order_key(x);
             if (j >= a.T - a.F) {
                 kept = true;
-            } else if (a.K > 0) {
-                kept = key > tk;
-                tie = key == tk;
+            } else {
+                if (a.K > 0) {
+                    kept = key > tk;
+                    tie = key == tk;
+                }
+                if (cmode == 1) {
+                    ckept = false;
+                } else if (cmode == 2) {
+                    ckept = key > cT;
+                    ctie = key == cT;
+                }
             }
             if (uwant > 0) {
                 ukept = key > uT;
@@ -338,18 +385,24 @@ __global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
         }
         // ranks of the ties among the cell's ties, in position order
         const uint32_t tb = __ballot_sync(FW_FULL, tie), ub = __ballot_sync(FW_FULL, utie);
+        const uint32_t cb2 = __ballot_sync(FW_FULL, ctie);
         if (lane == 0) {
             wt[wid] = __popc(tb);
             wu[wid] = __popc(ub);
+            wk[wid] = __popc(cb2);
         }
         __syncthreads();
-        int tbefore, ttotal, ubefore, utotal;
+        int tbefore, ttotal, ubefore, utotal, cbefore, ctotal;
         warp_counts<NW>(wt, wid, lane, tbefore, ttotal);
         warp_counts<NW>(wu, wid, lane, ubefore, utotal);
+        warp_counts<NW>(wk, wid, lane, cbefore, ctotal);
         if (tie) kept = ties_seen + tbefore + __popc(tb & lmask) < take;
         if (utie) ukept = uties_seen + ubefore + __popc(ub & lmask) < uwant;
+        if (ctie) ckept = cties_seen + cbefore + __popc(cb2 & lmask) < cwant;
+        kept = kept && ckept;
         ties_seen += ttotal;
         uties_seen += utotal;
+        cties_seen += ctotal;
         const uint32_t kb = __ballot_sync(FW_FULL, kept);
         if (lane == 0) wc[wid] = __popc(kb);
         __syncthreads();
@@ -362,7 +415,7 @@ __global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
             if (!kept) drop += x;
             if (!ukept) udrop += x;
         }
-        __syncthreads();  // wt, wu, wc are rewritten by the next chunk
+        __syncthreads();  // wt, wu, wk, wc are rewritten by the next chunk
     }
     const double tsum = warp_sum_d((double)tot), dsum = warp_sum_d((double)drop), usum = warp_sum_d((double)udrop);
     if (lane == 0) {
@@ -383,14 +436,25 @@ __global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
     }
 }
 
-// ragged compaction: block (cell, chunk) copies rows [offsets[c] + chunk*RPB, ...)
+// ragged compaction: block (cell, chunk) copies rows [offsets[c] + chunk*RPB, ...).
+// With dst_base, cell c's rows go to rows dst_base[c] + (q - offsets[c]) of the
+// output instead (a store with room per cell), provided they fit its capacity.
 constexpr int RPB = 256;  // rows per block
 __global__ void __launch_bounds__(256) k_compact(const uint4 *K, const uint4 *V, int T, int vec_per_row,
                                                  const int64_t *offsets, const int32_t *kept_pos, uint4 *Ko,
-                                                 uint4 *Vo, int chunks)
+                                                 uint4 *Vo, int chunks, const int64_t *dst_base,
+                                                 const int32_t *capacity, int32_t *status)
 {
     const int c = blockIdx.x / chunks;
     const int chunk = blockIdx.x - c * chunks;
+    const int64_t cnt = offsets[c + 1] - offsets[c];
+    int64_t shift = 0;
+    if (dst_base) {
+        const bool fits = cnt <= capacity[c];
+        if (chunk == 0 && threadIdx.x == 0 && status) status[c] = fits ? FW_OK : FW_ERR_WORKSPACE;
+        if (!fits) return;
+        shift = dst_base[c] - offsets[c];
+    }
     const int64_t beg = offsets[c] + (int64_t)chunk * RPB;
     const int64_t end = min(offsets[c + 1], beg + RPB);
     if (beg >= end) return;
@@ -399,9 +463,37 @@ __global__ void __launch_bounds__(256) k_compact(const uint4 *K, const uint4 *V,
         const int64_t q = beg + e / vec_per_row;
         const int part = (int)(e % vec_per_row);
         const int64_t src = ((int64_t)c * T + kept_pos[q]) * vec_per_row + part;
-        const int64_t dst = q * vec_per_row + part;
+        const int64_t dst = (q + shift) * vec_per_row + part;
         Ko[dst] = __ldg(K + src);
         Vo[dst] = __ldg(V + src);
+    }
+}
+
+// decode-time append: block c copies cell c's m new rows behind its filled
+// rows when they fit, then advances its count
+__global__ void __launch_bounds__(256) k_append(uint4 *Ks, uint4 *Vs, const int64_t *base, const int32_t *capacity,
+                                                int32_t *counts, const uint4 *nK, const uint4 *nV, int m,
+                                                int vec_per_row, int32_t *status)
+{
+    __shared__ int s_cnt;
+    const int c = blockIdx.x;
+    if (threadIdx.x == 0) s_cnt = counts[c];
+    __syncthreads();
+    const int cnt = s_cnt;
+    const bool fits = cnt >= 0 && (int64_t)cnt + m <= (int64_t)capacity[c];
+    if (fits) {
+        const int64_t dst0 = (base[c] + cnt) * vec_per_row;
+        const int64_t src0 = (int64_t)c * m * vec_per_row;
+        const int nvec = m * vec_per_row;
+        for (int e = threadIdx.x; e < nvec; e += blockDim.x) {
+            Ks[dst0 + e] = __ldg(nK + src0 + e);
+            Vs[dst0 + e] = __ldg(nV + src0 + e);
+        }
+    }
+    __syncthreads();  // every thread has read the old count
+    if (threadIdx.x == 0) {
+        if (fits) counts[c] = cnt + m;
+        if (status) status[c] = fits ? FW_OK : FW_ERR_WORKSPACE;
     }
 }
 
@@ -413,9 +505,13 @@ size_t contour_workspace(int cells, int T)
     return align256(4 * 256 * 4) + align256(sizeof(CState)) + 5 * align256((size_t)cells * 4);
 }
 
+size_t contour_capped_workspace(int cells, int T) { return contour_workspace(cells, T) + 2 * align256((size_t)cells * 4); }
+
+static bool cap_selects_host(const CArgs &a) { return a.cprefix && a.capnf > 0 && a.capnf < a.T - a.F; }
+
 fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64_t total_budget, int uniform_s,
                         int32_t *counts, int64_t *offsets, int32_t *kept_pos, float *tau, float *dropped_uniform,
-                        float *dropped_alloc, void *ws, size_t ws_bytes, cudaStream_t s)
+                        float *dropped_alloc, void *ws, size_t ws_bytes, cudaStream_t s, int cap)
 {
     (void)ws_bytes;
     CArgs a;
@@ -439,6 +535,15 @@ fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64
     a.uprefix = (uint32_t *)w;
     w += align256((size_t)cells * 4);
     a.urem = (uint32_t *)w;
+    a.capnf = -1;
+    a.cprefix = a.crem = nullptr;
+    if (cap >= 0) {  // the capped variant: two more per-cell arrays after the uncapped layout
+        w += align256((size_t)cells * 4);
+        a.cprefix = (uint32_t *)w;
+        w += align256((size_t)cells * 4);
+        a.crem = (uint32_t *)w;
+        a.capnf = cap - a.F;
+    }
     a.counts = counts;
     a.offsets = offsets;
     a.kept_pos = kept_pos;
@@ -447,7 +552,7 @@ fw_status contour_alloc(const float *scores, int cells, int T, int floor_, int64
     a.dropped_alloc = dropped_alloc;
     a.uniform_s = uniform_s;
     FW_LAUNCH(k_c_init, 1, 1024, 0, s, a);
-    if (a.K > 0 || (dropped_uniform && uniform_s > 0)) {
+    if (a.K > 0 || (dropped_uniform && uniform_s > 0) || cap_selects_host(a)) {
         for (int pass = 0; pass < 4; ++pass) FW_LAUNCH(k_c_pass, (unsigned)cells, CPT, 0, s, a, pass);
     }
     FW_LAUNCH(k_c_count, (unsigned)cells, CT, 0, s, a);
@@ -465,7 +570,30 @@ fw_status ragged_compact(const void *K, const void *V, int cells, int T, int row
     const int64_t grid = (int64_t)cells * chunks;
     if (grid >= ((int64_t)1 << 31)) return FW_ERR_UNSUPPORTED;
     FW_LAUNCH(k_compact, (unsigned)grid, 256, 0, s, (const uint4 *)K, (const uint4 *)V, T, vec, offsets, kept_pos,
-              (uint4 *)K_out, (uint4 *)V_out, chunks);
+              (uint4 *)K_out, (uint4 *)V_out, chunks, (const int64_t *)nullptr, (const int32_t *)nullptr,
+              (int32_t *)nullptr);
+    return FW_OK;
+}
+
+fw_status ragged_compact_to(const void *K, const void *V, int cells, int T, int row_bytes, const int64_t *offsets,
+                            const int32_t *kept_pos, const int64_t *base, const int32_t *capacity, void *K_store,
+                            void *V_store, int32_t *status, cudaStream_t s)
+{
+    const int vec = row_bytes / 16;
+    const int chunks = (T + RPB - 1) / RPB;
+    const int64_t grid = (int64_t)cells * chunks;
+    if (grid >= ((int64_t)1 << 31)) return FW_ERR_UNSUPPORTED;
+    FW_LAUNCH(k_compact, (unsigned)grid, 256, 0, s, (const uint4 *)K, (const uint4 *)V, T, vec, offsets, kept_pos,
+              (uint4 *)K_store, (uint4 *)V_store, chunks, base, capacity, status);
+    return FW_OK;
+}
+
+fw_status ragged_append(void *K_store, void *V_store, const int64_t *base, const int32_t *capacity, int32_t *counts,
+                        const void *new_K, const void *new_V, int cells, int m, int row_bytes, int32_t *status,
+                        cudaStream_t s)
+{
+    FW_LAUNCH(k_append, (unsigned)cells, 256, 0, s, (uint4 *)K_store, (uint4 *)V_store, base, capacity, counts,
+              (const uint4 *)new_K, (const uint4 *)new_V, m, row_bytes / 16, status);
     return FW_OK;
 }
 

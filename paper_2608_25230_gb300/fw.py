@@ -8,6 +8,7 @@ is no fallback path.
 from __future__ import annotations
 
 import ctypes as C
+import math
 import os
 
 import torch
@@ -64,6 +65,20 @@ _lib.fw_contour_alloc.argtypes = [vp, C.c_int32, C.c_int32, C.c_int32, C.c_int64
                                   vp, vp, C.c_size_t, vp]
 _lib.fw_contour_alloc_workspace.argtypes = [C.c_int32, C.c_int32]
 _lib.fw_contour_alloc_workspace.restype = C.c_size_t
+_lib.fw_contour_alloc_capped.argtypes = [vp, C.c_int32, C.c_int32, C.c_int32, C.c_int64, C.c_int32, C.c_int32, vp, vp,
+                                         vp, vp, vp, vp, vp, C.c_size_t, vp]
+_lib.fw_contour_alloc_capped.restype = C.c_int
+_lib.fw_contour_alloc_capped_workspace.argtypes = [C.c_int32, C.c_int32]
+_lib.fw_contour_alloc_capped_workspace.restype = C.c_size_t
+_lib.fw_ragged_compact_to.argtypes = [vp, vp, C.c_int32, C.c_int32, C.c_int32, vp, vp, vp, vp, vp, vp, vp, vp]
+_lib.fw_ragged_compact_to.restype = C.c_int
+_lib.fw_ragged_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, C.c_int32, C.c_int32, C.c_int32, vp, vp]
+_lib.fw_ragged_append.restype = C.c_int
+_lib.fw_window_score.argtypes = [vp, vp, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_float, C.c_int32, vp, vp,
+                                 vp, C.c_size_t, vp]
+_lib.fw_window_score.restype = C.c_int
+_lib.fw_window_score_workspace.argtypes = [C.c_int32, C.c_int32]
+_lib.fw_window_score_workspace.restype = C.c_size_t
 _lib.fw_ragged_compact.argtypes = [vp, vp, C.c_int32, C.c_int32, C.c_int32, vp, vp, C.c_int64, vp, vp, vp]
 _lib.fw_group_vote.argtypes = [C.POINTER(FwRows), vp, C.c_int32, C.POINTER(FwGapOut), vp, vp, vp, C.c_int32, vp,
                                vp, C.c_size_t, vp]
@@ -321,6 +336,28 @@ def contour_alloc(scores: torch.Tensor, *, floor: int, total_budget: int, unifor
     return out
 
 
+def contour_alloc_capped(scores: torch.Tensor, *, floor: int, total_budget: int, uniform_s: int, cap: int,
+                         stream=None):
+    """fw_contour_alloc_capped: the allocation truncated to `cap` entries per
+    cell.  kept_pos holds total_budget entries; offsets[-1] of them are valid."""
+    dev = scores.device
+    cells, T = scores.shape
+    out = dict(counts=torch.empty(cells, dtype=torch.int32, device=dev),
+               offsets=torch.empty(cells + 1, dtype=torch.int64, device=dev),
+               kept_pos=torch.empty(int(total_budget), dtype=torch.int32, device=dev),
+               tau=torch.empty(1, dtype=torch.float32, device=dev),
+               dropped_uniform=torch.empty(cells, dtype=torch.float32, device=dev),
+               dropped_alloc=torch.empty(cells, dtype=torch.float32, device=dev))
+    ws = _ws(_lib.fw_contour_alloc_capped_workspace(cells, T), dev)
+    st = _lib.fw_contour_alloc_capped(_ptr(scores), cells, T, int(floor), int(total_budget), int(uniform_s), int(cap),
+                                      _ptr(out["counts"]), _ptr(out["offsets"]), _ptr(out["kept_pos"]),
+                                      _ptr(out["tau"]), _ptr(out["dropped_uniform"]), _ptr(out["dropped_alloc"]),
+                                      _ptr(ws), ws.numel(), _stream(stream))
+    _check(st, "fw_contour_alloc_capped")
+    out["_ws"] = ws
+    return out
+
+
 def ragged_compact(K: torch.Tensor, V: torch.Tensor, offsets: torch.Tensor, kept_pos: torch.Tensor, total: int,
                    *, out=None, stream=None):
     cells, T, d = K.shape
@@ -334,6 +371,42 @@ def ragged_compact(K: torch.Tensor, V: torch.Tensor, offsets: torch.Tensor, kept
                                 _ptr(Ko), _ptr(Vo), _stream(stream))
     _check(st, "fw_ragged_compact")
     return Ko, Vo
+
+
+def ragged_compact_to(K: torch.Tensor, V: torch.Tensor, offsets: torch.Tensor, kept_pos: torch.Tensor,
+                      base: torch.Tensor, capacity: torch.Tensor, K_store: torch.Tensor, V_store: torch.Tensor,
+                      status: torch.Tensor = None, stream=None):
+    """fw_ragged_compact_to: kept rows into a store with room per cell."""
+    cells, T, d = K.shape
+    st = _lib.fw_ragged_compact_to(_ptr(K), _ptr(V), cells, T, d * K.element_size(), _ptr(offsets), _ptr(kept_pos),
+                                   _ptr(base), _ptr(capacity), _ptr(K_store), _ptr(V_store), _ptr(status),
+                                   _stream(stream))
+    _check(st, "fw_ragged_compact_to")
+
+
+def ragged_append(K_store: torch.Tensor, V_store: torch.Tensor, base: torch.Tensor, capacity: torch.Tensor,
+                  counts: torch.Tensor, new_K: torch.Tensor, new_V: torch.Tensor, status: torch.Tensor = None,
+                  stream=None):
+    """fw_ragged_append: new_K / new_V [cells][m][d] behind each cell's rows."""
+    cells, m, d = new_K.shape
+    st = _lib.fw_ragged_append(_ptr(K_store), _ptr(V_store), _ptr(base), _ptr(capacity), _ptr(counts), _ptr(new_K),
+                               _ptr(new_V), cells, m, d * new_K.element_size(), _ptr(status), _stream(stream))
+    _check(st, "fw_ragged_append")
+
+
+def window_score(Qw: torch.Tensor, K: torch.Tensor, *, scale: float = None, pool: int = 7, out=None, stream=None):
+    """fw_window_score.  Qw: bf16 (or int16 bits) [cells][w][d]; K: [cells][T][d].
+    Returns (scores [cells][T] fp32, status [cells])."""
+    cells, w, d = Qw.shape
+    T = K.shape[1]
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    scores = out if out is not None else torch.empty(cells, T, dtype=torch.float32, device=K.device)
+    status = torch.empty(cells, dtype=torch.int32, device=K.device)
+    ws = _ws(_lib.fw_window_score_workspace(cells, T), K.device)
+    st = _lib.fw_window_score(_ptr(Qw), _ptr(K), cells, T, d, w, C.c_float(scale), int(pool), _ptr(scores),
+                              _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
+    _check(st, "fw_window_score")
+    return scores, status
 
 
 def raw():

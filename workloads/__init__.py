@@ -365,6 +365,15 @@ def contour_cache(seed: int = 0, cells: int = 256, T: int = 32768, d: int = 128,
                       total_budget=total, uniform_s=total // cells)
 
 
+# Window queries for the observation-window score: the last w query rows of
+# every cell of a contour_cache, bf16 ~ N(0, 1) like its keys (w = 32, the
+# largest SnapKV window of App. D).
+def window_queries(seed: int = 0, cells: int = 256, w: int = 32, d: int = 128, backend: str = "numpy",
+                   device: str = "cuda"):
+    rng = make_rng(seed * 1000 + 5, backend, device)
+    return rng.to_bf16(rng.normal((cells, w, d)))
+
+
 # Mixed-profile sweep: 168,192 rows from five head profiles (rows, d, n),
 # GQA groups of 4 rows sharing a bf16 V block, logits tau*N(0,1) + sink +8 +
 # recency bump, tau ~ U[0.3, 4] per row, budget per group
