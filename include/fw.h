@@ -238,6 +238,45 @@ fw_status fw_pool_best_subset(const fw_rows *rows, const int32_t *k, int32_t nb,
 /* Workspace bytes: the pool of every (row, budget), 64 int32 each, and its size. */
 size_t fw_pool_best_subset_workspace(const fw_rows *rows, int32_t nb);
 
+/* The deployed selectors audited in Sec. 2.4 (App. D settings), as kept sets
+ * scored with Definition 2.1's es.  For budget s:
+ *   FW_SEL_STREAMING  the first min(4, s/2) positions and the last
+ *                     s - min(4, s/2) (StreamingLLM: sinks plus recency);
+ *   FW_SEL_H2O        the last s/2 positions and, of the others, the s - s/2
+ *                     of largest mass accumulated over the group's rows (the
+ *                     query rows sharing the KV head, i.e. one cache serving
+ *                     them all);
+ *   FW_SEL_SNAPKV     window w = max(1, min(32, s/2)): the last w positions and,
+ *                     of the others, the s - w of largest pooled vote (a key's
+ *                     mass summed over the group's last w rows, then the
+ *                     maximum over the 7 positions around it, clipped to the
+ *                     candidates);
+ *   FW_SEL_QUEST      pages of P = max(2, s/4) keys, the floor(s/P) pages of
+ *                     largest maximum logit (Quest's page bound, taken exact
+ *                     since the logits are given);
+ *   FW_SEL_QUEST16    the same with P = 16 (s >= 16; NaN below).
+ * Equal scores keep lower positions (pages) first. */
+typedef enum {
+    FW_SEL_STREAMING = 0,
+    FW_SEL_H2O = 1,
+    FW_SEL_SNAPKV = 2,
+    FW_SEL_QUEST = 3,
+    FW_SEL_QUEST16 = 4
+} fw_selector;
+#define FW_NUM_SELECTORS 5
+
+/* For every row, rule and budget: es [rows][FW_NUM_SELECTORS][nb] (NaN where
+ * the rule keeps nothing: s > n, or Quest-16 with s < 16); bits (may be NULL)
+ * [rows][FW_NUM_SELECTORS][nb][words] the kept sets, words = ceil(max_n/32)
+ * exactly.  s: HOST [nb] budgets, 1 <= s <= 4096, nb 1..4.  topk: a fw_gap_out
+ * filled by fw_dense_and_topk_gap for the same rows (o, row_max, row_sum used).
+ * Rows up to 65,536 keys (FW_ERR_UNSUPPORTED above). */
+fw_status fw_selector_audit(const fw_rows *rows, const int32_t *s, int32_t nb, const fw_gap_out *topk, float *es,
+                            uint32_t *bits, int32_t words, void *workspace, size_t workspace_bytes, void *stream);
+/* Workspace bytes: the accumulated masses (groups x max_n fp32), the window
+ * votes (groups x nb x max_n fp32) and the group-level sets. */
+size_t fw_selector_audit_workspace(const fw_rows *rows, int32_t nb);
+
 /* ContourKV allocation (Sec. 4).  scores: device [cells][T] fp32, finite and
  * >= 0.  Every cell keeps its recency floor (the last min(floor, T) positions)
  * plus the non-floor positions among the K = total_budget - cells*min(floor,T)

@@ -61,6 +61,7 @@ def lib():
             L.orc_ragged_compact_to.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp]
             L.orc_ragged_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, C.c_int, C.c_int, C.c_int, vp]
             L.orc_window_score.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, C.c_int, C.c_double, C.c_int, vp, vp]
+            L.orc_selector_audit.argtypes = [C.POINTER(_Rows), C.c_int, vp, C.c_int, vp, vp, C.c_int, vp, vp]
             L.orc_ragged_compact.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, C.c_int, vp, vp, vp, vp]
             L.orc_group_vote.argtypes = [C.POINTER(_Rows), C.c_int, vp, C.c_int, vp, vp, vp, vp, C.c_int,
                                          vp, vp, vp]
@@ -349,6 +350,26 @@ def window_score(Qw, K, scale, pool=7):
     st = lib().orc_window_score(_p(Qw), _p(K), cells, T, d, w, float(scale), int(pool), _p(scores), _p(votes))
     assert st == 0, st
     return scores, votes
+
+
+SELECTORS = ("streamingllm", "h2o", "snapkv", "quest", "quest16")
+
+
+def selector_audit(batch, s):
+    """f4: the deployed selectors' kept sets and their es (App. D settings).
+    s: budgets (nb).  Returns es [rows][5][nb], bits [rows][5][nb][words],
+    G [groups][max_n], pooled [groups][nb][max_n]."""
+    H = batch if isinstance(batch, HostRows) else HostRows(batch)
+    s = np.ascontiguousarray(np.atleast_1d(s), np.int32)
+    nb = len(s)
+    words = (H.max_n + 31) // 32
+    G = len(H.n)
+    out = dict(es=np.zeros((H.num_rows, 5, nb)), bits=np.zeros((H.num_rows, 5, nb, words), np.uint32),
+               G=np.zeros((G, H.max_n)), pooled=np.zeros((G, nb, H.max_n)))
+    st = lib().orc_selector_audit(C.byref(H.c), nb, _p(s), H.max_n, _p(out["es"]), _p(out["bits"]), words,
+                                  _p(out["G"]), _p(out["pooled"]))
+    assert st == 0, st
+    return out
 
 
 def num_threads() -> int:

@@ -1119,6 +1119,173 @@ int orc_window_score(const uint16_t *Qw, const uint16_t *K, int cells, int T, in
     return ORC_OK;
 }
 
+/* f4: the deployed selectors audited in Sec. 2.4 with App. D's settings, each
+ * a kept set scored with es (Definition 2.1).  For budget s:
+ *   StreamingLLM: positions j < min(4, s/2) and j >= n - (s - min(4, s/2));
+ *   H2O: positions j >= n - s/2, and of j < n - s/2 the s - s/2 of largest
+ *        accumulated mass G_j = sum over the group's rows of p_ij;
+ *   SnapKV: w = max(1, min(32, s/2)); positions j >= n - w, and of j < n - w
+ *        the s - w of largest pooled vote max_{|q - j| <= 3, q < n - w} vote_q,
+ *        vote_q = sum over the group's last min(w, R) rows of p_iq;
+ *   Quest (P = max(2, s/4)) and Quest-16 (P = 16, s >= 16): the floor(s/P)
+ *        pages of P consecutive keys with the largest maximum logit.
+ * Equal scores: lower position (page) first.  es NaN when the set is empty.
+ * Outputs: es [rows][5][nb]; bits [rows][5][nb][words] (may be NULL); G
+ * [groups][max_n] and pooled [groups][nb][max_n] (may be NULL; pooled is the
+ * vote itself at the window positions). */
+/* mark the first `take` entries of a sorted candidate list */
+static void mark_first(const keyed *a, int m, int take, unsigned char *in)
+{
+    for (int t = 0; t < take && t < m; ++t)
+        in[a[t].idx] = 1;
+}
+
+int orc_selector_audit(const orc_rows *R, int nb, const int32_t *s, int max_n, double *es, uint32_t *bits, int words,
+                       double *G_out, double *pooled_out)
+{
+    const int64_t groups = R->num_groups;
+    const int Rg = R->rows_per_group;
+    int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : bad)
+    for (int64_t g = 0; g < groups; ++g) {
+        const int n = R->n[g];
+        double *G = (double *)calloc((size_t)n + 1, sizeof(double));
+        double *vote = (double *)calloc((size_t)nb * n + 1, sizeof(double));
+        double *pooled = (double *)calloc((size_t)nb * n + 1, sizeof(double));
+        unsigned char *hset = (unsigned char *)calloc((size_t)nb * n + 1, 1);
+        unsigned char *sset = (unsigned char *)calloc((size_t)nb * n + 1, 1);
+        unsigned char *in = (unsigned char *)calloc((size_t)n + 1, 1);
+        keyed *o = (keyed *)malloc(sizeof(keyed) * ((size_t)n + 1));
+        /* accumulated masses and window votes over the group's rows */
+        for (int i = 0; i < Rg; ++i) {
+            instance I;
+            if (load_row(R, g * Rg + i, &I)) {
+                instance_free(&I);
+                bad |= 1;
+                continue;
+            }
+            for (int j = 0; j < n; ++j) {
+                G[j] += I.p[j];
+                for (int b = 0; b < nb; ++b) {
+                    int w = s[b] / 2 < 32 ? s[b] / 2 : 32;
+                    w = w < 1 ? 1 : w;
+                    if (i >= Rg - w)
+                        vote[(size_t)b * n + j] += I.p[j];
+                }
+            }
+            instance_free(&I);
+        }
+        /* the group-level sets */
+        for (int b = 0; b < nb; ++b) {
+            const int sb = s[b];
+            if (sb < 1 || sb > n)
+                continue;
+            const int r = sb / 2;
+            for (int j = 0; j < n - r; ++j) {
+                o[j].key = G[j];
+                o[j].idx = j;
+            }
+            qsort(o, (size_t)(n - r), sizeof(keyed), cmp_desc_key_asc_idx);
+            mark_first(o, n - r, sb - r, hset + (size_t)b * n);
+            for (int j = n - r; j < n; ++j)
+                hset[(size_t)b * n + j] = 1;
+            int w = sb / 2 < 32 ? sb / 2 : 32;
+            w = w < 1 ? 1 : w;
+            const int lim = n - w;
+            for (int j = 0; j < n; ++j) {
+                double v = vote[(size_t)b * n + j];
+                if (j < lim)
+                    for (int q = j - 3; q <= j + 3; ++q)
+                        if (q >= 0 && q < lim && vote[(size_t)b * n + q] > v)
+                            v = vote[(size_t)b * n + q];
+                pooled[(size_t)b * n + j] = v;
+            }
+            for (int j = 0; j < lim; ++j) {
+                o[j].key = pooled[(size_t)b * n + j];
+                o[j].idx = j;
+            }
+            qsort(o, (size_t)lim, sizeof(keyed), cmp_desc_key_asc_idx);
+            mark_first(o, lim, sb - w, sset + (size_t)b * n);
+            for (int j = lim; j < n; ++j)
+                sset[(size_t)b * n + j] = 1;
+        }
+        if (G_out)
+            for (int j = 0; j < n; ++j)
+                G_out[g * max_n + j] = G[j];
+        if (pooled_out)
+            for (int b = 0; b < nb; ++b)
+                for (int j = 0; j < n; ++j)
+                    pooled_out[(g * nb + b) * max_n + j] = pooled[(size_t)b * n + j];
+        /* every row: the five sets and their es */
+        for (int i = 0; i < Rg; ++i) {
+            const int64_t row = g * Rg + i;
+            instance I;
+            if (load_row(R, row, &I)) {
+                instance_free(&I);
+                continue;
+            }
+            for (int b = 0; b < nb; ++b) {
+                const int sb = s[b];
+                for (int sel = 0; sel < 5; ++sel) {
+                    memset(in, 0, (size_t)n);
+                    int any = sb >= 1 && sb <= n;
+                    if (any && sel == 0) {
+                        const int sinks = sb / 2 < 4 ? sb / 2 : 4;
+                        for (int j = 0; j < n; ++j)
+                            in[j] = j < sinks || j >= n - (sb - sinks);
+                    } else if (any && sel == 1) {
+                        memcpy(in, hset + (size_t)b * n, (size_t)n);
+                    } else if (any && sel == 2) {
+                        memcpy(in, sset + (size_t)b * n, (size_t)n);
+                    } else if (any) {
+                        const int P = sel == 3 ? (sb / 4 > 2 ? sb / 4 : 2) : 16;
+                        const int np = (n + P - 1) / P, mp = sb / P;
+                        if (sel == 4 && sb < 16)
+                            any = 0;
+                        if (mp < 1)
+                            any = 0;
+                        if (any) {
+                            for (int p = 0; p < np; ++p) {
+                                double m = -INFINITY;
+                                for (int j = p * P; j < n && j < p * P + P; ++j)
+                                    if ((double)I.logit[j] > m)
+                                        m = (double)I.logit[j];
+                                o[p].key = m;
+                                o[p].idx = p;
+                            }
+                            qsort(o, (size_t)np, sizeof(keyed), cmp_desc_key_asc_idx);
+                            for (int t = 0; t < mp && t < np; ++t)
+                                for (int j = o[t].idx * P; j < n && j < o[t].idx * P + P; ++j)
+                                    in[j] = 1;
+                        }
+                    }
+                    int cnt = 0;
+                    for (int j = 0; j < n; ++j)
+                        cnt += in[j];
+                    es[(row * 5 + sel) * nb + b] = cnt > 0 ? eval_set(&I, in, NULL).gap : NAN;
+                    if (bits) {
+                        uint32_t *wv = bits + ((row * 5 + sel) * nb + b) * (int64_t)words;
+                        for (int t = 0; t < words; ++t)
+                            wv[t] = 0u;
+                        for (int j = 0; j < n; ++j)
+                            if (in[j])
+                                wv[j >> 5] |= 1u << (j & 31);
+                    }
+                }
+            }
+            instance_free(&I);
+        }
+        free(o);
+        free(in);
+        free(sset);
+        free(hset);
+        free(pooled);
+        free(vote);
+        free(G);
+    }
+    return bad ? ORC_ERR_ARG : ORC_OK;
+}
+
 /* ---------------------------------------------------------- group vote */
 
 /* f1: the group vote (Sec. 2.1, shared kept sets).  Deployment keeps one set

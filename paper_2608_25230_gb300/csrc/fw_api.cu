@@ -337,4 +337,29 @@ fw_status fw_window_score(const void *Qw, const void *K, int32_t cells, int32_t 
     return window_score(Qw, K, cells, T, d, w, scale, pool, scores, workspace, status, (cudaStream_t)stream);
 }
 
+size_t fw_selector_audit_workspace(const fw_rows *rows, int32_t nb)
+{
+    RowsDev R;
+    if (check_rows(rows, R) != FW_OK || nb < 1 || nb > 4) return 0;
+    return selector_audit_workspace(R, nb);
+}
+
+fw_status fw_selector_audit(const fw_rows *rows, const int32_t *s, int32_t nb, const fw_gap_out *topk, float *es,
+                            uint32_t *bits, int32_t words, void *workspace, size_t workspace_bytes, void *stream)
+{
+    RowsDev R;
+    fw_status st = check_rows(rows, R);
+    if (st != FW_OK) return st;
+    if (nb < 1 || nb > 4 || !s || !topk || !es) return FW_ERR_INVALID_ARG;
+    for (int b = 0; b < nb; ++b)
+        if (s[b] < 1 || s[b] > 4096) return FW_ERR_INVALID_ARG;
+    if (!topk->o || !topk->row_max || !topk->row_sum) return FW_ERR_INVALID_ARG;
+    if (bits && words != (R.max_n + 31) / 32) return FW_ERR_INVALID_ARG;
+    if (R.max_n > 65536) return FW_ERR_UNSUPPORTED;
+    if (R.rows == 0) return FW_OK;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < selector_audit_workspace(R, nb))
+        return FW_ERR_WORKSPACE;
+    return selector_audit(R, s, nb, *topk, es, bits, words, workspace, (cudaStream_t)stream);
+}
+
 }  // extern "C"

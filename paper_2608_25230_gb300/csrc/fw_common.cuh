@@ -211,6 +211,96 @@ __device__ __forceinline__ void stage_value_cols(const VT *V, int n, int d, int 
     }
 }
 
+// CTA-wide selection of the m largest of n unsigned order keys, equal keys
+// taken in ascending index order: on return (every thread) T is the m-th
+// largest key and L the largest index taken among the keys equal to T; key j
+// is selected iff key(j) > T or (key(j) == T and j <= L).  1 <= m <= n.
+// Three radix passes (11, 11, 10 bits) over a 2048-bin shared histogram, then
+// an index-order scan of the keys equal to T.  key(j) is called for j < n by
+// every thread of the block (all threads must call this function).
+struct TopmSmem {
+    uint32_t hist[2048];
+    int wcnt[32];
+    uint32_t digit;
+    int rem, L;
+};
+template <typename KeyFn>
+__device__ __forceinline__ void block_topm(int n, int m, KeyFn key, TopmSmem &S, uint32_t &T, int &L)
+{
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, nt = blockDim.x, nw = nt >> 5;
+    uint32_t prefix = 0, pmask = 0;
+    int rem = m;
+    if (tid == 0) {
+        S.digit = 0u;
+        S.rem = 1;
+    }
+    for (int pass = 0; pass < 3; ++pass) {
+        const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
+        const int nbin = pass < 2 ? 2048 : 1024;
+        for (int i = tid; i < 2048; i += nt) S.hist[i] = 0u;
+        __syncthreads();
+        for (int j = tid; j < n; j += nt) {
+            const uint32_t u = key(j);
+            if ((u & pmask) == prefix) atomicAdd(&S.hist[(u >> shift) & (uint32_t)(nbin - 1)], 1u);
+        }
+        __syncthreads();
+        if (wid == 0) {
+            const int per = nbin / 32;  // bins in descending order, per lanes
+            const int top = nbin - 1 - lane * per;
+            int c = 0;
+            for (int q = 0; q < per; ++q) c += (int)S.hist[top - q];
+            int incl = c;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int y = __shfl_up_sync(FW_FULL, incl, off);
+                if (lane >= off) incl += y;
+            }
+            const int excl = incl - c;
+            if (excl < rem && rem <= incl) {
+                int acc = excl;
+                for (int q = 0; q < per; ++q) {
+                    const int h = (int)S.hist[top - q];
+                    if (acc + h >= rem) {
+                        S.digit = (uint32_t)(top - q);
+                        S.rem = rem - acc;
+                        break;
+                    }
+                    acc += h;
+                }
+            }
+        }
+        __syncthreads();
+        prefix |= S.digit << shift;
+        pmask |= (uint32_t)(nbin - 1) << shift;
+        rem = S.rem;
+        __syncthreads();
+    }
+    T = prefix;
+    // the rem-th key equal to T in index order
+    if (tid == 0) S.L = -1;
+    __syncthreads();
+    int run = 0;
+    for (int j0 = 0; j0 < n; j0 += nt) {
+        const int j = j0 + tid;
+        const bool eq = j < n && key(j) == T;
+        const unsigned bm = __ballot_sync(FW_FULL, eq);
+        if (lane == 0) S.wcnt[wid] = __popc(bm);
+        __syncthreads();
+        int before = run, tot = 0;
+        for (int w = 0; w < nw; ++w) {
+            if (w < wid) before += S.wcnt[w];
+            tot += S.wcnt[w];
+        }
+        before += __popc(bm & ((1u << lane) - 1u));
+        if (eq && before + 1 == rem) S.L = j;
+        run += tot;
+        __syncthreads();
+        if (S.L >= 0) break;
+    }
+    L = S.L;
+    __syncthreads();
+}
+
 // Dispatch on the value width d (multiples of 32 supported: 32, 64, 128, 256)
 // and the value dtype; binds DPL (dims per lane) and VT (element type).
 #define FW_DISPATCH(d, vdt, ...)                                                              \

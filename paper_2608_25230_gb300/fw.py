@@ -79,6 +79,11 @@ _lib.fw_window_score.argtypes = [vp, vp, C.c_int32, C.c_int32, C.c_int32, C.c_in
 _lib.fw_window_score.restype = C.c_int
 _lib.fw_window_score_workspace.argtypes = [C.c_int32, C.c_int32]
 _lib.fw_window_score_workspace.restype = C.c_size_t
+_lib.fw_selector_audit.argtypes = [C.POINTER(FwRows), vp, C.c_int32, C.POINTER(FwGapOut), vp, vp, C.c_int32, vp,
+                                   C.c_size_t, vp]
+_lib.fw_selector_audit.restype = C.c_int
+_lib.fw_selector_audit_workspace.argtypes = [C.POINTER(FwRows), C.c_int32]
+_lib.fw_selector_audit_workspace.restype = C.c_size_t
 _lib.fw_ragged_compact.argtypes = [vp, vp, C.c_int32, C.c_int32, C.c_int32, vp, vp, C.c_int64, vp, vp, vp]
 _lib.fw_group_vote.argtypes = [C.POINTER(FwRows), vp, C.c_int32, C.POINTER(FwGapOut), vp, vp, vp, C.c_int32, vp,
                                vp, C.c_size_t, vp]
@@ -407,6 +412,28 @@ def window_score(Qw: torch.Tensor, K: torch.Tensor, *, scale: float = None, pool
                               _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
     _check(st, "fw_window_score")
     return scores, status
+
+
+SELECTORS = ("streamingllm", "h2o", "snapkv", "quest", "quest16")
+
+
+def selector_audit(rows: Rows, s, topk: dict, *, bits=False, stream=None):
+    """fw_selector_audit: es of every deployed rule's kept set ([rows][5][nb],
+    rules in SELECTORS order) at the host budgets s; optionally the sets."""
+    dev, R = rows.device, rows.num_rows
+    s = [int(x) for x in s]
+    nb = len(s)
+    words = (rows.max_n + 31) // 32
+    out = dict(es=torch.empty(R, len(SELECTORS), nb, dtype=torch.float32, device=dev))
+    if bits:
+        out["bits"] = torch.empty(R, len(SELECTORS), nb, words, dtype=torch.int32, device=dev)
+    sh = (C.c_int32 * nb)(*s)
+    ws = _ws(_lib.fw_selector_audit_workspace(C.byref(rows.c), nb), dev)
+    st = _lib.fw_selector_audit(C.byref(rows.c), sh, nb, C.byref(topk["_c"]), _ptr(out["es"]), _ptr(out.get("bits")),
+                                words, _ptr(ws), ws.numel(), _stream(stream))
+    _check(st, "fw_selector_audit")
+    out["_ws"] = ws
+    return out
 
 
 def raw():
