@@ -13,9 +13,11 @@ Also timed in the same run (reported under "sections"), one line per config:
   exact_toy       256 rows, n=20, k=5, d=64: the whole path
   adversarial     512 rows each of flat, near-duplicate and planted-tie rows
   long_rows       4,096 rows x 32,768 keys, d=128, three budgets: gap, swap, vote
-  contour         ContourKV allocation + ragged compaction, 256 cells x 32,768 tokens
+  contour         ContourKV allocation + ragged compaction, 256 cells x 32,768 tokens;
+                  the capped (enforced) allocation, the window score, decode appends
   mixed_profiles  168,192 ragged rows (n 1,024..16,384, GQA-4, bf16 V): gap + swap
   pool            ES_pool (Definition 2.2) at s = 4/8/16/32 on mixed-profile rows
+  audit           the deployed selectors' es against ES_pool and top-mass (App. C)
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 """
@@ -470,6 +472,46 @@ def section_contour(fw, device, K, W, flush, peaks):
     total, times = time_steps(step, K, W, flush, lambda: None)
     ms = total / K
     parts = ev.take()[-2 * K:]
+    # the enforced mode: every cell capped at the uniform count
+    holder = {}
+
+    def capped_step():
+        holder["c"] = fw.contour_alloc_capped(cb.scores, floor=cb.floor, total_budget=cb.total_budget,
+                                              uniform_s=cb.uniform_s, cap=cb.uniform_s)
+
+    tc_, _ = time_steps(capped_step, K, W, flush, lambda: None)
+    ms_capped = tc_ / K
+    kept_capped = int(holder["c"]["offsets"][-1].item())
+    # the observation-window score (32 window queries per cell) on the cache's keys
+    Qw = workloads.window_queries(seed=0, cells=cb.cells, w=32, d=cb.d, backend="torch", device=device)
+    Qi = Qw.view(torch.int16)
+    wsc = torch.empty(cb.cells, cb.T, dtype=torch.float32, device=device)
+
+    def wscore_step():
+        fw.window_score(Qi, Kc, pool=7, out=wsc)
+
+    tw, _ = time_steps(wscore_step, K, W, flush, lambda: None)
+    ms_ws = tw / K
+    wbytes = cb.cells * cb.T * cb.d * 2 + cb.cells * 32 * cb.d * 2 + 2 * cb.cells * cb.T * 4
+    wflops = 2 * 2 * cb.cells * 32 * cb.T * cb.d  # two passes of the window products
+    # decode-time appends: one new row per cell into storage with 64 rows of room per cell
+    cnt = holder["c"]["counts"].to(torch.int32)
+    cap = (cnt + 64).to(torch.int32)
+    base = torch.cumsum(cap.to(torch.int64), 0) - cap.to(torch.int64)
+    rows_store = int((base[-1] + cap[-1]).item())
+    Ks = torch.empty(rows_store, cb.d, dtype=torch.int16, device=device)
+    Vs = torch.empty_like(Ks)
+    nK = torch.zeros(cb.cells, 1, cb.d, dtype=torch.int16, device=device)
+    nV = torch.zeros_like(nK)
+    fill = torch.zeros_like(cnt)
+    st_app = torch.empty_like(cnt)
+
+    def append_step():
+        fill.zero_()
+        fw.ragged_append(Ks, Vs, base, cap, fill, nK, nV, st_app)
+
+    ta, _ = time_steps(append_step, K, W, flush, lambda: None)
+    ms_app = ta / K
     ms_alloc = sum(t for t, tag in parts if tag == "alloc") / K
     ms_comp = sum(t for t, tag in parts if tag == "compact") / K
     nbytes = cb.cells * cb.T * 4 + 2 * 2 * cb.total_budget * cb.d * 2 + cb.total_budget * 4 + (cb.cells + 1) * 8
@@ -481,7 +523,19 @@ def section_contour(fw, device, K, W, flush, peaks):
                 roofline=roofline("hbm", ach, peaks["hbm_gbs"], "GB/s", traffic_of("contour", cb.total_budget),
                                   algorithmic_bytes=nbytes, kernel="k_c_* + k_compact"),
                 compact_roofline=roofline("hbm", cbytes / (ms_comp * 1e-3) / 1e9, peaks["hbm_gbs"], "GB/s",
-                                          kernel="k_compact", algorithmic_bytes=cbytes))
+                                          kernel="k_compact", algorithmic_bytes=cbytes),
+                capped=dict(path="fw_contour_alloc_capped, cap = uniform count (4,096): the enforced mode",
+                            ms_per_call=ms_capped, kept_rows=kept_capped),
+                window_score=dict(path="fw_window_score: 32 window queries x 256 cells x 32,768 keys, d=128, "
+                                       "pool 7 (TMA + tcgen05, two passes over K)",
+                                  ms_per_call=ms_ws, keys_per_s=cb.cells * cb.T / (ms_ws * 1e-3),
+                                  roofline=roofline("hbm", wbytes / (ms_ws * 1e-3) / 1e9, peaks["hbm_gbs"], "GB/s",
+                                                    kernel="k_wscore", algorithmic_bytes=wbytes,
+                                                    bytes_basis="K once, the window queries, votes and scores "
+                                                                "written; the kernel reads K twice"),
+                                  tensor_tflops=wflops / (ms_ws * 1e-3) / 1e12),
+                decode_append=dict(path="fw_ragged_append: one new K/V row per cell (256 cells, d=128)",
+                                   ms_per_call=ms_app, rows_per_s=cb.cells / (ms_app * 1e-3)))
 
 
 def section_mixed(fw, device, K, W, flush, peaks, rows_scale=1.0):
@@ -562,6 +616,37 @@ def section_pool(fw, device, K, W, flush, peaks, groups=256):
     return out
 
 
+def section_audit(fw, device, K, W, flush, peaks, groups=256):
+    """f4: the deployed selectors' es against ES_pool and top-mass at s = 4/8/16/32
+    on the first `groups` GQA groups of mixed profile B (n = 4,096, d = 128): the
+    audit call's time and the median of each rule's es / ES_pool."""
+    prof = workloads.MIXED_PROFILES[1]
+    b = workloads.mixed_profiles(seed=1, backend="torch", device=device, profiles=(prof,),
+                                 rows_scale=groups * 4 / prof[1])[0]
+    rows = fw.rows_from_batch(b, device)
+    R = rows.num_rows
+    sched = [s for s, _ in POOL_SCHED]
+    k = torch.tensor(sched, dtype=torch.int32, device=device).repeat(R, 1)
+    top = fw.dense_and_topk_gap(rows, k, kept_bits=False, o_kept=False)
+    holder = {}
+
+    def step():
+        holder["a"] = fw.selector_audit(rows, sched, top)
+
+    t, _ = time_steps(step, K, W, flush, lambda: None)
+    ms = t / K
+    pool = fw.pool_best_subset(rows, k, top, E=[e for _, e in POOL_SCHED])
+    es = holder["a"]["es"].double()
+    esp = pool["best_gap"].double()
+    ratios = {}
+    for j, s in enumerate(sched):
+        r = {name: float(torch.nanmedian(es[:, i, j] / esp[:, j]).item()) for i, name in enumerate(fw.SELECTORS)}
+        r["top_mass"] = float(torch.median(top["gap"].double()[:, j] / esp[:, j]).item())
+        ratios[f"s={s}"] = r
+    return dict(workload=f"mixed profile B, first {groups} GQA groups ({R} rows, n=4096, d=128)",
+                ms_per_call=ms, rows_per_s=R / (ms * 1e-3), median_es_over_ES_pool=ratios)
+
+
 # --------------------------------------------------------------------- main
 
 def main():
@@ -575,7 +660,7 @@ def main():
     ap.add_argument("--rows-scale", type=float, default=1.0,
                     help="fraction of the headline rows (profiling captures of a smaller case)")
     ap.add_argument("--only", default="all",
-                    choices=["all", "exact_toy", "adversarial", "long_rows", "contour", "mixed", "pool"],
+                    choices=["all", "exact_toy", "adversarial", "long_rows", "contour", "mixed", "pool", "audit"],
                     help="run one section alone and print its line (profiling captures)")
     ap.add_argument("--long-rows-per-head", type=int, default=512,
                     help="rows per head of the long-row section (profiling captures of a smaller case)")
@@ -630,7 +715,8 @@ def main():
         long_rows=lambda k, w: section_long_rows(fw, device, k, w, flush, peaks, rows_per_head=args.long_rows_per_head),
         contour=lambda k, w: section_contour(fw, device, k, w, flush, peaks),
         mixed=lambda k, w: section_mixed(fw, device, k, w, flush, peaks, rows_scale=args.mixed_rows_scale),
-        pool=lambda k, w: section_pool(fw, device, k, w, flush, peaks))
+        pool=lambda k, w: section_pool(fw, device, k, w, flush, peaks),
+        audit=lambda k, w: section_audit(fw, device, k, w, flush, peaks))
     if args.only != "all":
         if rank == 0:
             print(json.dumps(dict(section=args.only, **{"result": sections_fn[args.only](K, W)})), flush=True)
@@ -669,7 +755,7 @@ def main():
 
     sections = {}
     if not args.no_sections and rank == 0:
-        for name in ("exact_toy", "adversarial", "long_rows", "contour", "mixed", "pool"):
+        for name in ("exact_toy", "adversarial", "long_rows", "contour", "mixed", "pool", "audit"):
             sections[name] = sections_fn[name](5, 3)
 
     cpu = None

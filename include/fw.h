@@ -238,7 +238,7 @@ fw_status fw_pool_best_subset(const fw_rows *rows, const int32_t *k, int32_t nb,
 /* Workspace bytes: the pool of every (row, budget), 64 int32 each, and its size. */
 size_t fw_pool_best_subset_workspace(const fw_rows *rows, int32_t nb);
 
-/* The deployed selectors audited in Sec. 2.4 (App. D settings), as kept sets
+/* The deployed selectors audited in Sec. 2.3 (App. C settings), as kept sets
  * scored with Definition 2.1's es.  For budget s:
  *   FW_SEL_STREAMING  the first min(4, s/2) positions and the last
  *                     s - min(4, s/2) (StreamingLLM: sinks plus recency);

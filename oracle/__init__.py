@@ -356,7 +356,7 @@ SELECTORS = ("streamingllm", "h2o", "snapkv", "quest", "quest16")
 
 
 def selector_audit(batch, s):
-    """f4: the deployed selectors' kept sets and their es (App. D settings).
+    """f4: the deployed selectors' kept sets and their es (App. C settings).
     s: budgets (nb).  Returns es [rows][5][nb], bits [rows][5][nb][words],
     G [groups][max_n], pooled [groups][nb][max_n]."""
     H = batch if isinstance(batch, HostRows) else HostRows(batch)

@@ -1119,7 +1119,7 @@ int orc_window_score(const uint16_t *Qw, const uint16_t *K, int cells, int T, in
     return ORC_OK;
 }
 
-/* f4: the deployed selectors audited in Sec. 2.4 with App. D's settings, each
+/* f4: the deployed selectors audited in Sec. 2.3 with App. C's settings, each
  * a kept set scored with es (Definition 2.1).  For budget s:
  *   StreamingLLM: positions j < min(4, s/2) and j >= n - (s - min(4, s/2));
  *   H2O: positions j >= n - s/2, and of j < n - s/2 the s - s/2 of largest

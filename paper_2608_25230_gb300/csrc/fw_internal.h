@@ -89,7 +89,7 @@ size_t window_score_workspace(int cells, int T);
 fw_status window_score(const void *Qw, const void *K, int cells, int T, int d, int w, float scale, int pool,
                        float *scores, void *ws, int32_t *status, cudaStream_t s);
 
-// The deployed selectors' kept sets, scored (Sec. 2.4, App. D).
+// The deployed selectors' kept sets, scored (Sec. 2.3, App. C).
 size_t selector_audit_workspace(const RowsDev &R, int nb);
 fw_status selector_audit(const RowsDev &R, const int32_t *s, int nb, const fw_gap_out &topk, float *es,
                          uint32_t *bits, int words, void *ws, cudaStream_t st);

@@ -1,7 +1,7 @@
-// k_audit.cu -- the deployed selectors audited in Sec. 2.4 / App. D, as
+// k_audit.cu -- the deployed selectors audited in Sec. 2.3 / App. C, as
 // kernels: for every row and budget s, the kept set that each rule would
 // choose, scored with Definition 2.1's es(A) = ||m_A - mu|| (to be set against
-// the top-mass set and ES_pool).  The rules, with App. D's settings:
+// the top-mass set and ES_pool).  The rules, with App. C's settings:
 //   StreamingLLM  the first min(4, s/2) positions (sinks) and the last
 //                 s - sinks positions (recency);
 //   H2O           the last s/2 positions and, among the others, the

@@ -1,5 +1,5 @@
 """GPU parity for the selector audit (fw_selector_audit: StreamingLLM, H2O,
-SnapKV, Quest, Quest-16 with App. D's settings, each kept set scored with es)
+SnapKV, Quest, Quest-16 with App. C's settings, each kept set scored with es)
 against the fp64 oracle.  StreamingLLM and Quest sets are bit-exact (positions
 and exact logit maxima decide them).  H2O and SnapKV rank fp32 sums of masses
 over the group's rows; where their set differs from the oracle's, it must be a

@@ -1,4 +1,4 @@
-"""Pins for the selector-audit oracle (Sec. 2.4, App. D's settings): each
+"""Pins for the selector-audit oracle (Sec. 2.3, App. C's settings): each
 rule's kept set rebuilt with numpy sorts from its definition, and its es from
 the forced-weight output m_A = sum_A p v / p(A); set sizes; the rules that
 ignore the logits (StreamingLLM).  CPU only."""

@@ -367,7 +367,7 @@ def contour_cache(seed: int = 0, cells: int = 256, T: int = 32768, d: int = 128,
 
 # Window queries for the observation-window score: the last w query rows of
 # every cell of a contour_cache, bf16 ~ N(0, 1) like its keys (w = 32, the
-# largest SnapKV window of App. D).
+# largest SnapKV window of App. C).
 def window_queries(seed: int = 0, cells: int = 256, w: int = 32, d: int = 128, backend: str = "numpy",
                    device: str = "cuda"):
     rng = make_rng(seed * 1000 + 5, backend, device)
