@@ -2,6 +2,8 @@
 // kernel translation units.
 #pragma once
 
+#include <cuda.h>  // CUtensorMap (types only; the encoder is fetched from the driver at run time)
+
 #include "fw_common.cuh"
 
 namespace fw {
@@ -93,6 +95,11 @@ fw_status window_score(const void *Qw, const void *K, int cells, int T, int d, i
 size_t selector_audit_workspace(const RowsDev &R, int nb);
 fw_status selector_audit(const RowsDev &R, const int32_t *s, int nb, const fw_gap_out &topk, float *es,
                          uint32_t *bits, int words, void *ws, cudaStream_t st);
+
+// A TMA map of a 2-D bf16 tensor [rows][cols] (cols innermost, row stride
+// cols * 2 bytes) read in boxes of box_rows x 64 elements with the 128-byte
+// swizzle.  False if the driver's encoder is unavailable or refuses the map.
+bool make_tma_2d_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 
 // Number of SMs of the current device (queried once per device).
 fw_status device_sms(int *sms);

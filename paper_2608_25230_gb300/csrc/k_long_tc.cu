@@ -442,6 +442,439 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
     }
 }
 
+// ---------------------------------------------------------------------------
+// The same P.V with one copy warp: V tiles arrive by TMA (64 keys x 64 dims
+// boxes, 128-byte swizzle: the MN-major operand layout) and each row's 64
+// logits of a stage by one bulk copy, so the producer warps only build A.
+// Warp 0 copies, warp 1 issues the MMAs, warps 2..9 produce: a thread takes
+// 8 consecutive keys of one row (NB budgets known at compile time) and writes
+// one 16-byte vector per (band row, term).  Stages whose V rows would cross
+// the end of the group's block (the partial last stage, or a block not
+// aligned to whole rows) and logit rows that cannot be bulk-copied (n not a
+// multiple of 4, misaligned base) go through per-thread cp.async with zero
+// fill instead, tracked by the same barrier.
+template <int D> __host__ __device__ constexpr int pvm_pw() { return D == 128 ? 16 : 8; }  // producer warps
+template <int D> __host__ __device__ constexpr int pvm_nt() { return (pvm_pw<D>() + 2) * 32; }
+constexpr int PVM_BS = 3;                      // copy slots (V + ones + logits)
+
+__device__ __forceinline__ uint32_t cvt_bf16x2(float hi_elem, float lo_elem)
+{
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi_elem), "f"(lo_elem));
+    return r;
+}
+__device__ __forceinline__ void cp_async_mbar_arrive(uint64_t *bar)
+{
+    asm volatile("cp.async.mbarrier.arrive.shared.b64 [%0];" ::"r"(tc::smem_u32(bar)) : "memory");
+}
+
+template <int D, int NB>
+__global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_constant__ CUtensorMap tmV, const TcArgs a)
+{
+    constexpr int NBB = NB + 1;                 // bands
+    constexpr int RT = TM / NBB < MAXRT ? TM / NBB : MAXRT;
+    constexpr int PW = pvm_pw<D>();
+    constexpr int NT = pvm_nt<D>();
+    constexpr int NPROD = PW * 32;
+    constexpr int TPR = NPROD / MAXRT;          // producer threads per row
+    constexpr int KPTH = KS / TPR;              // keys per producer thread and stage (4 or 8)
+    constexpr int NVBOX = D / 64;               // 64-dim groups of V
+    constexpr int NG = NVBOX + 1;               // ... and one group of ones (the band masses)
+    constexpr int B_SLOT_BYTES = NG * KS * 128;
+    constexpr int DN = D + 16;                  // MMA N: the value dims, then 16 columns of masses
+    constexpr uint32_t TCOLS = NACC * DN <= 256 ? 256u : 512u;
+    constexpr int NC = D / 8;
+    constexpr int FCOLS = D / (PW / 4);         // accumulator columns flushed per warp (32)
+    extern __shared__ uint8_t smraw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~(uintptr_t)1023);
+    uint8_t *sA = sm;                                     // [ASLOTS][NSPLIT][TM x 128 B]
+    uint8_t *sB = sA + ASLOTS * A_SLOT_BYTES;             // [PVM_BS][NG][64 keys x 128 B]
+    float *sL = reinterpret_cast<float *>(sB + PVM_BS * B_SLOT_BYTES);  // [PVM_BS][32][64]
+    float *acc = reinterpret_cast<float *>(sA);           // epilogue: [TM][D + 1]
+    __shared__ __align__(8) uint64_t fullB[PVM_BS], freeB[PVM_BS], fullA[ASLOTS], freeA[ASLOTS], accfree[NACC];
+    __shared__ uint32_t s_taddr;
+    __shared__ int s_err;
+    __shared__ float rowM[MAXRT], rowZi[MAXRT];
+    __shared__ uint32_t rtk[MAXRT][4];
+    __shared__ int32_t rti[MAXRT][4];
+    __shared__ int rok[MAXRT];
+    __shared__ float bmass[MAXRT][5];
+
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int64_t g = blockIdx.x / a.tiles_per_group;
+    const int tile = (int)(blockIdx.x - g * a.tiles_per_group);
+    const int r0 = tile * RT;
+    const int nr = min(RT, a.R.R - r0);
+    const int n = a.R.n[g];
+    const int64_t voff = a.R.v_off[g];
+    const uint16_t *V = reinterpret_cast<const uint16_t *>(a.R.v) + voff;
+    const float *LG = a.R.logits + a.R.logit_off[g];
+    const bool vrows = voff % D == 0;  // the block starts on a whole row of the V tensor map
+    const bool lbulk = (n & 3) == 0 && (reinterpret_cast<uintptr_t>(LG) & 15) == 0;
+    const int nst = (n + KS - 1) / KS;
+
+    if (tid < MAXRT) {
+        const int r = tid;
+        rok[r] = 0;
+        if (r < nr) {
+            const int64_t row = g * a.R.R + r0 + r;
+            rok[r] = a.ws.status[row] == FW_OK;
+            rowM[r] = a.ws.M[row];
+            rowZi[r] = 1.f / a.ws.Z[row];
+            for (int b = 0; b < 4; ++b) {
+                rtk[r][b] = b < NB ? a.ws.tk[row * NB + b] : 0u;
+                rti[r][b] = b < NB ? a.ws.ti[row * NB + b] : -1;
+            }
+        }
+        for (int b = 0; b < 5; ++b) bmass[r][b] = 0.f;
+    }
+    if (tid == 0) {
+        s_err = 0;
+        for (int x = 0; x < PVM_BS; ++x) {
+            tc::mbar_init(&fullB[x], 1);
+            tc::mbar_init(&freeB[x], PW + 1);
+        }
+        for (int x = 0; x < ASLOTS; ++x) {
+            tc::mbar_init(&fullA[x], PW);
+            tc::mbar_init(&freeA[x], 1);
+        }
+        for (int x = 0; x < NACC; ++x) tc::mbar_init(&accfree[x], PW);
+        tc::mbar_init_fence();
+    }
+    // the ones group of every copy slot (constant; any swizzle of it reads 1.0)
+    for (int e = tid; e < PVM_BS * KS * 8; e += NT) {
+        const int slot = e / (KS * 8), q = e % (KS * 8);
+        reinterpret_cast<uint4 *>(sB + slot * B_SLOT_BYTES + NVBOX * (KS * 128))[q] =
+            make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    }
+    // rows of A past NBB * RT stay zero in every slot
+    for (int e = tid; e < ASLOTS * NSPLIT * TM * 8; e += NT) {
+        const int m = (e / 8) % TM;
+        if (m >= NBB * RT) reinterpret_cast<uint4 *>(sA)[e] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    tc::fence_async_smem();
+    if (wid == 1) tc::tmem_alloc(&s_taddr, TCOLS);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t taddr = s_taddr;
+
+    if (wid == 0) {
+        // ---------------------------------------------------------- copies
+        const uint32_t bbase = tc::smem_u32(sB);
+        int issued = 0;
+        bool ok = true;
+        for (int it = 0; it < nst; ++it) {
+            const int bs = it % PVM_BS, j0 = it * KS;
+            if (it >= PVM_BS) {
+                if (lane == 0) ok = tc::mbar_wait(&freeB[bs], (uint32_t)((it / PVM_BS) - 1) & 1u, WAIT_POLLS);
+                ok = __shfl_sync(FW_FULL, ok, 0);
+                if (!ok) break;
+            }
+            const int kn = min(KS, n - j0);  // keys of this stage
+            const bool vtma = vrows && kn == KS;
+            const bool live_row = lane < nr && rok[lane];
+            const float *lsrc = LG + (int64_t)(r0 + lane) * n + j0;
+            float *ldst = sL + (bs * MAXRT + lane) * KS;
+            // (1) the per-thread copies, each lane's tracked by the barrier: its
+            // pending count rises now and falls when they land, so the phase
+            // cannot complete before them whatever the order of what follows
+            if (!vtma) {  // V rows past the block's end are zero-filled
+                for (int e = lane; e < KS * NC; e += 32) {
+                    const int kk = e / NC, nc = e % NC;
+                    const int n2 = nc >> 3, c = nc & 7;
+                    const uint32_t dst = bbase + bs * B_SLOT_BYTES + n2 * (KS * 128) + (kk >> 3) * 1024 +
+                                         (kk & 7) * 128 + ((c ^ (kk & 7)) << 4);
+                    const bool in = kk < kn;
+                    cp_async16(dst, V + (int64_t)(in ? j0 + kk : 0) * D + nc * 8, in ? 16u : 0u);
+                }
+            }
+            if (!lbulk && live_row) {
+                const uint32_t d0 = tc::smem_u32(ldst);
+                for (int u = 0; u < kn; ++u) cp_async4(d0 + 4 * u, lsrc + u, 4u);
+            }
+            if (!vtma || !lbulk) cp_async_mbar_arrive(&fullB[bs]);
+            // (2) the barrier's one expected arrival, with the bytes of the bulk copies
+            uint32_t tx = vtma ? (uint32_t)(NVBOX * 64 * 128) : 0u;
+            if (lbulk) tx += (uint32_t)(__popc(__ballot_sync(FW_FULL, live_row)) * kn * 4);
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive_expect_tx(&fullB[bs], tx);
+            __syncwarp();
+            // (3) the bulk copies: V boxes by TMA, one logit row per lane
+            if (vtma && lane == 0)
+                for (int h = 0; h < NVBOX; ++h)
+                    tc::tma_load_2d(sB + bs * B_SLOT_BYTES + h * (KS * 128), &tmV, 64 * h, (int32_t)(voff / D + j0),
+                                    &fullB[bs]);
+            if (lbulk && live_row) tc::bulk_g2s(ldst, lsrc, (uint32_t)kn * 4u, &fullB[bs]);
+            ++issued;
+        }
+        if (!ok && lane == 0) atomicOr(&s_err, 1);
+        // the copies still in flight land before the CTA moves on
+        if (lane == 0)
+            for (int it = issued - PVM_BS < 0 ? 0 : issued - PVM_BS; it < issued; ++it)
+                if (!tc::mbar_wait(&fullB[it % PVM_BS], (uint32_t)(it / PVM_BS) & 1u, WAIT_POLLS)) atomicOr(&s_err, 1);
+        __syncwarp();
+    } else if (wid == 1) {
+        // -------------------------------------------------------------- MMA
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(TM, DN, false, true);
+            // descriptors of slot 0, k-step 0, term 0; the others differ by an
+            // address offset (>> 4) in the start field, which never carries out
+            // of it (shared memory stays below 256 KB)
+            const uint64_t ad0 = tc::sdesc_sw128(tc::smem_u32(sA), 16, 1024);
+            const uint64_t bd0 = tc::sdesc_sw128(tc::smem_u32(sB), KS * 128, 1024);
+            bool ok = true;
+            int last = -1;
+            for (int it = 0; it < nst && ok; ++it) {
+                const int bs = it % PVM_BS, as = it % ASLOTS;
+                ok = tc::mbar_wait(&fullB[bs], (uint32_t)(it / PVM_BS) & 1u, WAIT_POLLS);
+                if (ok) ok = tc::mbar_wait(&fullA[as], (uint32_t)(it / ASLOTS) & 1u, WAIT_POLLS);
+                const int ch = it / CH;
+                if (ok && it % CH == 0 && ch >= NACC)
+                    ok = tc::mbar_wait(&accfree[ch % NACC], (uint32_t)((ch - NACC) / NACC) & 1u, WAIT_POLLS);
+                if (!ok) break;
+                tc::fence_after_sync();
+                const uint32_t dacc = taddr + (uint32_t)((ch % NACC) * DN);
+                const bool fresh = it % CH == 0;
+                const uint64_t abase = ad0 + (uint64_t)((as * A_SLOT_BYTES) >> 4);
+                const uint64_t bbs = bd0 + (uint64_t)((bs * B_SLOT_BYTES) >> 4);
+#pragma unroll
+                for (int ks = 0; ks < KS / 16; ++ks) {
+                    const uint64_t bd = bbs + (uint64_t)((ks * 2048) >> 4);
+#pragma unroll
+                    for (int sp = 0; sp < NSPLIT; ++sp)
+                        tc::mma_bf16(dacc, abase + (uint64_t)((sp * A_SPLIT_BYTES + ks * 32) >> 4), bd, idesc,
+                                     !fresh || ks > 0 || sp > 0);
+                }
+                tc::commit(&freeA[as]);
+                tc::commit(&freeB[bs]);
+                last = it;
+            }
+            if (!ok) atomicOr(&s_err, 1);
+            if (last >= 0 && !tc::mbar_wait(&freeA[last % ASLOTS], (uint32_t)(last / ASLOTS) & 1u, WAIT_POLLS))
+                atomicOr(&s_err, 1);
+        }
+        __syncwarp();
+    } else {
+        // --------------------------------------------------------- producers
+        const int pw = wid - 2;                  // 0..PW-1
+        const int ptid = tid - 64;               // 0..NPROD-1
+        const int rr = ptid / TPR;               // row of the tile (0..31)
+        const int kq = ptid % TPR;               // this thread's KPTH keys of the stage
+        const int kc = kq * KPTH / 8, hk = (kq * KPTH) % 8;  // 8-key chunk and first key in it
+        const int quarter = wid & 3, part = pw >> 2;  // TMEM lanes / columns this warp flushes
+        float racc[FCOLS];
+#pragma unroll
+        for (int i = 0; i < FCOLS; ++i) racc[i] = 0.f;
+        float rmass = 0.f;
+        const bool live = rr < nr && rok[rr];
+        const float Mr = live ? rowM[rr] : 0.f, Zr = live ? rowZi[rr] : 0.f;
+        float xt[NB];
+        int tix[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            const uint32_t tk = live ? rtk[rr][b] : 0u;
+            xt[b] = __uint_as_float((tk & 0x80000000u) ? (tk & 0x7fffffffu) : ~tk);
+            tix[b] = live ? rti[rr][b] : -1;
+        }
+        uint32_t boff[NBB];
+#pragma unroll
+        for (int b = 0; b < NBB; ++b) {
+            const int m = b * RT + rr;
+            boff[b] = (uint32_t)((m >> 3) * 1024 + (m & 7) * 128 + ((kc ^ (m & 7)) << 4) + 2 * hk);
+        }
+        bool ok = true;
+        auto chunk_end = [&](int st) { return st % CH == CH - 1 || st == nst - 1; };
+        auto flush = [&](int st) {
+            tc::fence_after_sync();
+            const int buf = (st / CH) % NACC;
+            const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
+            float v[32];
+            tc::ld32(taddr + lanes + (uint32_t)(buf * DN + part * FCOLS), v);
+#pragma unroll
+            for (int i = 0; i < FCOLS; ++i) racc[i] += v[i];
+            if (part == 0) rmass += tc::ld1(taddr + lanes + (uint32_t)(buf * DN + D));
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&accfree[buf]);
+        };
+        for (int it = 0; it < nst; ++it) {
+            const int bs = it % PVM_BS, as = it % ASLOTS, j0 = it * KS;
+            if (ok) ok = tc::mbar_wait(&fullB[bs], (uint32_t)(it / PVM_BS) & 1u, WAIT_POLLS);
+            // the A slot was last read by the MMAs of stage it - ASLOTS (which also
+            // closes chunk it - ASLOTS for the flush below)
+            if (ok && it >= ASLOTS) ok = tc::mbar_wait(&freeA[as], (uint32_t)((it / ASLOTS) - 1) & 1u, WAIT_POLLS);
+            if (!ok) break;
+            uint8_t *aslot = sA + as * A_SLOT_BYTES;
+            if (rr < RT) {
+                const float *lr = sL + (bs * MAXRT + rr) * KS + kq * KPTH;
+                float xs[KPTH];
+#pragma unroll
+                for (int q = 0; q < KPTH / 4; ++q) {
+                    const float4 x4 = *reinterpret_cast<const float4 *>(lr + 4 * q);
+                    xs[4 * q] = x4.x, xs[4 * q + 1] = x4.y, xs[4 * q + 2] = x4.z, xs[4 * q + 3] = x4.w;
+                }
+                float pv[KPTH];
+                uint32_t bdp[KPTH / 2];  // bands of keys 2q, 2q + 1 as 2 x 16 bits
+                bool tie = false;
+#pragma unroll
+                for (int u = 0; u < KPTH; ++u) {
+                    const int j = j0 + kq * KPTH + u;
+                    const float x = xs[u];
+                    pv[u] = (live && j < n) ? __expf(x - Mr) * Zr : 0.f;
+                    int bd = 0;
+#pragma unroll
+                    for (int b = 0; b < NB; ++b) {
+                        bd += x < xt[b];
+                        tie |= x == xt[b];
+                    }
+                    if (u & 1) bdp[u >> 1] |= (uint32_t)bd << 16;
+                    else bdp[u >> 1] = (uint32_t)bd;
+                }
+                if (tie) {  // a key equal to a threshold: its index decides (rare)
+#pragma unroll
+                    for (int u = 0; u < KPTH; ++u) {
+                        const int j = j0 + kq * KPTH + u;
+                        const float x = xs[u];
+                        int bd = 0;
+#pragma unroll
+                        for (int b = 0; b < NB; ++b) bd += (x < xt[b]) | ((x == xt[b]) & (j > tix[b]));
+                        const uint32_t sh = (u & 1) ? 16u : 0u;
+                        bdp[u >> 1] = (bdp[u >> 1] & ~(0xffffu << sh)) | ((uint32_t)bd << sh);
+                    }
+                }
+                // three bf16 terms per mass, two keys per 32-bit word (key 2q low)
+                uint32_t ph[KPTH / 2], pm[KPTH / 2], pl[KPTH / 2];
+#pragma unroll
+                for (int q = 0; q < KPTH / 2; ++q) {
+                    const float a0 = pv[2 * q], a1 = pv[2 * q + 1];
+                    ph[q] = cvt_bf16x2(a1, a0);
+                    const float e0 = a0 - __uint_as_float(ph[q] << 16), e1 = a1 - __uint_as_float(ph[q] & 0xffff0000u);
+                    pm[q] = cvt_bf16x2(e1, e0);
+                    const float f0 = e0 - __uint_as_float(pm[q] << 16), f1 = e1 - __uint_as_float(pm[q] & 0xffff0000u);
+                    pl[q] = cvt_bf16x2(f1, f0);
+                }
+#pragma unroll
+                for (int b = 0; b < NBB; ++b) {
+                    uint32_t wh[KPTH / 2], wm[KPTH / 2], wl[KPTH / 2];
+#pragma unroll
+                    for (int q = 0; q < KPTH / 2; ++q) {
+                        const uint32_t msk = __vcmpeq2(bdp[q], (uint32_t)b * 0x00010001u);
+                        wh[q] = ph[q] & msk;
+                        wm[q] = pm[q] & msk;
+                        wl[q] = pl[q] & msk;
+                    }
+                    uint8_t *dst = aslot + boff[b];
+                    if constexpr (KPTH == 8) {
+                        *reinterpret_cast<uint4 *>(dst) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+                        *reinterpret_cast<uint4 *>(dst + A_SPLIT_BYTES) = make_uint4(wm[0], wm[1], wm[2], wm[3]);
+                        *reinterpret_cast<uint4 *>(dst + 2 * A_SPLIT_BYTES) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+                    } else {
+                        *reinterpret_cast<uint2 *>(dst) = make_uint2(wh[0], wh[1]);
+                        *reinterpret_cast<uint2 *>(dst + A_SPLIT_BYTES) = make_uint2(wm[0], wm[1]);
+                        *reinterpret_cast<uint2 *>(dst + 2 * A_SPLIT_BYTES) = make_uint2(wl[0], wl[1]);
+                    }
+                }
+            }
+            tc::fence_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                tc::mbar_arrive(&fullA[as]);
+                tc::mbar_arrive(&freeB[bs]);  // this warp has read the stage's logits
+            }
+            if (it >= ASLOTS && chunk_end(it - ASLOTS)) flush(it - ASLOTS);
+        }
+        // the last chunks: their MMAs complete before they are read
+        for (int st = nst - ASLOTS < 0 ? 0 : nst - ASLOTS; st < nst && ok; ++st) {
+            ok = tc::mbar_wait(&freeA[st % ASLOTS], (uint32_t)(st / ASLOTS) & 1u, WAIT_POLLS);
+            if (ok && chunk_end(st)) flush(st);
+        }
+        if (!ok && lane == 0) atomicOr(&s_err, 1);
+        const int m = quarter * 32 + lane;
+        if (part == 0 && m < NBB * RT) bmass[m % RT][m / RT] = rmass;
+        // accumulators -> shared for the per-row epilogue: every MMA has completed,
+        // so the A slots (which acc overlays) are idle
+#pragma unroll
+        for (int i = 0; i < FCOLS; ++i) acc[m * (D + 1) + part * FCOLS + i] = racc[i];
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    if (wid == 1) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(taddr, TCOLS);
+    }
+    if (wid < 2) return;
+    // --------------------------------------------------------------- epilogue
+    const bool failed = s_err != 0;
+    constexpr int CPT = D / 32;
+    for (int r = wid - 2; r < nr; r += PW) {
+        const int64_t row = g * a.R.R + r0 + r;
+        if (failed) {
+            if (lane == 0 && a.out.row_status) a.out.row_status[row] = FW_ERR_TIMEOUT;
+            continue;
+        }
+        if (!rok[r]) continue;
+        float S[NBB][CPT];
+#pragma unroll
+        for (int b = 0; b < NBB; ++b)
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) S[b][t] = acc[(b * RT + r) * (D + 1) + lane + 32 * t];
+        if (a.out.o) {
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) {
+                float o = 0.f;
+#pragma unroll
+                for (int b = 0; b < NBB; ++b) o += S[b][t];
+                a.out.o[row * D + lane + 32 * t] = o;
+            }
+        }
+        for (int b = 0; b < NB; ++b) {
+            const int kb = a.k[row * NB + b];
+            int sb = 0;
+            for (int b2 = 0; b2 < NB; ++b2) {
+                const int k2 = a.k[row * NB + b2];
+                sb += (k2 < kb) || (k2 == kb && b2 < b);
+            }
+            float PA = 0.f, PC = 0.f;
+#pragma unroll
+            for (int q = 0; q < NBB; ++q) {
+                if (q <= sb) PA += bmass[r][q];
+                else PC += bmass[r][q];
+            }
+            float s2 = 0.f;
+            float NAv[CPT];
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) {
+                float NA = 0.f, NCs = 0.f;
+#pragma unroll
+                for (int q = 0; q < NBB; ++q) {
+                    if (q <= sb) NA += S[q][t];
+                    else NCs += S[q][t];
+                }
+                NAv[t] = NA;
+                const float diff = PC * NA - PA * NCs;  // p(A) (m_A - mu)
+                s2 = fmaf(diff, diff, s2);
+            }
+            s2 = warp_sum(s2);
+            if (lane == 0) {
+                const float phi = sqrtf(s2);
+                a.out.gap[row * NB + b] = phi / PA;
+                a.out.dropped[row * NB + b] = PC;
+                if (a.out.phi) a.out.phi[row * NB + b] = phi;
+            }
+            if (a.out.o_kept)
+#pragma unroll
+                for (int t = 0; t < CPT; ++t) a.out.o_kept[(row * NB + b) * D + lane + 32 * t] = NAv[t] / PA;
+        }
+    }
+}
+
+template <int D> size_t pv_tma_smem()
+{
+    return 1024 + (size_t)ASLOTS * A_SLOT_BYTES + (size_t)PVM_BS * (D / 64 + 1) * KS * 128 +
+           (size_t)PVM_BS * MAXRT * KS * 4;
+}
+
 template <int D> size_t tc_smem(int RT)
 {
     return 1024 + 2048 + (size_t)ASLOTS * A_SLOT_BYTES + (size_t)BSLOTS * D * 128 + (size_t)BSLOTS * RT * KS * 4;
@@ -457,6 +890,31 @@ bool long_pv_tc_supported(const RowsDev &R, int nb)
 fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, const LongWs &L,
                      cudaStream_t s)
 {
+    // the copy-warp kernel (TMA for V, bulk copies for logits) when the driver
+    // can encode the V tensor map; the rows of the map are every whole row the
+    // block may address (boxes are only issued inside a group's own block)
+    CUtensorMap mv;
+    if (make_tma_2d_bf16(&mv, R.v, (uint64_t)1 << 31, (uint64_t)R.d, 64)) {
+        TcArgs a;
+        a.R = R;
+        a.k = k;
+        a.nb = nb;
+        a.out = out;
+        a.ws = L;
+        a.RT = TM / (nb + 1) < MAXRT ? TM / (nb + 1) : MAXRT;
+        a.tiles_per_group = (R.R + a.RT - 1) / a.RT;
+        const unsigned grid = (unsigned)(R.num_groups * a.tiles_per_group);
+        auto launch = [&](auto kernel, size_t smem) -> fw_status {
+            FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+            FW_LAUNCH(kernel, grid, (R.d == 128 ? pvm_nt<128>() : pvm_nt<64>()), smem, s, mv, a);
+            return FW_OK;
+        };
+#define FW_PV_NB(DD, NN) \
+    if (R.d == DD && nb == NN) return launch(k_long_pv_tma<DD, NN>, pv_tma_smem<DD>());
+        FW_PV_NB(128, 1) FW_PV_NB(128, 2) FW_PV_NB(128, 3) FW_PV_NB(128, 4)
+        FW_PV_NB(64, 1) FW_PV_NB(64, 2) FW_PV_NB(64, 3) FW_PV_NB(64, 4)
+#undef FW_PV_NB
+    }
     TcArgs a;
     a.R = R;
     a.k = k;

@@ -245,39 +245,6 @@ __global__ void __launch_bounds__(WS_THREADS, 2) k_wscore(const __grid_constant_
     }
 }
 
-using EncodeTiled = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                 const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
-                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiled encoder()
-{
-    static EncodeTiled fn = nullptr;
-    if (!fn) {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiled>(p);
-    }
-    return fn;
-}
-
-// A 2-D bf16 tensor [rows][cols] (cols innermost) read in boxes of box_rows x 64
-// with the 128-byte swizzle.
-bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows)
-{
-    EncodeTiled enc = encoder();
-    if (!enc) return false;
-    const cuuint64_t dims[2] = {cols, rows};
-    const cuuint64_t strides[1] = {cols * 2};
-    const cuuint32_t box[2] = {64, box_rows};
-    const cuuint32_t estr[2] = {1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 }  // namespace
 
 size_t window_score_workspace(int cells, int T) { return align256((size_t)cells * T * 4); }
@@ -286,8 +253,8 @@ fw_status window_score(const void *Qw, const void *K, int cells, int T, int d, i
                        float *scores, void *ws, int32_t *status, cudaStream_t s)
 {
     CUtensorMap mk, mq;
-    if (!make_map(&mk, K, (uint64_t)cells * T, (uint64_t)d, WS_KT)) return FW_ERR_CUDA;
-    if (!make_map(&mq, Qw, (uint64_t)cells * w, (uint64_t)d, WS_N)) return FW_ERR_CUDA;
+    if (!make_tma_2d_bf16(&mk, K, (uint64_t)cells * T, (uint64_t)d, WS_KT)) return FW_ERR_CUDA;
+    if (!make_tma_2d_bf16(&mq, Qw, (uint64_t)cells * w, (uint64_t)d, WS_N)) return FW_ERR_CUDA;
     WsArgs a;
     a.cells = cells;
     a.T = T;
