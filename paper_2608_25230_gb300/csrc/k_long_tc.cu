@@ -444,15 +444,18 @@ __global__ void __launch_bounds__(pv_threads<D>(), 1) k_long_pv_tc(const TcArgs 
 
 // ---------------------------------------------------------------------------
 // The same P.V with one copy warp: V tiles arrive by TMA (64 keys x 64 dims
-// boxes, 128-byte swizzle: the MN-major operand layout) and each row's 64
-// logits of a stage by one bulk copy, so the producer warps only build A.
-// Warp 0 copies, warp 1 issues the MMAs, warps 2..9 produce: a thread takes
-// 8 consecutive keys of one row (NB budgets known at compile time) and writes
-// one 16-byte vector per (band row, term).  Stages whose V rows would cross
-// the end of the group's block (the partial last stage, or a block not
-// aligned to whole rows) and logit rows that cannot be bulk-copied (n not a
-// multiple of 4, misaligned base) go through per-thread cp.async with zero
-// fill instead, tracked by the same barrier.
+// boxes, 128-byte swizzle: the MN-major operand layout) and the stage's
+// logits (64 per row) by 16-byte cp.async, half a warp per row, so the
+// producer warps only build A.  (One bulk copy per 256-byte logit row was
+// tried first: 32 small TMA requests per stage kept the stage time near
+// 1.3 us, about three times the MMA time.)  Warp 0 copies, warp 1 issues the
+// MMAs, the other warps produce: a thread takes KPTH consecutive keys of one
+// row (NB budgets known at compile time) and writes one vector per (band row,
+// term).  Stages whose V rows would cross the end of the group's block (the
+// partial last stage, or a block not aligned to whole rows) go through
+// per-thread cp.async with zero fill instead, and logit rows that are not
+// 16-byte aligned (n not a multiple of 4, misaligned base) through 4-byte
+// cp.async; the barrier tracks every kind.
 template <int D> __host__ __device__ constexpr int pvm_pw() { return D == 128 ? 16 : 8; }  // producer warps
 template <int D> __host__ __device__ constexpr int pvm_nt() { return (pvm_pw<D>() + 2) * 32; }
 constexpr int PVM_BS = 3;                      // copy slots (V + ones + logits)
@@ -561,7 +564,9 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
 
     if (wid == 0) {
         // ---------------------------------------------------------- copies
-        const uint32_t bbase = tc::smem_u32(sB);
+        const uint32_t bbase = tc::smem_u32(sB), lbase = tc::smem_u32(sL);
+        const uint32_t livemask = __ballot_sync(FW_FULL, lane < nr && rok[lane]);
+        const int lc = lane & 15, lh = lane >> 4;  // 16-byte chunk of a logit row, row parity
         int issued = 0;
         bool ok = true;
         for (int it = 0; it < nst; ++it) {
@@ -573,9 +578,7 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
             }
             const int kn = min(KS, n - j0);  // keys of this stage
             const bool vtma = vrows && kn == KS;
-            const bool live_row = lane < nr && rok[lane];
-            const float *lsrc = LG + (int64_t)(r0 + lane) * n + j0;
-            float *ldst = sL + (bs * MAXRT + lane) * KS;
+            const bool live_row = (livemask >> lane) & 1u;
             // (1) the per-thread copies, each lane's tracked by the barrier: its
             // pending count rises now and falls when they land, so the phase
             // cannot complete before them whatever the order of what follows
@@ -589,23 +592,30 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
                     cp_async16(dst, V + (int64_t)(in ? j0 + kk : 0) * D + nc * 8, in ? 16u : 0u);
                 }
             }
-            if (!lbulk && live_row) {
-                const uint32_t d0 = tc::smem_u32(ldst);
+            if (lbulk) {  // 16-byte copies, half a warp per row (kn is a multiple of 4)
+                const bool cin = lc * 4 < kn;
+                for (int rp = 0; rp < nr; rp += 2) {
+                    const int r = rp + lh;
+                    if ((livemask >> r) & 1u)
+                        cp_async16(lbase + (uint32_t)(((bs * MAXRT + r) * KS + lc * 4) * 4),
+                                   LG + (int64_t)(r0 + r) * n + j0 + (cin ? lc * 4 : 0), cin ? 16u : 0u);
+                }
+            } else if (live_row) {
+                const uint32_t d0 = lbase + (uint32_t)((bs * MAXRT + lane) * KS * 4);
+                const float *lsrc = LG + (int64_t)(r0 + lane) * n + j0;
                 for (int u = 0; u < kn; ++u) cp_async4(d0 + 4 * u, lsrc + u, 4u);
             }
-            if (!vtma || !lbulk) cp_async_mbar_arrive(&fullB[bs]);
-            // (2) the barrier's one expected arrival, with the bytes of the bulk copies
-            uint32_t tx = vtma ? (uint32_t)(NVBOX * 64 * 128) : 0u;
-            if (lbulk) tx += (uint32_t)(__popc(__ballot_sync(FW_FULL, live_row)) * kn * 4);
+            cp_async_mbar_arrive(&fullB[bs]);
+            // (2) the barrier's one expected arrival, with the bytes of the V boxes
+            const uint32_t tx = vtma ? (uint32_t)(NVBOX * 64 * 128) : 0u;
             __syncwarp();
             if (lane == 0) tc::mbar_arrive_expect_tx(&fullB[bs], tx);
             __syncwarp();
-            // (3) the bulk copies: V boxes by TMA, one logit row per lane
+            // (3) the V boxes by TMA
             if (vtma && lane == 0)
                 for (int h = 0; h < NVBOX; ++h)
                     tc::tma_load_2d(sB + bs * B_SLOT_BYTES + h * (KS * 128), &tmV, 64 * h, (int32_t)(voff / D + j0),
                                     &fullB[bs]);
-            if (lbulk && live_row) tc::bulk_g2s(ldst, lsrc, (uint32_t)kn * 4u, &fullB[bs]);
             ++issued;
         }
         if (!ok && lane == 0) atomicOr(&s_err, 1);
@@ -869,6 +879,469 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
     }
 }
 
+// ---------------------------------------------------------------------------
+// P.V for small groups (at most 8 rows share V, as under grouped-query
+// attention): the same band-expanded products, transposed,
+//   S^T[dim][(band, row)] = sum_j V[j][dim] P[(band, row)][j],
+// so that the value dimension is the MMA's M (128: the d = 128 dims, or the
+// d = 64 dims and 64 rows of zeros) and the NBB x RT (band, row) pairs its N
+// (16, 32 or 48 columns).  With the (band, row) pairs on M, a group of 4 rows
+// with one budget would fill 8 of the 128 tile rows and the tensor work would
+// be 16 times the useful work; here it is at most 3 split terms x the
+// padding of N, and the kernel streams V at the memory's pace.  The band
+// masses are summed by the producers (compensated, in registers) instead of
+// by a column of ones.  Warp 0 copies (V boxes by TMA, logits by cp.async),
+// warp 1 issues the MMAs, warps 2..5 build P^T (K-major, 128-byte swizzle)
+// and flush the TMEM chunk accumulators, each warp its 32 TMEM lanes (dims).
+constexpr int TN_BS = 4;                 // copy slots (V + logits)
+constexpr int TN_PW = 4;                 // producer / flush warps
+constexpr int TN_NT = (TN_PW + 2) * 32;  // threads
+template <int NB, int RT> __host__ __device__ constexpr int tn_cols() { return ((NB + 1) * RT + 15) / 16 * 16; }
+template <int NB, int RT> __host__ __device__ constexpr uint32_t tn_tcols()
+{
+    return NACC * tn_cols<NB, RT>() <= 32 ? 32u : (NACC * tn_cols<NB, RT>() <= 64 ? 64u : 128u);
+}
+
+template <int D, int NB, int RT>
+__global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__ CUtensorMap tmV, const TcArgs a)
+{
+    constexpr int NBB = NB + 1;                 // bands
+    constexpr int NP = NBB * RT;                // (band, row) pairs
+    constexpr int N = tn_cols<NB, RT>();        // MMA N
+    constexpr int NPROD = TN_PW * 32;
+    constexpr int TPR = NPROD / RT;             // producer threads per row (32 or 16)
+    constexpr int KPTH = KS / TPR;              // keys per producer thread and stage (2 or 4)
+    constexpr int NVBOX = D / 64;               // 64-dim blocks of V
+    constexpr int V_SLOT = 2 * KS * 128;        // two 64-row blocks of the M = 128 operand
+    constexpr int P_TERM = N * 128;             // one split term of P^T: N rows x 64 keys
+    constexpr int P_SLOT = NSPLIT * P_TERM;
+    constexpr uint32_t TCOLS = tn_tcols<NB, RT>();
+    constexpr int NC = D / 8;
+    static_assert(KPTH == 2 || KPTH == 4, "producer layout");
+    static_assert(NP * (D + 1) * 4 <= TN_BS * V_SLOT, "epilogue staging fits the V slots");
+    extern __shared__ uint8_t smraw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~(uintptr_t)1023);
+    uint8_t *sV = sm;                                     // [TN_BS][2][64 keys x 128 B]
+    uint8_t *sP = sV + TN_BS * V_SLOT;                    // [ASLOTS][NSPLIT][N x 128 B]
+    float *sL = reinterpret_cast<float *>(sP + ASLOTS * P_SLOT);  // [TN_BS][RT][64]
+    float *acc = reinterpret_cast<float *>(sV);           // epilogue: [NP][D + 1]
+    __shared__ __align__(8) uint64_t fullB[TN_BS], freeB[TN_BS], fullA[ASLOTS], freeA[ASLOTS], accfree[NACC];
+    __shared__ uint32_t s_taddr;
+    __shared__ int s_err;
+    __shared__ float rowM[RT], rowZi[RT];
+    __shared__ uint32_t rtk[RT][4];
+    __shared__ int32_t rti[RT][4];
+    __shared__ int rok[RT];
+    __shared__ float bmass[RT][5];
+
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int64_t g = blockIdx.x / a.tiles_per_group;
+    const int tile = (int)(blockIdx.x - g * a.tiles_per_group);
+    const int r0 = tile * RT;
+    const int nr = min(RT, a.R.R - r0);
+    const int n = a.R.n[g];
+    const int64_t voff = a.R.v_off[g];
+    const uint16_t *V = reinterpret_cast<const uint16_t *>(a.R.v) + voff;
+    const float *LG = a.R.logits + a.R.logit_off[g];
+    const bool vrows = voff % D == 0;  // the block starts on a whole row of the V tensor map
+    const bool l16 = (n & 3) == 0 && (reinterpret_cast<uintptr_t>(LG) & 15) == 0;
+    const int nst = (n + KS - 1) / KS;
+
+    if (tid < RT) {
+        const int r = tid;
+        rok[r] = 0;
+        if (r < nr) {
+            const int64_t row = g * a.R.R + r0 + r;
+            rok[r] = a.ws.status[row] == FW_OK;
+            rowM[r] = a.ws.M[row];
+            rowZi[r] = 1.f / a.ws.Z[row];
+            for (int b = 0; b < 4; ++b) {
+                rtk[r][b] = b < NB ? a.ws.tk[row * NB + b] : 0u;
+                rti[r][b] = b < NB ? a.ws.ti[row * NB + b] : -1;
+            }
+        }
+        for (int b = 0; b < 5; ++b) bmass[r][b] = 0.f;
+    }
+    if (tid == 0) {
+        s_err = 0;
+        for (int x = 0; x < TN_BS; ++x) {
+            tc::mbar_init(&fullB[x], 1);
+            tc::mbar_init(&freeB[x], TN_PW + 1);
+        }
+        for (int x = 0; x < ASLOTS; ++x) {
+            tc::mbar_init(&fullA[x], TN_PW);
+            tc::mbar_init(&freeA[x], 1);
+        }
+        for (int x = 0; x < NACC; ++x) tc::mbar_init(&accfree[x], TN_PW);
+        tc::mbar_init_fence();
+    }
+    // d = 64: the second 64-row block of every V slot is zero (M = 128 rows)
+    if (NVBOX == 1)
+        for (int e = tid; e < TN_BS * KS * 8; e += TN_NT) {
+            const int slot = e / (KS * 8), q = e % (KS * 8);
+            reinterpret_cast<uint4 *>(sV + slot * V_SLOT + KS * 128)[q] = make_uint4(0u, 0u, 0u, 0u);
+        }
+    // rows of P^T past the NP pairs stay zero in every slot and term
+    for (int e = tid; e < ASLOTS * NSPLIT * N * 8; e += TN_NT) {
+        const int m = (e / 8) % N;
+        if (m >= NP) reinterpret_cast<uint4 *>(sP)[e] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    tc::fence_async_smem();
+    if (wid == 1) tc::tmem_alloc(&s_taddr, TCOLS);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t taddr = s_taddr;
+
+    if (wid == 0) {
+        // ---------------------------------------------------------- copies
+        const uint32_t vbase = tc::smem_u32(sV), lbase = tc::smem_u32(sL);
+        const uint32_t livemask = __ballot_sync(FW_FULL, lane < nr && rok[lane]);
+        int issued = 0;
+        bool ok = true;
+        for (int it = 0; it < nst; ++it) {
+            const int bs = it % TN_BS, j0 = it * KS;
+            if (it >= TN_BS) {
+                if (lane == 0) ok = tc::mbar_wait(&freeB[bs], (uint32_t)((it / TN_BS) - 1) & 1u, WAIT_POLLS);
+                ok = __shfl_sync(FW_FULL, ok, 0);
+                if (!ok) break;
+            }
+            const int kn = min(KS, n - j0);  // keys of this stage
+            const bool vtma = vrows && kn == KS;
+            // (1) the per-thread copies, each lane's tracked by the barrier
+            if (!vtma) {  // V rows past the block's end are zero-filled
+                for (int e = lane; e < KS * NC; e += 32) {
+                    const int kk = e / NC, nc = e % NC;
+                    const int n2 = nc >> 3, c = nc & 7;
+                    const uint32_t dst = vbase + bs * V_SLOT + n2 * (KS * 128) + (kk >> 3) * 1024 +
+                                         (kk & 7) * 128 + ((c ^ (kk & 7)) << 4);
+                    const bool in = kk < kn;
+                    cp_async16(dst, V + (int64_t)(in ? j0 + kk : 0) * D + nc * 8, in ? 16u : 0u);
+                }
+            }
+            if (l16) {  // 16-byte chunks, 16 per row (kn is a multiple of 4)
+                for (int e = lane; e < RT * 16; e += 32) {
+                    const int r = e >> 4, c = e & 15;
+                    const bool cin = c * 4 < kn;
+                    if ((livemask >> r) & 1u)
+                        cp_async16(lbase + (uint32_t)(((bs * RT + r) * KS + c * 4) * 4),
+                                   LG + (int64_t)(r0 + r) * n + j0 + (cin ? c * 4 : 0), cin ? 16u : 0u);
+                }
+            } else {
+                for (int e = lane; e < RT * KS; e += 32) {
+                    const int r = e / KS, u = e % KS;
+                    if (((livemask >> r) & 1u) && u < kn)
+                        cp_async4(lbase + (uint32_t)(((bs * RT + r) * KS + u) * 4), LG + (int64_t)(r0 + r) * n + j0 + u,
+                                  4u);
+                }
+            }
+            cp_async_mbar_arrive(&fullB[bs]);
+            // (2) the barrier's one expected arrival, with the bytes of the V boxes
+            const uint32_t tx = vtma ? (uint32_t)(NVBOX * 64 * 128) : 0u;
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive_expect_tx(&fullB[bs], tx);
+            __syncwarp();
+            // (3) the V boxes by TMA
+            if (vtma && lane == 0)
+                for (int h = 0; h < NVBOX; ++h)
+                    tc::tma_load_2d(sV + bs * V_SLOT + h * (KS * 128), &tmV, 64 * h, (int32_t)(voff / D + j0),
+                                    &fullB[bs]);
+            ++issued;
+        }
+        if (!ok && lane == 0) atomicOr(&s_err, 1);
+        // the copies still in flight land before the CTA moves on
+        if (lane == 0)
+            for (int it = issued - TN_BS < 0 ? 0 : issued - TN_BS; it < issued; ++it)
+                if (!tc::mbar_wait(&fullB[it % TN_BS], (uint32_t)(it / TN_BS) & 1u, WAIT_POLLS)) atomicOr(&s_err, 1);
+        __syncwarp();
+    } else if (wid == 1) {
+        // -------------------------------------------------------------- MMA
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(128, N, true, false);
+            // V^T: MN-major, the two 64-row blocks KS * 128 bytes apart; P^T:
+            // K-major.  Other slots, k-steps and terms differ by an address
+            // offset (>> 4) in the start field, which never carries out of it.
+            const uint64_t ad0 = tc::sdesc_sw128(tc::smem_u32(sV), KS * 128, 1024);
+            const uint64_t bd0 = tc::sdesc_sw128(tc::smem_u32(sP), 16, 1024);
+            bool ok = true;
+            int last = -1;
+            for (int it = 0; it < nst && ok; ++it) {
+                const int bs = it % TN_BS, as = it % ASLOTS;
+                ok = tc::mbar_wait(&fullB[bs], (uint32_t)(it / TN_BS) & 1u, WAIT_POLLS);
+                if (ok) ok = tc::mbar_wait(&fullA[as], (uint32_t)(it / ASLOTS) & 1u, WAIT_POLLS);
+                const int ch = it / CH;
+                if (ok && it % CH == 0 && ch >= NACC)
+                    ok = tc::mbar_wait(&accfree[ch % NACC], (uint32_t)((ch - NACC) / NACC) & 1u, WAIT_POLLS);
+                if (!ok) break;
+                tc::fence_after_sync();
+                const uint32_t dacc = taddr + (uint32_t)((ch % NACC) * N);
+                const bool fresh = it % CH == 0;
+                const uint64_t abs_ = ad0 + (uint64_t)((bs * V_SLOT) >> 4);
+                const uint64_t bas = bd0 + (uint64_t)((as * P_SLOT) >> 4);
+#pragma unroll
+                for (int ks = 0; ks < KS / 16; ++ks) {
+                    const uint64_t ad = abs_ + (uint64_t)((ks * 2048) >> 4);
+#pragma unroll
+                    for (int sp = 0; sp < NSPLIT; ++sp)
+                        tc::mma_bf16(dacc, ad, bas + (uint64_t)((sp * P_TERM + ks * 32) >> 4), idesc,
+                                     !fresh || ks > 0 || sp > 0);
+                }
+                tc::commit(&freeA[as]);
+                tc::commit(&freeB[bs]);
+                last = it;
+            }
+            if (!ok) atomicOr(&s_err, 1);
+            if (last >= 0 && !tc::mbar_wait(&freeA[last % ASLOTS], (uint32_t)(last / ASLOTS) & 1u, WAIT_POLLS))
+                atomicOr(&s_err, 1);
+        }
+        __syncwarp();
+    } else {
+        // --------------------------------------------------------- producers
+        const int ptid = tid - 64;               // 0..NPROD-1
+        const int rr = ptid / TPR;               // row of the tile
+        const int kq = ptid % TPR;               // this thread's KPTH keys of the stage
+        const int kc = kq * KPTH / 8, hk = (kq * KPTH) % 8;  // 8-key chunk and first key in it
+        const int quarter = wid & 3;             // TMEM lanes (dims) this warp flushes
+        const bool fl = quarter < 2 * NVBOX;     // d = 64: lanes 64..127 hold zero rows
+        float racc[N];
+#pragma unroll
+        for (int i = 0; i < N; ++i) racc[i] = 0.f;
+        float ms[NBB], mc[NBB];                  // band masses, compensated
+#pragma unroll
+        for (int b = 0; b < NBB; ++b) ms[b] = mc[b] = 0.f;
+        const bool live = rr < nr && rok[rr];
+        const float Mr = live ? rowM[rr] : 0.f, Zr = live ? rowZi[rr] : 0.f;
+        float xt[NB];
+        int tix[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            const uint32_t tk = live ? rtk[rr][b] : 0u;
+            xt[b] = __uint_as_float((tk & 0x80000000u) ? (tk & 0x7fffffffu) : ~tk);
+            tix[b] = live ? rti[rr][b] : -1;
+        }
+        uint32_t boff[NBB];
+#pragma unroll
+        for (int b = 0; b < NBB; ++b) {
+            const int m = b * RT + rr;
+            boff[b] = (uint32_t)((m >> 3) * 1024 + (m & 7) * 128 + ((kc ^ (m & 7)) << 4) + 2 * hk);
+        }
+        bool ok = true;
+        auto chunk_end = [&](int st) { return st % CH == CH - 1 || st == nst - 1; };
+        auto flush = [&](int st) {
+            tc::fence_after_sync();
+            const int buf = (st / CH) % NACC;
+            if (fl) {
+                const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
+#pragma unroll
+                for (int c0 = 0; c0 < N; c0 += 16) {
+                    float v[16];
+                    tc::ld16(taddr + lanes + (uint32_t)(buf * N + c0), v);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) racc[c0 + i] += v[i];
+                }
+            }
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&accfree[buf]);
+        };
+        for (int it = 0; it < nst; ++it) {
+            const int bs = it % TN_BS, as = it % ASLOTS, j0 = it * KS;
+            if (ok) ok = tc::mbar_wait(&fullB[bs], (uint32_t)(it / TN_BS) & 1u, WAIT_POLLS);
+            // the P^T slot was last read by the MMAs of stage it - ASLOTS
+            if (ok && it >= ASLOTS) ok = tc::mbar_wait(&freeA[as], (uint32_t)((it / ASLOTS) - 1) & 1u, WAIT_POLLS);
+            if (!ok) break;
+            uint8_t *pslot = sP + as * P_SLOT;
+            const float *lr = sL + (bs * RT + rr) * KS + kq * KPTH;
+            float xs[KPTH];
+            if constexpr (KPTH == 4) {
+                const float4 x4 = *reinterpret_cast<const float4 *>(lr);
+                xs[0] = x4.x, xs[1] = x4.y, xs[2] = x4.z, xs[3] = x4.w;
+            } else {
+                const float2 x2 = *reinterpret_cast<const float2 *>(lr);
+                xs[0] = x2.x, xs[1] = x2.y;
+            }
+            float pv[KPTH];
+            uint32_t bdp[KPTH / 2];  // bands of keys 2q, 2q + 1 as 2 x 16 bits
+            bool tie = false;
+#pragma unroll
+            for (int u = 0; u < KPTH; ++u) {
+                const int j = j0 + kq * KPTH + u;
+                const float x = xs[u];
+                pv[u] = (live && j < n) ? __expf(x - Mr) * Zr : 0.f;
+                int bd = 0;
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    bd += x < xt[b];
+                    tie |= x == xt[b];
+                }
+                if (u & 1) bdp[u >> 1] |= (uint32_t)bd << 16;
+                else bdp[u >> 1] = (uint32_t)bd;
+            }
+            if (tie) {  // a key equal to a threshold: its index decides (rare)
+#pragma unroll
+                for (int u = 0; u < KPTH; ++u) {
+                    const int j = j0 + kq * KPTH + u;
+                    const float x = xs[u];
+                    int bd = 0;
+#pragma unroll
+                    for (int b = 0; b < NB; ++b) bd += (x < xt[b]) | ((x == xt[b]) & (j > tix[b]));
+                    const uint32_t sh = (u & 1) ? 16u : 0u;
+                    bdp[u >> 1] = (bdp[u >> 1] & ~(0xffffu << sh)) | ((uint32_t)bd << sh);
+                }
+            }
+            // band masses (Kahan-compensated: up to n / KPTH additions per thread)
+#pragma unroll
+            for (int u = 0; u < KPTH; ++u) {
+                const int bd = (int)((bdp[u >> 1] >> ((u & 1) * 16)) & 0xffffu);
+#pragma unroll
+                for (int b = 0; b < NBB; ++b) {
+                    const float y = (bd == b ? pv[u] : 0.f) - mc[b];
+                    const float t = ms[b] + y;
+                    mc[b] = (t - ms[b]) - y;
+                    ms[b] = t;
+                }
+            }
+            // three bf16 terms per mass, two keys per 32-bit word (key 2q low)
+            uint32_t ph[KPTH / 2], pm[KPTH / 2], pl[KPTH / 2];
+#pragma unroll
+            for (int q = 0; q < KPTH / 2; ++q) {
+                const float a0 = pv[2 * q], a1 = pv[2 * q + 1];
+                ph[q] = cvt_bf16x2(a1, a0);
+                const float e0 = a0 - __uint_as_float(ph[q] << 16), e1 = a1 - __uint_as_float(ph[q] & 0xffff0000u);
+                pm[q] = cvt_bf16x2(e1, e0);
+                const float f0 = e0 - __uint_as_float(pm[q] << 16), f1 = e1 - __uint_as_float(pm[q] & 0xffff0000u);
+                pl[q] = cvt_bf16x2(f1, f0);
+            }
+#pragma unroll
+            for (int b = 0; b < NBB; ++b) {
+                uint32_t wh[KPTH / 2], wm[KPTH / 2], wl[KPTH / 2];
+#pragma unroll
+                for (int q = 0; q < KPTH / 2; ++q) {
+                    const uint32_t msk = __vcmpeq2(bdp[q], (uint32_t)b * 0x00010001u);
+                    wh[q] = ph[q] & msk;
+                    wm[q] = pm[q] & msk;
+                    wl[q] = pl[q] & msk;
+                }
+                uint8_t *dst = pslot + boff[b];
+                if constexpr (KPTH == 4) {
+                    *reinterpret_cast<uint2 *>(dst) = make_uint2(wh[0], wh[1]);
+                    *reinterpret_cast<uint2 *>(dst + P_TERM) = make_uint2(wm[0], wm[1]);
+                    *reinterpret_cast<uint2 *>(dst + 2 * P_TERM) = make_uint2(wl[0], wl[1]);
+                } else {
+                    *reinterpret_cast<uint32_t *>(dst) = wh[0];
+                    *reinterpret_cast<uint32_t *>(dst + P_TERM) = wm[0];
+                    *reinterpret_cast<uint32_t *>(dst + 2 * P_TERM) = wl[0];
+                }
+            }
+            tc::fence_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                tc::mbar_arrive(&fullA[as]);
+                tc::mbar_arrive(&freeB[bs]);  // this warp has read the stage's logits
+            }
+            if (it >= ASLOTS && chunk_end(it - ASLOTS)) flush(it - ASLOTS);
+        }
+        // the last chunks: their MMAs complete before they are read
+        for (int st = nst - ASLOTS < 0 ? 0 : nst - ASLOTS; st < nst && ok; ++st) {
+            ok = tc::mbar_wait(&freeA[st % ASLOTS], (uint32_t)(st / ASLOTS) & 1u, WAIT_POLLS);
+            if (ok && chunk_end(st)) flush(st);
+        }
+        if (!ok && lane == 0) atomicOr(&s_err, 1);
+        // band masses: the TPR threads of a row (a warp, or half of one) combine
+#pragma unroll
+        for (int b = 0; b < NBB; ++b) {
+            float v = ms[b] - mc[b];
+#pragma unroll
+            for (int o = TPR / 2; o >= 1; o >>= 1) v += __shfl_xor_sync(FW_FULL, v, o);
+            if (kq == 0 && rr < RT) bmass[rr][b] = v;
+        }
+        // accumulators -> shared for the per-row epilogue: every MMA has
+        // completed and every copy has landed, so the V slots (which acc
+        // overlays) are idle
+        if (fl) {
+            const int dim = quarter * 32 + lane;
+#pragma unroll
+            for (int m = 0; m < NP; ++m) acc[m * (D + 1) + dim] = racc[m];
+        }
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    if (wid == 1) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(taddr, TCOLS);
+    }
+    if (wid < 2) return;
+    // --------------------------------------------------------------- epilogue
+    const bool failed = s_err != 0;
+    constexpr int CPT = D / 32;
+    for (int r = wid - 2; r < nr; r += TN_PW) {
+        const int64_t row = g * a.R.R + r0 + r;
+        if (failed) {
+            if (lane == 0 && a.out.row_status) a.out.row_status[row] = FW_ERR_TIMEOUT;
+            continue;
+        }
+        if (!rok[r]) continue;
+        float S[NBB][CPT];
+#pragma unroll
+        for (int b = 0; b < NBB; ++b)
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) S[b][t] = acc[(b * RT + r) * (D + 1) + lane + 32 * t];
+        if (a.out.o) {
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) {
+                float o = 0.f;
+#pragma unroll
+                for (int b = 0; b < NBB; ++b) o += S[b][t];
+                a.out.o[row * D + lane + 32 * t] = o;
+            }
+        }
+        for (int b = 0; b < NB; ++b) {
+            const int kb = a.k[row * NB + b];
+            int sb = 0;
+            for (int b2 = 0; b2 < NB; ++b2) {
+                const int k2 = a.k[row * NB + b2];
+                sb += (k2 < kb) || (k2 == kb && b2 < b);
+            }
+            float PA = 0.f, PC = 0.f;
+#pragma unroll
+            for (int q = 0; q < NBB; ++q) {
+                if (q <= sb) PA += bmass[r][q];
+                else PC += bmass[r][q];
+            }
+            float s2 = 0.f;
+            float NAv[CPT];
+#pragma unroll
+            for (int t = 0; t < CPT; ++t) {
+                float NA = 0.f, NCs = 0.f;
+#pragma unroll
+                for (int q = 0; q < NBB; ++q) {
+                    if (q <= sb) NA += S[q][t];
+                    else NCs += S[q][t];
+                }
+                NAv[t] = NA;
+                const float diff = PC * NA - PA * NCs;  // p(A) (m_A - mu)
+                s2 = fmaf(diff, diff, s2);
+            }
+            s2 = warp_sum(s2);
+            if (lane == 0) {
+                const float phi = sqrtf(s2);
+                a.out.gap[row * NB + b] = phi / PA;
+                a.out.dropped[row * NB + b] = PC;
+                if (a.out.phi) a.out.phi[row * NB + b] = phi;
+            }
+            if (a.out.o_kept)
+#pragma unroll
+                for (int t = 0; t < CPT; ++t) a.out.o_kept[(row * NB + b) * D + lane + 32 * t] = NAv[t] / PA;
+        }
+    }
+}
+
+template <int NB, int RT> size_t pv_tn_smem()
+{
+    return 1024 + (size_t)TN_BS * 2 * KS * 128 + (size_t)ASLOTS * NSPLIT * tn_cols<NB, RT>() * 128 +
+           (size_t)TN_BS * RT * KS * 4;
+}
+
 template <int D> size_t pv_tma_smem()
 {
     return 1024 + (size_t)ASLOTS * A_SLOT_BYTES + (size_t)PVM_BS * (D / 64 + 1) * KS * 128 +
@@ -903,6 +1376,25 @@ fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_ou
         a.ws = L;
         a.RT = TM / (nb + 1) < MAXRT ? TM / (nb + 1) : MAXRT;
         a.tiles_per_group = (R.R + a.RT - 1) / a.RT;
+        if (R.R <= 8) {  // small groups: the transposed products
+            const int rt = R.R <= 4 ? 4 : 8;
+            a.RT = rt;
+            a.tiles_per_group = 1;
+            const unsigned grid = (unsigned)R.num_groups;
+            auto launch_tn = [&](auto kernel, size_t smem) -> fw_status {
+                FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+                FW_LAUNCH(kernel, grid, TN_NT, smem, s, mv, a);
+                return FW_OK;
+            };
+#define FW_PV_TN(DD, NN, RR) \
+    if (R.d == DD && nb == NN && rt == RR) return launch_tn(k_long_pv_tn<DD, NN, RR>, pv_tn_smem<NN, RR>());
+#define FW_PV_TN_D(DD) \
+    FW_PV_TN(DD, 1, 4) FW_PV_TN(DD, 2, 4) FW_PV_TN(DD, 3, 4) FW_PV_TN(DD, 4, 4) \
+    FW_PV_TN(DD, 1, 8) FW_PV_TN(DD, 2, 8) FW_PV_TN(DD, 3, 8) FW_PV_TN(DD, 4, 8)
+            FW_PV_TN_D(128) FW_PV_TN_D(64)
+#undef FW_PV_TN_D
+#undef FW_PV_TN
+        }
         const unsigned grid = (unsigned)(R.num_groups * a.tiles_per_group);
         auto launch = [&](auto kernel, size_t smem) -> fw_status {
             FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));

@@ -87,6 +87,23 @@ def test_long_bf16_band_counts(fw, nb, d):
     compare(fw, rows_batch(L, V, k, v_dtype="bf16", R=R))
 
 
+@pytest.mark.parametrize("R,nb,d", [(1, 1, 64), (3, 2, 128), (4, 1, 64), (4, 4, 128), (5, 3, 64), (8, 4, 128),
+                                    (8, 2, 64), (2, 3, 128)])
+def test_long_bf16_small_groups(fw, R, nb, d):
+    # groups of at most 8 rows take the transposed P.V (value dims on the
+    # MMA's M, (band, row) pairs on N); n = 1000 leaves a partial 64-key stage,
+    # n = 1001 also sends the logits through 4-byte copies
+    for n in (1000, 1001, 4096):
+        rng = np.random.default_rng(100 * R + 10 * nb + d + n)
+        G = 5
+        L = (rng.normal(size=(G * R, n)) * rng.uniform(0.3, 3.0, size=(G * R, 1))).astype(np.float32)
+        L[:, 0] += 5.0
+        V = rng.normal(size=(G, n, d)).astype(np.float32)
+        ks = [7, 100, 333, n - 1][:nb]
+        k = np.tile(np.array(ks, np.int32), (G * R, 1))
+        compare(fw, rows_batch(L, V, k, v_dtype="bf16", R=R))
+
+
 def test_mixed_profiles_reduced(fw):
     for b in workloads.mixed_profiles(seed=0, rows_scale=2e-3):
         compare(fw, b)
