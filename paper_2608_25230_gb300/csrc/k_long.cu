@@ -279,69 +279,82 @@ __global__ void __launch_bounds__(LT) k_long_select(const SelArgs a)
 }
 
 // ------------------------------------------------------ linear-bin select
-// Rows of at most SEL_MAX_N keys.  Persistent CTAs walk rows; a row's logits
-// arrive in shared memory by bulk copy.  The k-th largest key of every budget
-// comes from one histogram of SNB linear bins over [min, max] of the row (a
-// monotone map of the float, so the bins split the key order), the bin holding
-// the k-th key, and an exact rank among that bin's keys.  Rows whose threshold
+// Rows of at most SEL_MAX_N keys.  Persistent CTAs walk rows, and a row's
+// logits stay in registers: thread t holds keys 4 (t + NT q) + c (q < VPT / 4,
+// c < 4).  While a row is processed, the CTA's next row arrives in shared
+// memory by bulk copy (rows that are whole 16-byte vectors; others are read
+// from global memory directly), so its HBM time overlaps this row's work.  The k-th largest key of every budget comes
+// from one histogram of SNB linear bins over [min, max] of the row (a monotone
+// map of the float, so the bins split the key order), the bin holding the
+// k-th key, and an exact rank among that bin's keys.  Rows whose threshold
 // bin holds more than SCAP keys (heavy ties) are listed for the radix select,
-// which runs on them after this kernel.
+// which runs on them after this kernel.  (A first version kept the row in
+// shared memory, loaded after the previous row was done, with every pass a
+// shared-memory sweep and a divergent candidate test; it ran at 13 % of HBM
+// bandwidth.)
 constexpr int SEL_MAX_N = 32768;  // longest row of the linear-bin select
 constexpr int SNB = 2048;         // linear bins
-constexpr int SCAP = 1024;        // keys of a threshold bin ranked directly
+constexpr int SCAP = 512;         // keys of a threshold bin ranked directly
+constexpr int WCAP = 64;          // threshold-bin keys one warp gathers
+constexpr uint32_t SEL_CHUNK = 32768;  // bytes per bulk-copy instruction
 constexpr uint32_t SEL_WAIT = 1u << 22;  // polls of a row-copy wait before it gives up
-constexpr uint32_t SEL_CHUNK = 32768;    // bytes per bulk-copy instruction
 
-__device__ __forceinline__ bool row_bulk_ok(const RowsDev &R, int64_t row, int &n, const float *&lg)
-{
-    const int64_t g = row / R.R;
-    const int64_t ri = row - g * R.R;
-    n = R.n[g];
-    const int64_t off = R.logit_off[g] + ri * n;
-    lg = R.logits + off;
-    return (n & 3) == 0 && (reinterpret_cast<uintptr_t>(lg) & 15) == 0;
-}
+template <int NT> __host__ __device__ constexpr int sel_minb() { return NT >= 1024 ? 1 : (NT >= 512 ? 2 : 4); }
 
-template <int NT>
-__global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
+template <int NT, int VPT>
+__global__ void __launch_bounds__(NT, sel_minb<NT>()) k_long_select_reg(const SelArgs a)
 {
-    extern __shared__ __align__(16) float sbuf[];  // [max_n] the row's logits
+    constexpr int NW = NT / 32;
+    constexpr int V4 = VPT / 4;
+    constexpr int BPT = SNB / NT;  // bins per thread in the scan
+    static_assert(SNB % NT == 0 && VPT % 4 == 0, "layout");
     __shared__ uint32_t hist[SNB];
     __shared__ uint32_t ckey[4][SCAP];
     __shared__ int32_t cidx[4][SCAP];
-    __shared__ float red_a[32], red_b[32];
-    __shared__ uint32_t wsum[32];
-    __shared__ int s_tb[4], s_cnt[4], s_ti[4], s_kv[4], s_rem[4], s_bcnt[4], s_err;
+    __shared__ uint32_t wkey[NW][WCAP];  // each warp's hits: order key, index, bin
+    __shared__ int32_t widx[NW][WCAP];
+    __shared__ int16_t wbin[NW][WCAP];
+    __shared__ int wnum[NW], wbud[NW][4];
+    __shared__ float red_a[NW], red_b[NW];
+    __shared__ uint32_t wsum[NW];
+    __shared__ int s_tb[4], s_ti[4], s_kv[4], s_rem[4], s_bcnt[4];
     __shared__ uint32_t s_T[4];
+    __shared__ int s_staged, s_err;
     __shared__ __align__(8) uint64_t full;
-    constexpr int NW = NT / 32;
-    constexpr int BPT = SNB / NT;  // bins per thread in the scan
+    extern __shared__ __align__(16) float sbuf[];  // [max_n] the CTA's next row, by bulk copy
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int nb = a.nb;
+    // the bulk copy of row r into sbuf (thread 0; rows that are not 16-byte
+    // aligned whole vectors are read from global memory instead)
+    auto stage = [&](int64_t r) -> int {
+        if (r >= a.R.rows) return 0;
+        const int64_t g2 = r / a.R.R;
+        const int n2 = a.R.n[g2];
+        const float *lg2 = a.R.logits + a.R.logit_off[g2] + (r - g2 * a.R.R) * n2;
+        if ((n2 & 3) != 0 || (reinterpret_cast<uintptr_t>(lg2) & 15) != 0 || n2 < 1) return 0;
+        const uint32_t bytes = (uint32_t)n2 * 4u;
+        tc::fence_async_smem();
+        tc::mbar_arrive_expect_tx(&full, bytes);
+        for (uint32_t o = 0; o < bytes; o += SEL_CHUNK)
+            tc::bulk_g2s(reinterpret_cast<char *>(sbuf) + o, reinterpret_cast<const char *>(lg2) + o,
+                         bytes - o < SEL_CHUNK ? bytes - o : SEL_CHUNK, &full);
+        return 1;
+    };
     if (tid == 0) {
         tc::mbar_init(&full, 1);
         tc::mbar_init_fence();
         s_err = 0;
+        s_staged = stage(blockIdx.x);
     }
     __syncthreads();
     uint32_t phase = 0;
     int64_t fail_row = -1;
     for (int64_t row = blockIdx.x; row < a.R.rows; row += gridDim.x) {
-        int n;
-        const float *lg;
-        const bool bulk = row_bulk_ok(a.R, row, n, lg);
-        // ---- the row into shared memory; max, min and finiteness on the way
-        if (bulk) {
-            if (tid == 0) {
-                tc::fence_async_smem();
-                const uint32_t bytes = (uint32_t)n * 4u;
-                tc::mbar_arrive_expect_tx(&full, bytes);
-                for (uint32_t o = 0; o < bytes; o += SEL_CHUNK) {
-                    const uint32_t c = bytes - o < SEL_CHUNK ? bytes - o : SEL_CHUNK;
-                    tc::bulk_g2s(reinterpret_cast<char *>(sbuf) + o, reinterpret_cast<const char *>(lg) + o, c,
-                                 &full);
-                }
-            }
+        const int64_t g = row / a.R.R;
+        const int n = a.R.n[g];
+        const float *lg = a.R.logits + a.R.logit_off[g] + (row - g * a.R.R) * n;
+        const bool staged = s_staged != 0;
+        if (staged) {
             if (wid == 0 && !tc::mbar_wait(&full, phase, SEL_WAIT)) s_err = 1;  // (every writer stores 1)
             phase ^= 1u;
             __syncthreads();
@@ -349,39 +362,45 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
                 fail_row = row;
                 break;
             }
-        } else {
-            for (int j = tid; j < n; j += NT) sbuf[j] = lg[j];
-            __syncthreads();
         }
-        // the next row heads for L2 while this one is processed
-        if (tid == 0 && row + gridDim.x < a.R.rows) {
-            int n2;
-            const float *lg2;
-            if (row_bulk_ok(a.R, row + gridDim.x, n2, lg2)) {
-                const uint32_t bytes = (uint32_t)n2 * 4u;
-                for (uint32_t o = 0; o < bytes; o += SEL_CHUNK)
-                    tc::bulk_prefetch_l2(reinterpret_cast<const char *>(lg2) + o,
-                                         bytes - o < SEL_CHUNK ? bytes - o : SEL_CHUNK);
+        // ---- the row into registers (zero past its end)
+        float x[VPT];
+#pragma unroll
+        for (int q = 0; q < V4; ++q) {
+            const int j0 = 4 * (tid + NT * q);
+            if (staged) {
+                float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (j0 < n) v = reinterpret_cast<const float4 *>(sbuf)[tid + NT * q];
+                x[4 * q] = v.x, x[4 * q + 1] = v.y, x[4 * q + 2] = v.z, x[4 * q + 3] = v.w;
+            } else {
+#pragma unroll
+                for (int c = 0; c < 4; ++c) x[4 * q + c] = j0 + c < n ? __ldg(lg + j0 + c) : 0.f;
             }
         }
-        // f(j, x) for every key, four per shared-memory load
+        __syncthreads();  // sbuf is read and s_staged consumed: the next row may land
+        if (tid == 0) s_staged = stage(row + gridDim.x);
+        // f(j, x) for every key of the row; a vector slot q is whole when all
+        // threads' keys in it are inside the row (uniform test)
         auto for_keys = [&](auto &&f) {
-            const int n4 = n >> 2;
-            for (int q = tid; q < n4; q += NT) {
-                const float4 v = reinterpret_cast<const float4 *>(sbuf)[q];
-                f(4 * q, v.x);
-                f(4 * q + 1, v.y);
-                f(4 * q + 2, v.z);
-                f(4 * q + 3, v.w);
+#pragma unroll
+            for (int q = 0; q < V4; ++q) {
+                const int j0 = 4 * (tid + NT * q);
+                if (4 * NT * (q + 1) <= n) {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) f(j0 + c, x[4 * q + c]);
+                } else if (4 * NT * q < n) {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        if (j0 + c < n) f(j0 + c, x[4 * q + c]);
+                }
             }
-            for (int j = 4 * n4 + tid; j < n; j += NT) f(j, sbuf[j]);
         };
         float m = -INFINITY, mn = INFINITY;
         bool nan = false;
-        for_keys([&](int, float x) {
-            nan |= x != x;
-            m = fmaxf(m, x);
-            mn = fminf(mn, x);
+        for_keys([&](int, float v) {
+            nan |= v != v;
+            m = fmaxf(m, v);
+            mn = fminf(mn, v);
         });
         m = warp_max(m);
         mn = warp_min(mn);
@@ -390,15 +409,10 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
             red_b[wid] = mn;
         }
         for (int i = tid; i < SNB; i += NT) hist[i] = 0u;
-        if (tid < 4) s_cnt[tid] = 0;
         if (tid < nb) s_kv[tid] = a.k[row * nb + tid];
         bool bad = __syncthreads_or(nan) || n < 1;
-        m = red_a[0];
-        mn = red_b[0];
-        for (int w = 1; w < NW; ++w) {
-            m = fmaxf(m, red_a[w]);
-            mn = fminf(mn, red_b[w]);
-        }
+        m = warp_max(lane < NW ? red_a[lane] : -INFINITY);  // (every warp, every lane: the same)
+        mn = warp_min(lane < NW ? red_b[lane] : INFINITY);
         bad |= !isfinite(m) || !isfinite(mn);  // (an infinite key is the max or the min)
         int status = bad ? FW_ERR_NONFINITE : FW_OK;
         for (int b = 0; b < nb; ++b) {
@@ -413,17 +427,16 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
         auto bin_of = [&](float v) { return (int)fminf((v * 0.5f - hmn) * scl, (float)(SNB - 1)); };
         float se = 0.f;
         if (status == FW_OK) {
-            for_keys([&](int, float x) {
-                se += __expf(x - m);
-                atomicAdd(&hist[bin_of(x)], 1u);
+            for_keys([&](int, float v) {
+                se += __expf(v - m);
+                atomicAdd(&hist[bin_of(v)], 1u);
             });
         }
         se = warp_sum(se);
         __syncthreads();  // red_a reads above are done
         if (lane == 0) red_a[wid] = se;
         __syncthreads();
-        float Z = 0.f;
-        for (int w = 0; w < NW; ++w) Z += red_a[w];
+        const float Z = warp_sum(lane < NW ? red_a[lane] : 0.f);
         if (tid == 0) {
             a.ws.M[row] = m;
             a.ws.Z[row] = Z;
@@ -432,7 +445,10 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
             if (a.out.row_sum) a.out.row_sum[row] = Z;
             if (a.out.row_status) a.out.row_status[row] = status;
         }
-        if (status != FW_OK) continue;  // (uniform)
+        if (status != FW_OK) {  // (uniform)
+            __syncthreads();
+            continue;
+        }
         // ---- keys above each bin (bins from the top), the bin of each budget's k-th key
         uint32_t hv[BPT], loc = 0;
 #pragma unroll
@@ -448,8 +464,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
         }
         if (lane == 31) wsum[wid] = inc;
         __syncthreads();
-        uint32_t above = inc - loc;
-        for (int w = 0; w < wid; ++w) above += wsum[w];
+        uint32_t above = inc - loc + __reduce_add_sync(FW_FULL, lane < wid ? wsum[lane] : 0u);
 #pragma unroll
         for (int i = 0; i < BPT; ++i) {
             const int bn = SNB - 1 - (tid * BPT + i);
@@ -473,54 +488,110 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
             __syncthreads();
             continue;
         }
-        // ---- the threshold bins' keys, then their exact ranks
-        int gb[4], glo = SNB, ghi = -1;
+        // ---- the threshold bins' keys.  Each warp gathers its hits in its own
+        // buffer (ballot offsets, no atomics: the hits are sparse, and
+        // same-address shared atomics from many warps serialise), then the
+        // buffers are concatenated per budget.
+        int gb[4];
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            gb[b] = b < nb ? s_tb[b] : -1;
-            if (b < nb) {
-                glo = min(glo, gb[b]);
-                ghi = max(ghi, gb[b]);
-            }
-        }
-        for_keys([&](int j, float x) {
-            const int bn = bin_of(x);
-            if (bn < glo || bn > ghi) return;
-#pragma unroll
-            for (int b = 0; b < 4; ++b)
-                if (bn == gb[b]) {
-                    const int p = atomicAdd(&s_cnt[b], 1);
-                    ckey[b][p] = order_key(x);
-                    cidx[b][p] = j;
-                }
-        });
-        __syncthreads();
-        // thread t ranks candidate t mod 256 (and every 256th after it) of
-        // budget t / 256, so the budgets' ranks run side by side
+        for (int b = 0; b < 4; ++b) gb[b] = b < nb ? s_tb[b] : -1;
         {
-            constexpr int CPB = NT / 4;  // threads per budget
-            const int b = tid / CPB;
-            if (b < nb) {
-                const int cb = s_bcnt[b];
-                const int want = s_rem[b] - 1;
-                for (int c = tid % CPB; c < cb; c += CPB) {
-                    const uint32_t kc = ckey[b][c];
-                    const int ic = cidx[b][c];
-                    int r = 0;
-#pragma unroll 4
-                    for (int c2 = 0; c2 < cb; ++c2) {
-                        const uint32_t k2 = ckey[b][c2];
-                        r += k2 > kc || (k2 == kc && cidx[b][c2] < ic);
+            int wc = 0;                 // this warp's hits (uniform)
+            int bc[4] = {0, 0, 0, 0};   // ... per budget
+            const uint32_t lt = (1u << lane) - 1u;
+#pragma unroll
+            for (int q = 0; q < V4; ++q) {
+                if (4 * NT * q >= n) break;  // (uniform)
+                const int j0 = 4 * (tid + NT * q);
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    const float v = x[4 * q + c];
+                    const int bn = bin_of(v);
+                    const bool in = j0 + c < n;
+                    bool h[4];
+#pragma unroll
+                    for (int b = 0; b < 4; ++b) h[b] = in && bn == gb[b];
+                    const bool hit = h[0] | h[1] | h[2] | h[3];
+                    const uint32_t mk = __ballot_sync(FW_FULL, hit);
+                    if (mk) {
+                        const int pos = wc + __popc(mk & lt);
+                        if (hit && pos < WCAP) {
+                            wkey[wid][pos] = order_key(v);
+                            widx[wid][pos] = j0 + c;
+                            wbin[wid][pos] = (int16_t)bn;
+                        }
+                        wc += __popc(mk);
+#pragma unroll
+                        for (int b = 0; b < 4; ++b) bc[b] += __popc(__ballot_sync(FW_FULL, h[b]));
                     }
-                    if (r == want) {
-                        s_T[b] = kc;
-                        s_ti[b] = ic;
+                }
+            }
+            if (lane == 0) {
+                wnum[wid] = wc;
+#pragma unroll
+                for (int b = 0; b < 4; ++b) wbud[wid][b] = bc[b];
+            }
+        }
+        __syncthreads();
+        // a warp with more hits than its buffer holds (keys of a threshold bin
+        // bunched in one warp's stretch) leaves the row to the radix select
+        if (__syncthreads_or(tid < NW && wnum[tid] > WCAP)) {
+            if (tid == 0) a.redo_list[atomicAdd(a.redo_count, 1)] = (int32_t)row;
+            __syncthreads();
+            continue;
+        }
+        {
+            const uint32_t lt = (1u << lane) - 1u;
+            int off[4], run[4];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                off[b] = (int)__reduce_add_sync(FW_FULL, lane < wid ? (uint32_t)wbud[lane][b] : 0u);  // (NW <= 32)
+                run[b] = 0;
+            }
+            const int nw_ = wnum[wid];
+            for (int e0 = 0; e0 < nw_; e0 += 32) {
+                const int e = e0 + lane;
+                const int bn = e < nw_ ? wbin[wid][e] : -2;
+#pragma unroll
+                for (int b = 0; b < 4; ++b) {
+                    const bool mt = bn == gb[b];
+                    const uint32_t bm = __ballot_sync(FW_FULL, mt);
+                    const int p = off[b] + run[b] + __popc(bm & lt);
+                    if (mt && p < SCAP) {  // (p < s_bcnt[b] <= SCAP: the bins match the histogram's)
+                        ckey[b][p] = wkey[wid][e];
+                        cidx[b][p] = widx[wid][e];
                     }
+                    run[b] += __popc(bm);
                 }
             }
         }
         __syncthreads();
-        // ---- thresholds and kept bits (a warp per 32 consecutive keys)
+        // the exact rank of every candidate among its budget's, a warp per
+        // candidate (lanes split the comparisons)
+        {
+            const int p1 = s_bcnt[0], p2 = p1 + (nb > 1 ? s_bcnt[1] : 0), p3 = p2 + (nb > 2 ? s_bcnt[2] : 0),
+                      p4 = p3 + (nb > 3 ? s_bcnt[3] : 0);
+            for (int t = wid; t < p4; t += NW) {
+                const int b = (t >= p1) + (t >= p2) + (t >= p3);
+                const int base = b == 0 ? 0 : (b == 1 ? p1 : (b == 2 ? p2 : p3));
+                const int cb = s_bcnt[b];
+                const int c = t - base;
+                const uint32_t kc = ckey[b][c];
+                const int ic = cidx[b][c];
+                uint32_t r = 0;
+                for (int c2 = lane; c2 < cb; c2 += 32) {
+                    const uint32_t k2 = ckey[b][c2];
+                    r += k2 > kc || (k2 == kc && cidx[b][c2] < ic);
+                }
+                r = __reduce_add_sync(FW_FULL, r);
+                if (lane == 0 && (int)r == s_rem[b] - 1) {
+                    s_T[b] = kc;
+                    s_ti[b] = ic;
+                }
+            }
+        }
+        __syncthreads();
+        // ---- thresholds and kept bits
         if (tid < nb) {
             a.ws.tk[row * nb + tid] = s_T[tid];
             a.ws.ti[row * nb + tid] = s_ti[tid];
@@ -528,23 +599,31 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
             if (a.out.thr_idx) a.out.thr_idx[row * nb + tid] = s_ti[tid];
         }
         if (a.out.kept_bits) {
-            // keys strictly above each threshold by one compare and a ballot; the
-            // keys equal to it (all in its bin, so among the candidates) up to
-            // the tie index are added after
+            // keys strictly above each threshold by one compare; a warp's 4 keys
+            // per lane in slot q are 128 consecutive keys, so the 8 lanes of an
+            // octet make one 32-bit word.  The keys equal to the threshold (all
+            // in its bin, so among the candidates) up to the tie index are
+            // added after.
             const int nw = a.out.kept_words;
             float xt[4];
 #pragma unroll
             for (int b = 0; b < 4; ++b) xt[b] = b < nb ? key_float(s_T[b]) : INFINITY;
-            for (int w = wid; w < nw; w += NW) {
-                const int j = w * 32 + lane;
-                const float x = j < n ? sbuf[j] : -INFINITY;
-                uint32_t mine = 0u;  // lane b keeps budget b's word
+#pragma unroll
+            for (int q = 0; q < V4; ++q) {
+                const int j0 = 4 * (tid + NT * q);
+                const int w = j0 >> 5;
 #pragma unroll
                 for (int b = 0; b < 4; ++b) {
-                    const uint32_t word = __ballot_sync(FW_FULL, x > xt[b]);
-                    if (lane == b) mine = word;
+                    if (b >= nb) break;
+                    uint32_t bits = 0u;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) bits |= (uint32_t)(j0 + c < n && x[4 * q + c] > xt[b]) << c;
+                    bits <<= (j0 & 31);
+                    bits |= __shfl_xor_sync(FW_FULL, bits, 1);
+                    bits |= __shfl_xor_sync(FW_FULL, bits, 2);
+                    bits |= __shfl_xor_sync(FW_FULL, bits, 4);
+                    if ((lane & 7) == 0 && w < nw) a.out.kept_bits[(row * nb + b) * (int64_t)nw + w] = bits;
                 }
-                if (lane < nb) a.out.kept_bits[(row * nb + lane) * (int64_t)nw + w] = mine;
             }
             __syncthreads();  // the words above are visible to the block
             constexpr int CPB = NT / 4;
@@ -559,7 +638,7 @@ __global__ void __launch_bounds__(NT, 1) k_long_select_bins(const SelArgs a)
                 }
             }
         }
-        __syncthreads();  // sbuf, s_T, s_ti, hist and candidates are reused by the next row
+        __syncthreads();  // s_T, s_ti, hist and candidates are reused by the next row
     }
     if (fail_row >= 0 && tid == 0) {
         // a row copy did not arrive in time: after a last bounded wait for it,
@@ -775,8 +854,12 @@ fw_status long_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out 
             FW_LAUNCH(kernel, (unsigned)grid, nt, smem, s, sa);
             return FW_OK;
         };
-        const fw_status st = R.max_n <= 8192 ? launch(k_long_select_bins<512>, 512)
-                                              : launch(k_long_select_bins<1024>, 1024);
+        const fw_status st = R.max_n <= 1024    ? launch(k_long_select_reg<256, 4>, 256)
+                             : R.max_n <= 2048  ? launch(k_long_select_reg<256, 8>, 256)
+                             : R.max_n <= 4096  ? launch(k_long_select_reg<256, 16>, 256)
+                             : R.max_n <= 8192  ? launch(k_long_select_reg<512, 16>, 512)
+                             : R.max_n <= 16384 ? launch(k_long_select_reg<512, 32>, 512)
+                                                : launch(k_long_select_reg<1024, 32>, 1024);
         if (st != FW_OK) return st;
         // the listed rows (crowded threshold bins) by the radix select
         const size_t smem = (size_t)R.max_n * 4;
