@@ -450,7 +450,7 @@ def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
                 group_vote=dict(path="fw_group_vote: one set per KV head by summed mass, all rows scored",
                                 ms_per_call=ms_vote, rows_per_s=R / (ms_vote * 1e-3),
                                 roofline=roofline("hbm", vach, peaks["hbm_gbs"], "GB/s", traffic_of("group_vote", R),
-                                                  kernel="k_vote_mass + k_vote_select + k_vote_eval",
+                                                  kernel="k_vote_mass + k_vote_select + k_long_pv_tma (vote mode: tcgen05 band-masked P.V)",
                                                   algorithmic_bytes=vbytes)))
 
 

@@ -46,6 +46,13 @@ struct LongWs {
 bool long_pv_tc_supported(const RowsDev &R, int nb);
 fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, const LongWs &L,
                      cudaStream_t s);
+// The group vote's scoring on the same tensor-core kernels: every row of a
+// group against the group's nested sets (key j kept by budget b when
+// key(mass_j) > thr[b], or equal and j <= tidx[b]); writes gap, dropped and
+// row_status.  FW_ERR_UNSUPPORTED when the rows do not fit them.
+fw_status long_pv_vote(const RowsDev &R, int nb, const float *M, const float *Z, const float *mass,
+                       int64_t mass_stride, const uint32_t *thr, const int32_t *tidx, const int32_t *s_budget,
+                       const int32_t *gflag, float *gap, float *dropped, int32_t *row_status, cudaStream_t s);
 size_t long_gap_workspace(const RowsDev &R, int nb);
 fw_status long_gap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, void *ws,
                    size_t ws_bytes, cudaStream_t s);

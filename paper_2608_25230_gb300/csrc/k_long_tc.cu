@@ -20,7 +20,9 @@
 // it into fp32 registers with round-to-nearest two stages after the chunk ends,
 // when its MMAs have long completed, so that no producer ever waits on the MMAs
 // it has just enabled.  The epilogue combines
-// the bands exactly as the CUDA-core kernel does:
+// the bands exactly as the CUDA-core kernel does (the TMA-fed kernels below
+// also serve the group vote, whose bands come from the group's summed masses
+// and shared thresholds instead of each row's own):
 //   N_A = sum of the bands inside A, N_{A^c} = the rest,
 //   p(A) (m_A - mu) = pbar(A) N_A - p(A) N_{A^c}.
 #include <cuda_bf16.h>
@@ -54,6 +56,15 @@ struct TcArgs {
     LongWs ws;
     int tiles_per_group;
     int RT;
+    // the group vote (vmass != NULL): one kept set per group, key j kept by
+    // budget b when key(G_j) > vthr[b] or (key(G_j) == vthr[b] and j <= vtidx[b]);
+    // the budgets are vs (per group), ws.M / ws.Z the rows' softmax statistics
+    const float *vmass;     // [groups][vmstride] summed masses G
+    int64_t vmstride;
+    const uint32_t *vthr;   // [groups][nb]
+    const int32_t *vtidx;   // [groups][nb] (-1: budget out of range)
+    const int32_t *vs;      // [groups][nb]
+    const int32_t *vgflag;  // [groups] nonzero: a logit of the group is not finite
 };
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes)
@@ -493,6 +504,7 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
     uint8_t *sA = sm;                                     // [ASLOTS][NSPLIT][TM x 128 B]
     uint8_t *sB = sA + ASLOTS * A_SLOT_BYTES;             // [PVM_BS][NG][64 keys x 128 B]
     float *sL = reinterpret_cast<float *>(sB + PVM_BS * B_SLOT_BYTES);  // [PVM_BS][32][64]
+    float *sG = sL + PVM_BS * MAXRT * KS;                 // [PVM_BS][64] the vote's G
     float *acc = reinterpret_cast<float *>(sA);           // epilogue: [TM][D + 1]
     __shared__ __align__(8) uint64_t fullB[PVM_BS], freeB[PVM_BS], fullA[ASLOTS], freeA[ASLOTS], accfree[NACC];
     __shared__ uint32_t s_taddr;
@@ -502,6 +514,9 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
     __shared__ int32_t rti[MAXRT][4];
     __shared__ int rok[MAXRT];
     __shared__ float bmass[MAXRT][5];
+    __shared__ uint32_t vT[4];   // the vote's thresholds, budgets ascending
+    __shared__ int32_t vL[4];
+    __shared__ int rstat[MAXRT];
 
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int64_t g = blockIdx.x / a.tiles_per_group;
@@ -512,6 +527,8 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
     const int64_t voff = a.R.v_off[g];
     const uint16_t *V = reinterpret_cast<const uint16_t *>(a.R.v) + voff;
     const float *LG = a.R.logits + a.R.logit_off[g];
+    const bool vote = a.vmass != nullptr;
+    const float *GB = vote ? a.vmass + g * a.vmstride : nullptr;
     const bool vrows = voff % D == 0;  // the block starts on a whole row of the V tensor map
     const bool lbulk = (n & 3) == 0 && (reinterpret_cast<uintptr_t>(LG) & 15) == 0;
     const int nst = (n + KS - 1) / KS;
@@ -521,15 +538,39 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
         rok[r] = 0;
         if (r < nr) {
             const int64_t row = g * a.R.R + r0 + r;
-            rok[r] = a.ws.status[row] == FW_OK;
+            if (vote) {
+                bool inv = false;
+                for (int b = 0; b < NB; ++b) inv |= a.vtidx[g * NB + b] < 0;
+                rstat[r] = a.vgflag[g] ? FW_ERR_NONFINITE : (inv ? FW_ERR_INVALID_ARG : FW_OK);
+                rok[r] = rstat[r] == FW_OK;
+            } else {
+                rok[r] = a.ws.status[row] == FW_OK;
+            }
             rowM[r] = a.ws.M[row];
             rowZi[r] = 1.f / a.ws.Z[row];
             for (int b = 0; b < 4; ++b) {
-                rtk[r][b] = b < NB ? a.ws.tk[row * NB + b] : 0u;
-                rti[r][b] = b < NB ? a.ws.ti[row * NB + b] : -1;
+                rtk[r][b] = b < NB && !vote ? a.ws.tk[row * NB + b] : 0u;
+                rti[r][b] = b < NB && !vote ? a.ws.ti[row * NB + b] : -1;
             }
         }
         for (int b = 0; b < 5; ++b) bmass[r][b] = 0.f;
+    }
+    if (vote && tid == MAXRT) {  // the group's budgets in ascending order (the sets are nested along it)
+        int sv[4], ov[4];
+        for (int b = 0; b < 4; ++b) {
+            sv[b] = b < NB ? a.vs[g * NB + b] : 0x7fffffff;
+            ov[b] = b;
+        }
+        for (int x = 1; x < NB; ++x)
+            for (int y = x; y > 0 && sv[y] < sv[y - 1]; --y) {
+                const int t1 = sv[y], t2 = ov[y];
+                sv[y] = sv[y - 1], ov[y] = ov[y - 1];
+                sv[y - 1] = t1, ov[y - 1] = t2;
+            }
+        for (int b = 0; b < 4; ++b) {
+            vT[b] = b < NB ? a.vthr[g * NB + ov[b]] : 0u;
+            vL[b] = b < NB ? a.vtidx[g * NB + ov[b]] : -1;
+        }
     }
     if (tid == 0) {
         s_err = 0;
@@ -605,6 +646,9 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
                 const float *lsrc = LG + (int64_t)(r0 + lane) * n + j0;
                 for (int u = 0; u < kn; ++u) cp_async4(d0 + 4 * u, lsrc + u, 4u);
             }
+            if (vote)  // the stage's summed masses (zero past the row)
+                for (int e = lane; e < KS; e += 32)
+                    cp_async4(tc::smem_u32(sG + bs * KS + e), GB + j0 + (e < kn ? e : 0), e < kn ? 4u : 0u);
             cp_async_mbar_arrive(&fullB[bs]);
             // (2) the barrier's one expected arrival, with the bytes of the V boxes
             const uint32_t tx = vtma ? (uint32_t)(NVBOX * 64 * 128) : 0u;
@@ -733,10 +777,16 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
                     const float x = xs[u];
                     pv[u] = (live && j < n) ? __expf(x - Mr) * Zr : 0.f;
                     int bd = 0;
+                    if (vote) {
+                        const uint32_t gk = order_key(sG[bs * KS + kq * KPTH + u]);
 #pragma unroll
-                    for (int b = 0; b < NB; ++b) {
-                        bd += x < xt[b];
-                        tie |= x == xt[b];
+                        for (int b = 0; b < NB; ++b) bd += !(gk > vT[b] || (gk == vT[b] && j <= vL[b]));
+                    } else {
+#pragma unroll
+                        for (int b = 0; b < NB; ++b) {
+                            bd += x < xt[b];
+                            tie |= x == xt[b];
+                        }
                     }
                     if (u & 1) bdp[u >> 1] |= (uint32_t)bd << 16;
                     else bdp[u >> 1] = (uint32_t)bd;
@@ -823,7 +873,14 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
             if (lane == 0 && a.out.row_status) a.out.row_status[row] = FW_ERR_TIMEOUT;
             continue;
         }
-        if (!rok[r]) continue;
+        if (vote && lane == 0 && a.out.row_status) a.out.row_status[row] = rstat[r];
+        if (!rok[r]) {
+            if (vote && lane < NB) {  // no set to score
+                a.out.gap[row * NB + lane] = __int_as_float(0x7fc00000);
+                if (a.out.dropped) a.out.dropped[row * NB + lane] = __int_as_float(0x7fc00000);
+            }
+            continue;
+        }
         float S[NBB][CPT];
 #pragma unroll
         for (int b = 0; b < NBB; ++b)
@@ -839,10 +896,10 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
             }
         }
         for (int b = 0; b < NB; ++b) {
-            const int kb = a.k[row * NB + b];
+            const int kb = vote ? a.vs[g * NB + b] : a.k[row * NB + b];
             int sb = 0;
             for (int b2 = 0; b2 < NB; ++b2) {
-                const int k2 = a.k[row * NB + b2];
+                const int k2 = vote ? a.vs[g * NB + b2] : a.k[row * NB + b2];
                 sb += (k2 < kb) || (k2 == kb && b2 < b);
             }
             float PA = 0.f, PC = 0.f;
@@ -869,7 +926,7 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
             if (lane == 0) {
                 const float phi = sqrtf(s2);
                 a.out.gap[row * NB + b] = phi / PA;
-                a.out.dropped[row * NB + b] = PC;
+                if (a.out.dropped) a.out.dropped[row * NB + b] = PC;
                 if (a.out.phi) a.out.phi[row * NB + b] = phi;
             }
             if (a.out.o_kept)
@@ -924,6 +981,7 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
     uint8_t *sV = sm;                                     // [TN_BS][2][64 keys x 128 B]
     uint8_t *sP = sV + TN_BS * V_SLOT;                    // [ASLOTS][NSPLIT][N x 128 B]
     float *sL = reinterpret_cast<float *>(sP + ASLOTS * P_SLOT);  // [TN_BS][RT][64]
+    float *sG = sL + TN_BS * RT * KS;                     // [TN_BS][64] the vote's G
     float *acc = reinterpret_cast<float *>(sV);           // epilogue: [NP][D + 1]
     __shared__ __align__(8) uint64_t fullB[TN_BS], freeB[TN_BS], fullA[ASLOTS], freeA[ASLOTS], accfree[NACC];
     __shared__ uint32_t s_taddr;
@@ -933,6 +991,9 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
     __shared__ int32_t rti[RT][4];
     __shared__ int rok[RT];
     __shared__ float bmass[RT][5];
+    __shared__ uint32_t vT[4];   // the vote's thresholds, budgets ascending
+    __shared__ int32_t vL[4];
+    __shared__ int rstat[RT];
 
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int64_t g = blockIdx.x / a.tiles_per_group;
@@ -943,6 +1004,8 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
     const int64_t voff = a.R.v_off[g];
     const uint16_t *V = reinterpret_cast<const uint16_t *>(a.R.v) + voff;
     const float *LG = a.R.logits + a.R.logit_off[g];
+    const bool vote = a.vmass != nullptr;
+    const float *GB = vote ? a.vmass + g * a.vmstride : nullptr;
     const bool vrows = voff % D == 0;  // the block starts on a whole row of the V tensor map
     const bool l16 = (n & 3) == 0 && (reinterpret_cast<uintptr_t>(LG) & 15) == 0;
     const int nst = (n + KS - 1) / KS;
@@ -952,15 +1015,39 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
         rok[r] = 0;
         if (r < nr) {
             const int64_t row = g * a.R.R + r0 + r;
-            rok[r] = a.ws.status[row] == FW_OK;
+            if (vote) {
+                bool inv = false;
+                for (int b = 0; b < NB; ++b) inv |= a.vtidx[g * NB + b] < 0;
+                rstat[r] = a.vgflag[g] ? FW_ERR_NONFINITE : (inv ? FW_ERR_INVALID_ARG : FW_OK);
+                rok[r] = rstat[r] == FW_OK;
+            } else {
+                rok[r] = a.ws.status[row] == FW_OK;
+            }
             rowM[r] = a.ws.M[row];
             rowZi[r] = 1.f / a.ws.Z[row];
             for (int b = 0; b < 4; ++b) {
-                rtk[r][b] = b < NB ? a.ws.tk[row * NB + b] : 0u;
-                rti[r][b] = b < NB ? a.ws.ti[row * NB + b] : -1;
+                rtk[r][b] = b < NB && !vote ? a.ws.tk[row * NB + b] : 0u;
+                rti[r][b] = b < NB && !vote ? a.ws.ti[row * NB + b] : -1;
             }
         }
         for (int b = 0; b < 5; ++b) bmass[r][b] = 0.f;
+    }
+    if (vote && tid == RT) {  // the group's budgets in ascending order (the sets are nested along it)
+        int sv[4], ov[4];
+        for (int b = 0; b < 4; ++b) {
+            sv[b] = b < NB ? a.vs[g * NB + b] : 0x7fffffff;
+            ov[b] = b;
+        }
+        for (int x = 1; x < NB; ++x)
+            for (int y = x; y > 0 && sv[y] < sv[y - 1]; --y) {
+                const int t1 = sv[y], t2 = ov[y];
+                sv[y] = sv[y - 1], ov[y] = ov[y - 1];
+                sv[y - 1] = t1, ov[y - 1] = t2;
+            }
+        for (int b = 0; b < 4; ++b) {
+            vT[b] = b < NB ? a.vthr[g * NB + ov[b]] : 0u;
+            vL[b] = b < NB ? a.vtidx[g * NB + ov[b]] : -1;
+        }
     }
     if (tid == 0) {
         s_err = 0;
@@ -1035,6 +1122,9 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
                                   4u);
                 }
             }
+            if (vote)  // the stage's summed masses (zero past the row)
+                for (int e = lane; e < KS; e += 32)
+                    cp_async4(tc::smem_u32(sG + bs * KS + e), GB + j0 + (e < kn ? e : 0), e < kn ? 4u : 0u);
             cp_async_mbar_arrive(&fullB[bs]);
             // (2) the barrier's one expected arrival, with the bytes of the V boxes
             const uint32_t tx = vtma ? (uint32_t)(NVBOX * 64 * 128) : 0u;
@@ -1169,10 +1259,16 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
                 const float x = xs[u];
                 pv[u] = (live && j < n) ? __expf(x - Mr) * Zr : 0.f;
                 int bd = 0;
+                if (vote) {
+                    const uint32_t gk = order_key(sG[bs * KS + kq * KPTH + u]);
 #pragma unroll
-                for (int b = 0; b < NB; ++b) {
-                    bd += x < xt[b];
-                    tie |= x == xt[b];
+                    for (int b = 0; b < NB; ++b) bd += !(gk > vT[b] || (gk == vT[b] && j <= vL[b]));
+                } else {
+#pragma unroll
+                    for (int b = 0; b < NB; ++b) {
+                        bd += x < xt[b];
+                        tie |= x == xt[b];
+                    }
                 }
                 if (u & 1) bdp[u >> 1] |= (uint32_t)bd << 16;
                 else bdp[u >> 1] = (uint32_t)bd;
@@ -1280,7 +1376,14 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
             if (lane == 0 && a.out.row_status) a.out.row_status[row] = FW_ERR_TIMEOUT;
             continue;
         }
-        if (!rok[r]) continue;
+        if (vote && lane == 0 && a.out.row_status) a.out.row_status[row] = rstat[r];
+        if (!rok[r]) {
+            if (vote && lane < NB) {  // no set to score
+                a.out.gap[row * NB + lane] = __int_as_float(0x7fc00000);
+                if (a.out.dropped) a.out.dropped[row * NB + lane] = __int_as_float(0x7fc00000);
+            }
+            continue;
+        }
         float S[NBB][CPT];
 #pragma unroll
         for (int b = 0; b < NBB; ++b)
@@ -1296,10 +1399,10 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
             }
         }
         for (int b = 0; b < NB; ++b) {
-            const int kb = a.k[row * NB + b];
+            const int kb = vote ? a.vs[g * NB + b] : a.k[row * NB + b];
             int sb = 0;
             for (int b2 = 0; b2 < NB; ++b2) {
-                const int k2 = a.k[row * NB + b2];
+                const int k2 = vote ? a.vs[g * NB + b2] : a.k[row * NB + b2];
                 sb += (k2 < kb) || (k2 == kb && b2 < b);
             }
             float PA = 0.f, PC = 0.f;
@@ -1326,7 +1429,7 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
             if (lane == 0) {
                 const float phi = sqrtf(s2);
                 a.out.gap[row * NB + b] = phi / PA;
-                a.out.dropped[row * NB + b] = PC;
+                if (a.out.dropped) a.out.dropped[row * NB + b] = PC;
                 if (a.out.phi) a.out.phi[row * NB + b] = phi;
             }
             if (a.out.o_kept)
@@ -1339,13 +1442,13 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
 template <int NB, int RT> size_t pv_tn_smem()
 {
     return 1024 + (size_t)TN_BS * 2 * KS * 128 + (size_t)ASLOTS * NSPLIT * tn_cols<NB, RT>() * 128 +
-           (size_t)TN_BS * RT * KS * 4;
+           (size_t)TN_BS * RT * KS * 4 + (size_t)TN_BS * KS * 4;
 }
 
 template <int D> size_t pv_tma_smem()
 {
     return 1024 + (size_t)ASLOTS * A_SLOT_BYTES + (size_t)PVM_BS * (D / 64 + 1) * KS * 128 +
-           (size_t)PVM_BS * MAXRT * KS * 4;
+           (size_t)PVM_BS * MAXRT * KS * 4 + (size_t)PVM_BS * KS * 4;
 }
 
 template <int D> size_t tc_smem(int RT)
@@ -1360,61 +1463,84 @@ bool long_pv_tc_supported(const RowsDev &R, int nb)
     return R.v_dtype == FW_BF16 && (R.d == 64 || R.d == 128) && nb >= 1 && nb <= 4;
 }
 
-fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, const LongWs &L,
-                     cudaStream_t s)
+namespace {
+
+// The TMA-fed kernels (transposed products for groups of at most 8 rows);
+// FW_ERR_UNSUPPORTED when no instantiation fits.
+fw_status launch_pv_tma(TcArgs a, const CUtensorMap &mv, cudaStream_t s)
 {
-    // the copy-warp kernel (TMA for V, bulk copies for logits) when the driver
-    // can encode the V tensor map; the rows of the map are every whole row the
-    // block may address (boxes are only issued inside a group's own block)
-    CUtensorMap mv;
-    if (make_tma_2d_bf16(&mv, R.v, (uint64_t)1 << 31, (uint64_t)R.d, 64)) {
-        TcArgs a;
-        a.R = R;
-        a.k = k;
-        a.nb = nb;
-        a.out = out;
-        a.ws = L;
-        a.RT = TM / (nb + 1) < MAXRT ? TM / (nb + 1) : MAXRT;
-        a.tiles_per_group = (R.R + a.RT - 1) / a.RT;
-        if (R.R <= 8) {  // small groups: the transposed products
-            const int rt = R.R <= 4 ? 4 : 8;
-            a.RT = rt;
-            a.tiles_per_group = 1;
-            const unsigned grid = (unsigned)R.num_groups;
-            auto launch_tn = [&](auto kernel, size_t smem) -> fw_status {
-                FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-                FW_LAUNCH(kernel, grid, TN_NT, smem, s, mv, a);
-                return FW_OK;
-            };
+    const RowsDev &R = a.R;
+    const int nb = a.nb;
+    if (R.R <= 8) {  // small groups: the transposed products
+        const int rt = R.R <= 4 ? 4 : 8;
+        a.RT = rt;
+        a.tiles_per_group = 1;
+        const unsigned grid = (unsigned)R.num_groups;
+        auto launch_tn = [&](auto kernel, size_t smem) -> fw_status {
+            FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+            FW_LAUNCH(kernel, grid, TN_NT, smem, s, mv, a);
+            return FW_OK;
+        };
 #define FW_PV_TN(DD, NN, RR) \
     if (R.d == DD && nb == NN && rt == RR) return launch_tn(k_long_pv_tn<DD, NN, RR>, pv_tn_smem<NN, RR>());
 #define FW_PV_TN_D(DD) \
     FW_PV_TN(DD, 1, 4) FW_PV_TN(DD, 2, 4) FW_PV_TN(DD, 3, 4) FW_PV_TN(DD, 4, 4) \
     FW_PV_TN(DD, 1, 8) FW_PV_TN(DD, 2, 8) FW_PV_TN(DD, 3, 8) FW_PV_TN(DD, 4, 8)
-            FW_PV_TN_D(128) FW_PV_TN_D(64)
+        FW_PV_TN_D(128) FW_PV_TN_D(64)
 #undef FW_PV_TN_D
 #undef FW_PV_TN
-        }
-        const unsigned grid = (unsigned)(R.num_groups * a.tiles_per_group);
-        auto launch = [&](auto kernel, size_t smem) -> fw_status {
-            FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-            FW_LAUNCH(kernel, grid, (R.d == 128 ? pvm_nt<128>() : pvm_nt<64>()), smem, s, mv, a);
-            return FW_OK;
-        };
+        return FW_ERR_UNSUPPORTED;
+    }
+    a.RT = TM / (nb + 1) < MAXRT ? TM / (nb + 1) : MAXRT;
+    a.tiles_per_group = (R.R + a.RT - 1) / a.RT;
+    const unsigned grid = (unsigned)(R.num_groups * a.tiles_per_group);
+    auto launch = [&](auto kernel, size_t smem) -> fw_status {
+        FW_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        FW_LAUNCH(kernel, grid, (R.d == 128 ? pvm_nt<128>() : pvm_nt<64>()), smem, s, mv, a);
+        return FW_OK;
+    };
 #define FW_PV_NB(DD, NN) \
     if (R.d == DD && nb == NN) return launch(k_long_pv_tma<DD, NN>, pv_tma_smem<DD>());
-        FW_PV_NB(128, 1) FW_PV_NB(128, 2) FW_PV_NB(128, 3) FW_PV_NB(128, 4)
-        FW_PV_NB(64, 1) FW_PV_NB(64, 2) FW_PV_NB(64, 3) FW_PV_NB(64, 4)
+    FW_PV_NB(128, 1) FW_PV_NB(128, 2) FW_PV_NB(128, 3) FW_PV_NB(128, 4)
+    FW_PV_NB(64, 1) FW_PV_NB(64, 2) FW_PV_NB(64, 3) FW_PV_NB(64, 4)
 #undef FW_PV_NB
-    }
+    return FW_ERR_UNSUPPORTED;
+}
+
+TcArgs base_args(const RowsDev &R, int nb, const fw_gap_out &out, const LongWs &L)
+{
     TcArgs a;
     a.R = R;
-    a.k = k;
+    a.k = nullptr;
     a.nb = nb;
     a.out = out;
     a.ws = L;
     a.RT = TM / (nb + 1) < MAXRT ? TM / (nb + 1) : MAXRT;
     a.tiles_per_group = (R.R + a.RT - 1) / a.RT;
+    a.vmass = nullptr;
+    a.vmstride = 0;
+    a.vthr = nullptr;
+    a.vtidx = nullptr;
+    a.vs = nullptr;
+    a.vgflag = nullptr;
+    return a;
+}
+
+}  // namespace
+
+fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out &out, const LongWs &L,
+                     cudaStream_t s)
+{
+    TcArgs a = base_args(R, nb, out, L);
+    a.k = k;
+    // the copy-warp kernels (TMA for V) when the driver can encode the V
+    // tensor map; the rows of the map are every whole row the block may
+    // address (boxes are only issued inside a group's own block)
+    CUtensorMap mv;
+    if (make_tma_2d_bf16(&mv, R.v, (uint64_t)1 << 31, (uint64_t)R.d, 64)) {
+        const fw_status st = launch_pv_tma(a, mv, s);
+        if (st != FW_ERR_UNSUPPORTED) return st;
+    }
     const unsigned grid = (unsigned)(R.num_groups * a.tiles_per_group);
     if (R.d == 128) {
         const size_t smem = tc_smem<128>(a.RT);
@@ -1426,6 +1552,30 @@ fw_status long_pv_tc(const RowsDev &R, const int32_t *k, int nb, const fw_gap_ou
         FW_LAUNCH(k_long_pv_tc<64>, grid, pv_threads<64>(), smem, s, a);
     }
     return FW_OK;
+}
+
+fw_status long_pv_vote(const RowsDev &R, int nb, const float *M, const float *Z, const float *mass,
+                       int64_t mass_stride, const uint32_t *thr, const int32_t *tidx, const int32_t *s_budget,
+                       const int32_t *gflag, float *gap, float *dropped, int32_t *row_status, cudaStream_t s)
+{
+    if (!long_pv_tc_supported(R, nb)) return FW_ERR_UNSUPPORTED;
+    fw_gap_out out{};
+    out.gap = gap;
+    out.dropped = dropped;
+    out.row_status = row_status;
+    LongWs L{};
+    L.M = const_cast<float *>(M);
+    L.Z = const_cast<float *>(Z);
+    TcArgs a = base_args(R, nb, out, L);
+    a.vmass = mass;
+    a.vmstride = mass_stride;
+    a.vthr = thr;
+    a.vtidx = tidx;
+    a.vs = s_budget;
+    a.vgflag = gflag;
+    CUtensorMap mv;
+    if (!make_tma_2d_bf16(&mv, R.v, (uint64_t)1 << 31, (uint64_t)R.d, 64)) return FW_ERR_UNSUPPORTED;
+    return launch_pv_tma(a, mv, s);
 }
 
 }  // namespace fw

@@ -21,6 +21,11 @@
 //                  order) that first contains it; members add p_j v_j to their
 //                  band.  Prefix sums over the bands give every budget's m_A,
 //                  suffix sums its dropped mass.
+// For bf16 values with d = 64 or 128 the scoring runs instead on the long-row
+// path's tensor-core P.V kernels in their vote mode (k_long_tc.cu): the rows
+// of a group share V and the nested sets, so the band-masked products of all
+// the group's rows are one contraction, and V is streamed once per tile of
+// rows rather than gathered once per row.
 #include <algorithm>
 #include <climits>
 
@@ -473,6 +478,13 @@ fw_status group_vote(const RowsDev &R, const int32_t *s, int nb, const fw_gap_ou
     FW_CUDA_CHECK(cudaFuncSetAttribute(k_vote_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sel_smem));
     FW_LAUNCH(k_vote_select, (unsigned)std::min<int64_t>(R.num_groups, 1 << 20), VS_T, sel_smem, st, a);
 
+    // bf16 values: the scoring as band-masked P.V products on the tensor cores
+    // (the rows of a group share V and the set); otherwise one warp per row
+    {
+        const fw_status vs = long_pv_vote(R, nb, a.M, a.Z, a.mass, R.max_n, a.thr, a.tidx, a.s, a.gflag, gap,
+                                          dropped, row_status, st);
+        if (vs != FW_ERR_UNSUPPORTED) return vs;
+    }
     const unsigned ge = (unsigned)std::min<int64_t>((R.rows + VE_W - 1) / VE_W, 1 << 24);
     FW_DISPATCH(R.d, R.v_dtype, { FW_LAUNCH((k_vote_eval<DPL, VT>), ge, VE_W * 32, 0, st, a); });
     return FW_OK;
