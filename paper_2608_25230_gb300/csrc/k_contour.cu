@@ -312,31 +312,46 @@ __global__ void __launch_bounds__(1024) k_c_offsets(CArgs a)
     }
 }
 
-// exclusive and total sums over the warps of the values v[w] (w < NW), for
-// every thread of the block
-template <int NW>
-__device__ __forceinline__ void warp_counts(const int *v, int wid, int lane, int &before, int &total)
-{
-    int x = lane < NW ? v[lane] : 0;
-    int inc = x;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(FW_FULL, inc, o);
-        if (lane >= o) inc += y;
-    }
-    before = __shfl_sync(FW_FULL, inc - x, wid);
-    total = __shfl_sync(FW_FULL, inc, 31);
-}
-
 // per cell, positions in order: the ordered compaction of the kept positions,
 // the dropped mass of the allocation, and the cell's own top-uniform_s set
 // (keys above its threshold, then the first equal ones in position order) with
-// the dropped mass outside it
-constexpr int CTE = 1024;  // threads of an emit block
-__global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
+// the dropped mass outside it.  A thread takes EPT consecutive positions of a
+// chunk of CTE * EPT, so a chunk costs two block scans: the tie counts (the
+// global threshold's, the uniform set's and the cap's, packed in one 64-bit
+// word) and the kept counts.
+constexpr int CTE = 512;  // threads of an emit block (two per SM: the cells fit one wave)
+constexpr int EPT = 8;    // positions per thread and chunk
+
+// Exclusive prefix (over the block's threads, in thread order) and total of v.
+template <int NW, typename U>
+__device__ __forceinline__ void block_scan(U v, U *wsum, int wid, int lane, U &before, U &total)
+{
+    U inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const U y = __shfl_up_sync(FW_FULL, inc, o);
+        if (lane >= o) inc += y;
+    }
+    if (lane == 31) wsum[wid] = inc;
+    __syncthreads();
+    const U w = lane < NW ? wsum[lane] : (U)0;
+    U winc = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const U y = __shfl_up_sync(FW_FULL, winc, o);
+        if (lane >= o) winc += y;
+    }
+    before = __shfl_sync(FW_FULL, winc - w, wid) + inc - v;
+    total = __shfl_sync(FW_FULL, winc, 31);
+    __syncthreads();  // wsum is rewritten by the next scan
+}
+
+__global__ void __launch_bounds__(CTE, 2) k_c_emit(CArgs a)
 {
     constexpr int NW = CTE / 32;
-    __shared__ int wc[NW], wt[NW], wu[NW], wk[NW];
+    constexpr int CH = CTE * EPT;  // positions per chunk
+    __shared__ unsigned long long wsum64[NW];
+    __shared__ uint32_t wsum32[NW];
     __shared__ double red[NW], red2[NW], red3[NW];
     const int c = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
@@ -349,73 +364,102 @@ __global__ void __launch_bounds__(CTE) k_c_emit(CArgs a)
     const int cmode = a.capnf < 0 || a.capnf >= a.T - a.F ? 0 : (a.capnf == 0 ? 1 : 2);
     const uint32_t cT = cmode == 2 ? a.cprefix[c] : 0u;
     const int cwant = cmode == 2 ? (int)a.crem[c] : 0;
-    int cties_seen = 0;
     const float *s = a.scores + (int64_t)c * a.T;
-    const uint32_t lmask = (1u << lane) - 1u;
-    int written = 0, ties_seen = 0, uties_seen = 0;
+    const bool vec = (a.T & 3) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0;
+    const int nfe = a.T - a.F;  // positions before the floor
+    int64_t written = 0;
+    int ties_seen = 0, uties_seen = 0, cties_seen = 0;
     // per-thread sums of T / CTE positive terms in fp32 (relative error below
     // 1e-5); the sums over threads in fp64
     float tot = 0.f, drop = 0.f, udrop = 0.f;
-    float xn = tid < a.T ? __ldg(s + tid) : 0.f;  // the next chunk's score, loaded a chunk ahead
-    for (int j0 = 0; j0 < a.T; j0 += CTE) {
-        const int j = j0 + tid;
-        bool kept = false, tie = false, ukept = false, utie = false, ckept = true, ctie = false;
-        const float x = xn;
-        if (j + CTE < a.T) xn = __ldg(s + j + CTE);
-        if (j < a.T) {
-            const uint32_t key = order_key(x);
-            if (j >= a.T - a.F) {
-                kept = true;
-            } else {
-                if (a.K > 0) {
-                    kept = key > tk;
-                    tie = key == tk;
+    auto load4 = [&](int j, float (&x)[EPT]) {
+        if (vec && j + EPT <= a.T) {
+#pragma unroll
+            for (int h = 0; h < EPT; h += 4) {
+                const float4 v = __ldg(reinterpret_cast<const float4 *>(s + j + h));
+                x[h] = v.x, x[h + 1] = v.y, x[h + 2] = v.z, x[h + 3] = v.w;
+            }
+        } else {
+#pragma unroll
+            for (int u = 0; u < EPT; ++u) x[u] = j + u < a.T ? __ldg(s + j + u) : 0.f;
+        }
+    };
+    float xn[EPT];
+    load4(EPT * tid, xn);  // the next chunk's scores, loaded a chunk ahead
+    for (int j0 = 0; j0 < a.T; j0 += CH) {
+        const int jt = j0 + EPT * tid;  // this thread's first position
+        float x[EPT];
+#pragma unroll
+        for (int u = 0; u < EPT; ++u) x[u] = xn[u];
+        if (j0 + CH < a.T) load4(jt + CH, xn);
+        // flags as bit masks (bit u: position jt + u)
+        uint32_t kept = 0u, tie = 0u, ukept = 0u, utie = 0u, ckept = 0u, ctie = 0u;
+#pragma unroll
+        for (int u = 0; u < EPT; ++u) {
+            const int j = jt + u;
+            const uint32_t bit = 1u << u;
+            bool k_ = false, t_ = false, uk_ = false, ut_ = false, ck_ = true, ct_ = false;
+            if (j < a.T) {
+                const uint32_t key = order_key(x[u]);
+                if (j >= nfe) {
+                    k_ = true;
+                } else {
+                    if (a.K > 0) {
+                        k_ = key > tk;
+                        t_ = key == tk;
+                    }
+                    if (cmode == 1) {
+                        ck_ = false;
+                    } else if (cmode == 2) {
+                        ck_ = key > cT;
+                        ct_ = key == cT;
+                    }
                 }
-                if (cmode == 1) {
-                    ckept = false;
-                } else if (cmode == 2) {
-                    ckept = key > cT;
-                    ctie = key == cT;
+                if (uwant > 0) {
+                    uk_ = key > uT;
+                    ut_ = key == uT;
                 }
             }
-            if (uwant > 0) {
-                ukept = key > uT;
-                utie = key == uT;
-            }
+            kept |= k_ ? bit : 0u;
+            tie |= t_ ? bit : 0u;
+            ukept |= uk_ ? bit : 0u;
+            utie |= ut_ ? bit : 0u;
+            ckept |= ck_ ? bit : 0u;
+            ctie |= ct_ ? bit : 0u;
         }
         // ranks of the ties among the cell's ties, in position order
-        const uint32_t tb = __ballot_sync(FW_FULL, tie), ub = __ballot_sync(FW_FULL, utie);
-        const uint32_t cb2 = __ballot_sync(FW_FULL, ctie);
-        if (lane == 0) {
-            wt[wid] = __popc(tb);
-            wu[wid] = __popc(ub);
-            wk[wid] = __popc(cb2);
+        unsigned long long tb, ttot;
+        block_scan<NW>((unsigned long long)__popc(tie) | ((unsigned long long)__popc(utie) << 21) |
+                           ((unsigned long long)__popc(ctie) << 42),
+                       wsum64, wid, lane, tb, ttot);
+        int rt = ties_seen + (int)(tb & 0x1fffffu), ru = uties_seen + (int)((tb >> 21) & 0x1fffffu),
+            rc = cties_seen + (int)(tb >> 42);
+#pragma unroll
+        for (int u = 0; u < EPT; ++u) {
+            const uint32_t bit = 1u << u;
+            if (tie & bit) kept = rt++ < take ? (kept | bit) : (kept & ~bit);
+            if (utie & bit) ukept = ru++ < uwant ? (ukept | bit) : (ukept & ~bit);
+            if (ctie & bit) ckept = rc++ < cwant ? (ckept | bit) : (ckept & ~bit);
         }
-        __syncthreads();
-        int tbefore, ttotal, ubefore, utotal, cbefore, ctotal;
-        warp_counts<NW>(wt, wid, lane, tbefore, ttotal);
-        warp_counts<NW>(wu, wid, lane, ubefore, utotal);
-        warp_counts<NW>(wk, wid, lane, cbefore, ctotal);
-        if (tie) kept = ties_seen + tbefore + __popc(tb & lmask) < take;
-        if (utie) ukept = uties_seen + ubefore + __popc(ub & lmask) < uwant;
-        if (ctie) ckept = cties_seen + cbefore + __popc(cb2 & lmask) < cwant;
-        kept = kept && ckept;
-        ties_seen += ttotal;
-        uties_seen += utotal;
-        cties_seen += ctotal;
-        const uint32_t kb = __ballot_sync(FW_FULL, kept);
-        if (lane == 0) wc[wid] = __popc(kb);
-        __syncthreads();
-        int before, total;
-        warp_counts<NW>(wc, wid, lane, before, total);
-        if (kept) a.kept_pos[base + written + before + __popc(kb & lmask)] = j;
-        written += total;
-        if (j < a.T) {
-            tot += x;
-            if (!kept) drop += x;
-            if (!ukept) udrop += x;
+        kept &= ckept;
+        ties_seen += (int)(ttot & 0x1fffffu);
+        uties_seen += (int)((ttot >> 21) & 0x1fffffu);
+        cties_seen += (int)(ttot >> 42);
+        uint32_t kbef, ktot;
+        block_scan<NW>((uint32_t)__popc(kept), wsum32, wid, lane, kbef, ktot);
+        int64_t w = base + written + kbef;
+#pragma unroll
+        for (int u = 0; u < EPT; ++u) {
+            const int j = jt + u;
+            const uint32_t bit = 1u << u;
+            if (kept & bit) a.kept_pos[w++] = j;
+            if (j < a.T) {
+                tot += x[u];
+                if (!(kept & bit)) drop += x[u];
+                if (!(ukept & bit)) udrop += x[u];
+            }
         }
-        __syncthreads();  // wt, wu, wk, wc are rewritten by the next chunk
+        written += ktot;
     }
     const double tsum = warp_sum_d((double)tot), dsum = warp_sum_d((double)drop), usum = warp_sum_d((double)udrop);
     if (lane == 0) {
