@@ -45,17 +45,29 @@ N_KEYS, K_SEL = 24, 6
 SUBSETS_PER_ROW = math.comb(N_KEYS, K_SEL)
 POOL_SCHED = ((4, 24), (8, 12), (16, 6), (32, 4))  # (s, E): the candidate-set schedule of App. B
 
-# DRAM bytes (read + write) per unit of work, from one-kernel ncu captures on
-# reduced cases (dram__bytes_read.sum + dram__bytes_write.sum; the commands are
-# in profiles/), scaled to a full launch by the units it processes.  None where
-# the kernel changed after its capture.
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, ncu, one pass,
+# cold caches per kernel) per unit of each line, from kernel-filtered captures
+# of reduced cases of the same workloads (the commands are listed with the
+# summaries under profiles/), scaled to a full launch by the units it
+# processes; None where a kernel changed after its capture:
+#   fw_best_subset  the headline path's kernels at --rows-scale 0.1, per row
+#   long_gap        8 heads x 128 rows: per-row logit bytes of k_long_select_reg
+#                   and k_long_pv_tma scaled to 4,096 rows, plus each head's
+#                   value block once (8 x 8.4 MB), per row
+#   group_vote      the same for k_vote_mass + k_vote_select + k_long_pv_tma
+#   contour         64 cells: k_c_* of one allocation + k_compact, per kept row
+#   compact         k_compact alone, per kept row
+#   window_score    k_wscore, per key (it reads K twice)
+#   mixed_gap       --mixed-rows-scale 0.1, one gap call per profile, per row
 TRAFFIC_PER_UNIT = {
-    # kernel: (bytes per unit, unit)
-    "fw_best_subset": None,
-    "long_gap": None,
-    "group_vote": None,
-    "contour": None,
-    "mixed_gap": None,
+    # line: (bytes per unit, unit)
+    "fw_best_subset": (40328.0, "row"),
+    "long_gap": (282648.0, "row"),
+    "group_vote": (280709.0, "row"),
+    "contour": (1023.7, "kept row"),
+    "compact": (831.0, "kept row"),
+    "window_score": (519.2, "key"),
+    "mixed_gap": (322689.0, "row"),
 }
 
 
@@ -454,8 +466,8 @@ def section_long_rows(fw, device, K, W, flush, peaks, rows_per_head=512):
                                                   algorithmic_bytes=vbytes)))
 
 
-def section_contour(fw, device, K, W, flush, peaks):
-    cb = workloads.contour_cache(seed=0, backend="torch", device=device)
+def section_contour(fw, device, K, W, flush, peaks, cells=256):
+    cb = workloads.contour_cache(seed=0, cells=cells, backend="torch", device=device)
     Kc, Vc = cb.K.view(torch.int16), cb.V.view(torch.int16)
     Ko = torch.empty(cb.total_budget, cb.d, dtype=torch.int16, device=device)
     Vo = torch.empty_like(Ko)
@@ -517,24 +529,26 @@ def section_contour(fw, device, K, W, flush, peaks):
     nbytes = cb.cells * cb.T * 4 + 2 * 2 * cb.total_budget * cb.d * 2 + cb.total_budget * 4 + (cb.cells + 1) * 8
     ach = nbytes / (ms * 1e-3) / 1e9
     cbytes = 2 * 2 * cb.total_budget * cb.d * 2
-    return dict(workload="contour_cache: 256 cells x 32768 tokens, d=128 bf16 K/V, budget 1/8, floor 32",
+    return dict(workload=f"contour_cache: {cb.cells} cells x 32768 tokens, d=128 bf16 K/V, budget 1/8, floor 32",
                 path="a7-a8 (fw_contour_alloc + fw_ragged_compact)", metric="kept KV rows/s",
                 value=cb.total_budget / (ms * 1e-3), ms_per_step=ms, ms_alloc=ms_alloc, ms_compact=ms_comp,
                 roofline=roofline("hbm", ach, peaks["hbm_gbs"], "GB/s", traffic_of("contour", cb.total_budget),
                                   algorithmic_bytes=nbytes, kernel="k_c_* + k_compact"),
                 compact_roofline=roofline("hbm", cbytes / (ms_comp * 1e-3) / 1e9, peaks["hbm_gbs"], "GB/s",
-                                          kernel="k_compact", algorithmic_bytes=cbytes),
+                                          traffic_of("compact", cb.total_budget), kernel="k_compact",
+                                          algorithmic_bytes=cbytes),
                 capped=dict(path="fw_contour_alloc_capped, cap = uniform count (4,096): the enforced mode",
                             ms_per_call=ms_capped, kept_rows=kept_capped),
-                window_score=dict(path="fw_window_score: 32 window queries x 256 cells x 32,768 keys, d=128, "
+                window_score=dict(path=f"fw_window_score: 32 window queries x {cb.cells} cells x 32,768 keys, d=128, "
                                        "pool 7 (TMA + tcgen05, two passes over K)",
                                   ms_per_call=ms_ws, keys_per_s=cb.cells * cb.T / (ms_ws * 1e-3),
                                   roofline=roofline("hbm", wbytes / (ms_ws * 1e-3) / 1e9, peaks["hbm_gbs"], "GB/s",
+                                                    traffic_of("window_score", cb.cells * cb.T),
                                                     kernel="k_wscore", algorithmic_bytes=wbytes,
                                                     bytes_basis="K once, the window queries, votes and scores "
                                                                 "written; the kernel reads K twice"),
                                   tensor_tflops=wflops / (ms_ws * 1e-3) / 1e12),
-                decode_append=dict(path="fw_ragged_append: one new K/V row per cell (256 cells, d=128)",
+                decode_append=dict(path=f"fw_ragged_append: one new K/V row per cell ({cb.cells} cells, d=128)",
                                    ms_per_call=ms_app, rows_per_s=cb.cells / (ms_app * 1e-3)))
 
 
@@ -666,6 +680,8 @@ def main():
                     help="rows per head of the long-row section (profiling captures of a smaller case)")
     ap.add_argument("--mixed-rows-scale", type=float, default=1.0,
                     help="fraction of the mixed-profile rows (profiling captures of a smaller case)")
+    ap.add_argument("--contour-cells", type=int, default=256,
+                    help="cells of the contour workload (profiling captures of a smaller case)")
     args = ap.parse_args()
     K, W = args.steps, max(3, args.warmup)
 
@@ -713,7 +729,7 @@ def main():
         exact_toy=lambda k, w: section_exact_toy(fw, device, k, w, flush, peaks),
         adversarial=lambda k, w: section_adversarial(fw, device, k, w, flush, peaks),
         long_rows=lambda k, w: section_long_rows(fw, device, k, w, flush, peaks, rows_per_head=args.long_rows_per_head),
-        contour=lambda k, w: section_contour(fw, device, k, w, flush, peaks),
+        contour=lambda k, w: section_contour(fw, device, k, w, flush, peaks, cells=args.contour_cells),
         mixed=lambda k, w: section_mixed(fw, device, k, w, flush, peaks, rows_scale=args.mixed_rows_scale),
         pool=lambda k, w: section_pool(fw, device, k, w, flush, peaks),
         audit=lambda k, w: section_audit(fw, device, k, w, flush, peaks))
