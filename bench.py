@@ -192,18 +192,27 @@ class EnumWorkload:
         self.E = E
         self.ev = Events()
         self.last = None
+        # one stream per group: the groups are independent, so one group's
+        # kernels fill the SMs another group's launch tails leave idle
+        self.streams = [torch.cuda.Stream() for _ in self.rows]
 
     def step(self, time_enum=False):
         fw = self.fw
+        main = torch.cuda.current_stream()
+        for st in self.streams:
+            st.wait_stream(main)
         outs = []
-        for rows, k2, k1, kmax in zip(self.rows, self.k2, self.k1, self.kmax):
-            top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
-            sw = fw.swap_refine(rows, k2, top, E=self.E, max_swaps=32)
-            e0 = self.ev.start() if time_enum else None
-            bs = fw.best_subset(rows, k1, k_max=kmax)
-            if time_enum:
-                self.ev.stop(e0, rows.num_rows)
+        for st, rows, k2, k1, kmax in zip(self.streams, self.rows, self.k2, self.k1, self.kmax):
+            with torch.cuda.stream(st):
+                top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
+                sw = fw.swap_refine(rows, k2, top, E=self.E, max_swaps=32)
+                e0 = self.ev.start() if time_enum else None
+                bs = fw.best_subset(rows, k1, k_max=kmax)
+                if time_enum:
+                    self.ev.stop(e0, rows.num_rows)
             outs.append((top, sw, bs))
+        for st in self.streams:
+            main.wait_stream(st)
         self.last = outs
         return outs
 
@@ -228,8 +237,8 @@ class EnumWorkload:
 class EnumE2E:
     """The same step through the public API from pinned host buffers: inputs are
     copied to the device, results copied back, inside the timed region.  The
-    five groups are pipelined: a copy stream uploads group g + 1 while the
-    compute stream works on group g (each group's compute waits for its own
+    five groups are pipelined: a copy stream uploads group g + 1 while group
+    g computes on its own stream (each group's compute waits for its own
     upload; the uploads of a step wait for the previous step's compute)."""
 
     def __init__(self, wl: EnumWorkload):
@@ -273,14 +282,19 @@ class EnumE2E:
                 ev.record(cs)
                 ready.append(ev)
         self.upload_ev.append((u0, ready[-1]))
-        for ev, rows, k2, k1, hout in zip(ready, wl.rows, wl.k2, wl.k1, self.out_host):
-            main.wait_event(ev)
-            top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
-            sw = fw.swap_refine(rows, k2, top, E=N_KEYS, max_swaps=32)
-            bs = fw.best_subset(rows, k1, k_max=K_SEL)
-            for h, t in zip(hout, (top["gap"], top["dropped"], sw["refined_gap"], bs["best_gap"], bs["best_rank"],
-                                   bs["best_idx"][:, :K_SEL])):
-                h.copy_(t.reshape(h.shape), non_blocking=True)
+        for st in wl.streams:
+            st.wait_stream(main)
+        for st, ev, rows, k2, k1, hout in zip(wl.streams, ready, wl.rows, wl.k2, wl.k1, self.out_host):
+            with torch.cuda.stream(st):
+                st.wait_event(ev)
+                top = fw.dense_and_topk_gap(rows, k2, kept_bits=False)
+                sw = fw.swap_refine(rows, k2, top, E=N_KEYS, max_swaps=32)
+                bs = fw.best_subset(rows, k1, k_max=K_SEL)
+                for h, t in zip(hout, (top["gap"], top["dropped"], sw["refined_gap"], bs["best_gap"],
+                                       bs["best_rank"], bs["best_idx"][:, :K_SEL])):
+                    h.copy_(t.reshape(h.shape), non_blocking=True)
+        for st in wl.streams:
+            main.wait_stream(st)
         return self.out_host
 
     def upload_ms(self, last):
