@@ -52,7 +52,11 @@ constexpr int TK = 2;        // kept keys per thread in the first-round product 
 constexpr int TS = 8;        // pool slots per thread in that tile (4 threads cover 32)
 constexpr int QL = 4;        // lanes per kept key in the round pass
 constexpr int KPI = SWT / QL;  // kept keys per block iteration of the pass
-constexpr int LS_BPS = 3;    // resident blocks per SM
+// resident blocks per SM: three for rows up to 8,192 keys (short rounds, whose
+// fixed per-round costs want more blocks), two above (the registers keep the
+// next key's value row, table entries and mass in flight without spilling)
+constexpr int LS_BPS_SHORT = 3, LS_BPS_LONG = 2, LS_LONG_N = 8192;
+inline int ls_bps(const RowsDev &R) { return R.max_n > LS_LONG_N ? LS_BPS_LONG : LS_BPS_SHORT; }
 
 struct LSArgs {
     RowsDev R;
@@ -323,8 +327,8 @@ __device__ __forceinline__ float any_score(float4 sq, float cij, float p_i, floa
     return vector_pair_score<DPL, VT>(vr, mu, g, Wt, Ep, q, p_i, sq.w, P, P2, N);
 }
 
-template <int DPL, typename VT>
-__global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
+template <int DPL, typename VT, int BPS>
+__global__ void __launch_bounds__(SWT, BPS) k_long_swap(const LSArgs a)
 {
     constexpr int d = DPL * 32;
     const int Ep = a.Ep;         // pool slots, a multiple of 32
@@ -762,20 +766,24 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
                         score_key(t, i, vr, sg, sn, p_i, sn, false, cq0);
                     }
                 } else {
-                    // software pipeline: the value row of the next iteration and the
-                    // kept index of the one after are in flight during this one
+                    // software pipeline: the value row, table entries and mass of
+                    // the next iteration and the kept index of the one after are in
+                    // flight during this one
                     const int niter = (nk + KPI - 1) / KPI;
                     int i_cur = kb[gq < nk ? gq : nk - 1];
                     int i_next = kb[gq + KPI < nk ? gq + KPI : nk - 1];
                     LaneRow<DPL, VT> row;
                     row.load(V + (int64_t)i_cur * d, sub);
+                    float cq0[8];
+                    load_cq0(gq < nk ? gq : nk - 1, cq0);
+                    float p_i = pk[gq < nk ? gq : nk - 1], x2 = xk[gq < nk ? gq : nk - 1];
                     for (int it = 0; it < niter; ++it) {
                         const int t = it * KPI + gq;
                         const bool valid = t < nk;
-                        const int ts = valid ? t : nk - 1;
-                        float cq0[8];
-                        load_cq0(ts, cq0);
-                        const float p_i = pk[ts], x2 = xk[ts];
+                        const int tn = t + KPI < nk ? t + KPI : nk - 1;
+                        float cqn[8];
+                        load_cq0(tn, cqn);
+                        const float p_n = pk[tn], x2_n = xk[tn];
                         LaneRow<DPL, VT> rown;
                         rown.load(V + (int64_t)i_next * d, sub);
                         const int tnn = t + 2 * KPI;
@@ -791,6 +799,10 @@ __global__ void __launch_bounds__(SWT, LS_BPS) k_long_swap(const LSArgs a)
                         row = rown;
                         i_cur = i_next;
                         i_next = i_nn;
+#pragma unroll
+                        for (int m = 0; m < 8; ++m) cq0[m] = cqn[m];
+                        p_i = p_n;
+                        x2 = x2_n;
                     }
                 }
                 first = false;
@@ -897,13 +909,13 @@ template <int DPL> size_t ls_smem(int Ep)
 
 }  // namespace
 
-// LS_BPS resident blocks per SM (the launch bounds guarantee the registers for
-// it); the workspace is sized by the same count, queried from the current device
+// ls_bps(R) resident blocks per SM (the launch bounds guarantee the registers
+// for it); the workspace is sized by the same count, queried from the current device
 static unsigned ls_grid(const RowsDev &R)
 {
     int sms = 0;
     if (device_sms(&sms) != FW_OK) sms = 152;  // no device: the size query still answers
-    return (unsigned)std::min<int64_t>(R.rows, (int64_t)sms * LS_BPS);
+    return (unsigned)std::min<int64_t>(R.rows, (int64_t)sms * ls_bps(R));
 }
 
 static size_t ls_array_bytes(const RowsDev &R) { return align256((size_t)ls_grid(R) * R.max_n * 4); }
@@ -954,11 +966,12 @@ fw_status long_swap(const RowsDev &R, const int32_t *k, int nb, const fw_gap_out
     a.pbuf = (float *)(w + 2 * arr);
     a.xbuf = (float *)(w + 3 * arr);
     a.cbuf = (float *)(w + 4 * arr);
+    const bool lng = ls_bps(R) == LS_BPS_LONG;
     FW_DISPATCH(R.d, R.v_dtype, {
         const size_t smem = ls_smem<DPL>(a.Ep);
-        FW_CUDA_CHECK(cudaFuncSetAttribute(k_long_swap<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)smem));
-        FW_LAUNCH((k_long_swap<DPL, VT>), grid, SWT, smem, s, a);
+        auto kern = lng ? k_long_swap<DPL, VT, LS_BPS_LONG> : k_long_swap<DPL, VT, LS_BPS_SHORT>;
+        FW_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        FW_LAUNCH(kern, grid, SWT, smem, s, a);
     });
     return FW_OK;
 }
