@@ -161,12 +161,28 @@ __global__ void __launch_bounds__(CPT) k_c_pass(CArgs a, int pass)
         if (cap && j < nf && (key & pmask) == cpre) atomicAdd(&hc[dg], 1u);
     };
     if ((a.T & 3) == 0 && (reinterpret_cast<uintptr_t>(sc) & 15) == 0) {
-        for (int q = threadIdx.x; q < a.T / 4; q += CPT) {
-            const float4 v = __ldg(reinterpret_cast<const float4 *>(sc) + q);
-            visit(4 * q, v.x);
-            visit(4 * q + 1, v.y);
-            visit(4 * q + 2, v.z);
-            visit(4 * q + 3, v.w);
+        // LD vectors per thread in flight before any is used (one at a time
+        // left each block waiting on a memory round trip per vector: a block
+        // per cell, 256 cells, too few bytes in flight per SM)
+        constexpr int LD = 8;
+        const int nq = a.T / 4;
+        for (int q0 = threadIdx.x; q0 < nq; q0 += LD * CPT) {
+            float4 v[LD];
+#pragma unroll
+            for (int u = 0; u < LD; ++u) {
+                const int q = q0 + u * CPT;
+                v[u] = q < nq ? __ldg(reinterpret_cast<const float4 *>(sc) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int u = 0; u < LD; ++u) {
+                const int q = q0 + u * CPT;
+                if (q < nq) {
+                    visit(4 * q, v[u].x);
+                    visit(4 * q + 1, v[u].y);
+                    visit(4 * q + 2, v[u].z);
+                    visit(4 * q + 3, v[u].w);
+                }
+            }
         }
     } else {
         for (int j = threadIdx.x; j < a.T; j += CPT) visit(j, __ldg(sc + j));
@@ -223,10 +239,36 @@ __global__ void __launch_bounds__(CT) k_c_count(CArgs a)
     const uint32_t tk = s_tk;
     int gt = 0, eq = 0;
     if (a.K > 0) {
-        for (int j = threadIdx.x; j < a.T - a.F; j += CT) {
-            const uint32_t key = order_key(__ldg(a.scores + (int64_t)c * a.T + j));
-            gt += key > tk;
-            eq += key == tk;
+        // eight 16-byte loads per thread in flight before any is used
+        const float *sc = a.scores + (int64_t)c * a.T;
+        const int nf = a.T - a.F;
+        auto tally = [&](int j, float x) {
+            if (j < nf) {
+                const uint32_t key = order_key(x);
+                gt += key > tk;
+                eq += key == tk;
+            }
+        };
+        if ((a.T & 3) == 0 && (reinterpret_cast<uintptr_t>(sc) & 15) == 0) {
+            const int nq = (nf + 3) / 4;
+            for (int q0 = threadIdx.x; q0 < nq; q0 += 8 * CT) {
+                float4 v[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int q = q0 + u * CT;
+                    v[u] = q < nq ? __ldg(reinterpret_cast<const float4 *>(sc) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int j = 4 * (q0 + u * CT);
+                    tally(j, v[u].x);
+                    tally(j + 1, v[u].y);
+                    tally(j + 2, v[u].z);
+                    tally(j + 3, v[u].w);
+                }
+            }
+        } else {
+            for (int j = threadIdx.x; j < nf; j += CT) tally(j, __ldg(sc + j));
         }
     }
     for (int o = 16; o > 0; o >>= 1) {
