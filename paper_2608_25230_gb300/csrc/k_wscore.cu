@@ -44,6 +44,16 @@ struct WsArgs {
 
 __device__ __forceinline__ void ws_named_barrier() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
+// 2^x by the hardware approximation (ex2.approx.ftz: ~2 ulp, well inside the
+// score's 1e-4 tolerance); the per-(key, query) exponentials are most of the
+// epilogue's work
+__device__ __forceinline__ float ex2a(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // combine two (max, sum of 2^(x - max)) pairs
 __device__ __forceinline__ void ms_merge(float &m, float &z, float m2, float z2)
 {
@@ -202,21 +212,27 @@ __global__ void __launch_bounds__(WS_THREADS, 2) k_wscore(const __grid_constant_
             if (!ok) continue;
             const int j = t * WS_KT + q4 * 32 + lane;
             const int lim = T - w;  // query i sees keys j <= lim + i
+            // a tile whose keys every query sees (all but the cell's last) skips the masks
+            const bool open = t * WS_KT + WS_KT - 1 <= lim && w == WS_N;
             if (pass == 0) {
+                // running (max, sum) with one exponential per element: when x
+                // raises the max the old sum is scaled by 2^(m - x), else
+                // 2^(x - m) is added
 #pragma unroll
                 for (int i = 0; i < WS_N; ++i) {
-                    if (j < T && i < w && j <= lim + i) {
+                    if (open || (j < T && i < w && j <= lim + i)) {
                         const float x = v[i] * scale2;
-                        const float mn = fmaxf(m[i], x);
-                        z[i] = (m[i] == -INFINITY ? 0.f : z[i] * exp2f(m[i] - mn)) + exp2f(x - mn);
-                        m[i] = mn;
+                        const float dx = x - m[i];
+                        const float e = ex2a(-fabsf(dx));
+                        z[i] = dx > 0.f ? fmaf(z[i], e, 1.f) : z[i] + e;
+                        m[i] = fmaxf(m[i], x);
                     }
                 }
             } else if (j < T) {
                 float vote = 0.f;
 #pragma unroll
                 for (int i = 0; i < WS_N; ++i)
-                    if (i < w && j <= lim + i) vote += exp2f(v[i] * scale2 - m[i]) * z[i];
+                    if (open || (i < w && j <= lim + i)) vote = fmaf(ex2a(fmaf(v[i], scale2, -m[i])), z[i], vote);
                 a.votes[(int64_t)c * T + j] = vote;
             }
         }
