@@ -235,7 +235,10 @@ fw_status fw_pool_best_subset(const fw_rows *rows, const int32_t *k, int32_t nb,
                               const fw_gap_out *topk, float *best_gap, int32_t *best_idx, int32_t k_max,
                               float *topk_gap, int64_t *n_cand, int32_t *row_status, void *workspace,
                               size_t workspace_bytes, void *stream);
-/* Workspace bytes: the pool of every (row, budget), 64 int32 each, and its size. */
+/* Workspace bytes: the pool of every (row, budget), 64 int32 each, and its
+ * size; then, for each warp of the enumeration launch (4 blocks of 4 warps
+ * per SM of the current device, fewer for small batches), a buffer of 4,096
+ * re-scoring candidates and an fp64 Gram matrix of the pool (64 KB). */
 size_t fw_pool_best_subset_workspace(const fw_rows *rows, int32_t nb);
 
 /* The deployed selectors audited in Sec. 2.3 (App. C settings), as kept sets

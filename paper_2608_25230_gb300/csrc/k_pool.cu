@@ -16,17 +16,21 @@
 //                 the sums over all members but the lowest held while the
 //                 lowest member runs (O(m) shared-memory reads per subset).
 //                 Every subset gets an fp32 score es^2 and a rigorous interval
-//                 around it (the rounding of the Gram products and of the
-//                 sums, bounded by (sum_pool |u|)^2); the subsets whose lower
-//                 end does not exceed the least upper end are re-scored by the
-//                 warp in fp64 from the definition (N_A / p(A) - o), and the
-//                 least es wins, exact ties to the smallest colex rank of the
-//                 members' pool positions.
+//                 around it (the rounding of the Gram sums, bounded by
+//                 (sum_pool |u|)^2); the subsets whose lower end does not
+//                 exceed the least upper end are buffered (4,096 per warp, in
+//                 the workspace) and re-scored in fp64 as
+//                 es^2 = (sum_{a,b in A} G_ab) / p(A)^2 from an fp64 copy of
+//                 the Gram matrix (the products u_a . u_b formed in fp64 from
+//                 the fp32 masses, the bf16 / fp32 values and o), and the least
+//                 es wins, exact ties to the smallest colex rank of the
+//                 members' pool positions.  (Re-scoring from the value rows
+//                 cost |A| dependent row loads per candidate; flat rows send
+//                 ~1,000 candidates per item.)
 //
 // Nothing waits on another block; a buffer of re-scoring candidates that
-// overflows (rows with very many near-equal subsets) falls back to a slower
-// per-lane re-scoring pass over the same candidates, so the answer stays
-// exact.
+// overflows falls back to a per-lane re-scoring pass over the same
+// candidates, so the answer stays exact.
 #include <algorithm>
 #include <climits>
 
@@ -40,7 +44,8 @@ constexpr int PE_W = 4;              // k_pool_enum: warps per block, one (row, 
 constexpr int PMAX = 64;             // pool keys
 constexpr int PSMAX = 32;            // largest budget
 constexpr int PB_STAGE_MAX = 49152;  // keys per row staged in shared memory
-constexpr int CBUF = 32;             // re-scoring candidates buffered per warp
+constexpr int GCAP = 4096;           // re-scoring candidates buffered per warp (workspace)
+constexpr int PE_BPS = 4;            // k_pool_enum blocks per SM in the launch (each warp owns workspace)
 constexpr uint64_t PE_MAX_SUBSETS = 1ull << 32;
 constexpr int GLD = PMAX + 1;        // Gram row stride (odd: conflict-free columns)
 
@@ -77,6 +82,8 @@ struct PoolArgs {
     float *topk_gap;           // [rows][nb] or null
     int32_t *row_status;       // [rows] or null
     int64_t *n_cand;           // [rows][nb] re-scored subsets, or null
+    uint64_t *gcand;           // ws [gridDim.x * PE_W][GCAP] candidate masks of each warp
+    double *g64;               // ws [gridDim.x * PE_W][PMAX * PMAX] fp64 Gram matrix of each warp
 };
 
 // ------------------------------------------------------------ the pool
@@ -306,7 +313,6 @@ struct EnumSm {
     float G[PMAX * GLD];
     float pp[PMAX];
     float t[PMAX];        // t_x = sum_y G_xy = u_x . U
-    uint64_t cand[CBUF];  // re-scoring candidates (pool-position masks of A)
     int32_t pidx[PMAX];
     int ncand;
 };
@@ -341,24 +347,32 @@ __device__ __forceinline__ double es_warp(const VT *V, const float *o_lane, cons
     return sqrt(e2);
 }
 
-// the same, by one lane alone (fallback when the candidate buffer overflows)
-template <int DPL, typename VT>
-__device__ double es_lane(const VT *V, const float *o, const EnumSm &S, uint64_t A)
+// es of the pool positions in A from the fp64 Gram matrix: lane i sums the row
+// of A's i-th member over A (|A| <= 32), the warp adds the rows.
+__device__ __forceinline__ double es_gram_warp(const double *g, const EnumSm &S, uint64_t A, int lane)
 {
-    constexpr int d = DPL * 32;
-    double PA = 0.0;
-    for (uint64_t w = A; w; w &= w - 1) PA += (double)S.pp[__ffsll((long long)w) - 1];
-    double e2 = 0.0;
-    for (int c = 0; c < d; ++c) {
-        double N = 0.0;
-        for (uint64_t w = A; w; w &= w - 1) {
-            const int x = __ffsll((long long)w) - 1;
-            N = fma((double)S.pp[x], (double)load_v(V, (int64_t)S.pidx[x] * d + c), N);
-        }
-        const double diff = N / PA - (double)o[c];
-        e2 = fma(diff, diff, e2);
+    double rs = 0.0, pa = 0.0;
+    int i = 0;
+    for (uint64_t w = A; w; w &= w - 1, ++i) {
+        if (i != lane) continue;
+        const int x = __ffsll((long long)w) - 1;
+        pa = (double)S.pp[x];
+        for (uint64_t w2 = A; w2; w2 &= w2 - 1) rs += g[x * PMAX + __ffsll((long long)w2) - 1];
     }
-    return sqrt(e2);
+    const double Q = warp_sum_d(rs), PA = warp_sum_d(pa);
+    return sqrt(fmax(Q, 0.0)) / PA;
+}
+
+// the same by one lane alone (fallback when the candidate buffer overflows)
+__device__ double es_gram_lane(const double *g, const EnumSm &S, uint64_t A)
+{
+    double Q = 0.0, PA = 0.0;
+    for (uint64_t w = A; w; w &= w - 1) {
+        const int x = __ffsll((long long)w) - 1;
+        PA += (double)S.pp[x];
+        for (uint64_t w2 = A; w2; w2 &= w2 - 1) Q += g[x * PMAX + __ffsll((long long)w2) - 1];
+    }
+    return sqrt(fmax(Q, 0.0)) / PA;
 }
 
 // Walks the colex ranks [lo, hi) of m-subsets C of the pool and calls
@@ -412,6 +426,9 @@ __global__ void __launch_bounds__(PE_W * 32) k_pool_enum(PoolArgs a)
     constexpr int d = DPL * 32;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     EnumSm &S = reinterpret_cast<EnumSm *>(smraw)[wid];
+    const int64_t wslot = (int64_t)blockIdx.x * PE_W + wid;
+    uint64_t *gc = a.gcand + wslot * GCAP;
+    double *g64 = a.g64 + wslot * (PMAX * PMAX);
     const int64_t items = a.R.rows * a.nb;
     for (int64_t it = (int64_t)blockIdx.x * PE_W + wid; it < items; it += (int64_t)gridDim.x * PE_W) {
         const int64_t r = it / a.nb;
@@ -451,20 +468,26 @@ __global__ void __launch_bounds__(PE_W * 32) k_pool_enum(PoolArgs a)
         }
         if (lane == 0) S.ncand = 0;
         __syncwarp();
-        // Gram matrix of u = p (v - o): the warp forms each product across d
+        // Gram matrix of u = p (v - o) in fp64 (the warp forms each product
+        // across d): the fp64 copy for the re-scoring, its fp32 rounding for
+        // the walk
         for (int x = 0; x < P; ++x) {
-            float dx[DPL];
-            load_row_part<DPL, VT>(V, S.pidx[x], lane, dx);
+            float vx[DPL];
+            load_row_part<DPL, VT>(V, S.pidx[x], lane, vx);
+            double dx[DPL];
 #pragma unroll
-            for (int c = 0; c < DPL; ++c) dx[c] -= ol[c];
+            for (int c = 0; c < DPL; ++c) dx[c] = (double)vx[c] - (double)ol[c];
             for (int y = x; y < P; ++y) {
-                float dy[DPL];
-                load_row_part<DPL, VT>(V, S.pidx[y], lane, dy);
-                float acc = 0.f;
+                float vy[DPL];
+                load_row_part<DPL, VT>(V, S.pidx[y], lane, vy);
+                double acc = 0.0;
 #pragma unroll
-                for (int c = 0; c < DPL; ++c) acc = fmaf(dx[c], dy[c] - ol[c], acc);
-                acc = warp_sum(acc) * S.pp[x] * S.pp[y];
-                if (lane == 0) S.G[x * GLD + y] = S.G[y * GLD + x] = acc;
+                for (int c = 0; c < DPL; ++c) acc = fma(dx[c], (double)vy[c] - (double)ol[c], acc);
+                acc = warp_sum_d(acc) * (double)S.pp[x] * (double)S.pp[y];
+                if (lane == 0) {
+                    S.G[x * GLD + y] = S.G[y * GLD + x] = (float)acc;
+                    g64[x * PMAX + y] = g64[y * PMAX + x] = acc;
+                }
             }
         }
         __syncwarp();
@@ -506,7 +529,7 @@ __global__ void __launch_bounds__(PE_W * 32) k_pool_enum(PoolArgs a)
             if (low <= U) {
                 ++ncand;
                 const int slot = atomicAdd(&S.ncand, 1);
-                if (slot < CBUF) S.cand[slot] = direct ? Cm : (all & ~Cm);
+                if (slot < GCAP) gc[slot] = direct ? Cm : (all & ~Cm);
                 else over = 1;
             }
         });
@@ -521,8 +544,8 @@ __global__ void __launch_bounds__(PE_W * 32) k_pool_enum(PoolArgs a)
         } else if (!over) {
             const int nc = S.ncand;
             for (int q = 0; q < nc; ++q) {
-                const uint64_t A = S.cand[q];
-                const double es = es_warp<DPL, VT>(V, ol, S, A, lane);
+                const uint64_t A = gc[q];
+                const double es = es_gram_warp(g64, S, A, lane);
                 const uint64_t rank = colex_rank64(A);
                 if (es < bes || (es == bes && rank < brank)) {
                     bes = es;
@@ -532,11 +555,10 @@ __global__ void __launch_bounds__(PE_W * 32) k_pool_enum(PoolArgs a)
             }
         } else {
             // every lane re-scores its own candidates alone
-            const float *orow = a.o + r * d;
             walk(S, P, m, direct, lo, hi, UU, PU, Eabs, pe, [&](uint64_t Cm, float low, float) {
                 if (low <= U) {
                     const uint64_t A = direct ? Cm : (all & ~Cm);
-                    const double es = es_lane<DPL, VT>(V, orow, S, A);
+                    const double es = es_gram_lane(g64, S, A);
                     const uint64_t rank = colex_rank64(A);
                     if (es < bes || (es == bes && rank < brank)) {
                         bes = es;
@@ -586,9 +608,24 @@ __global__ void __launch_bounds__(PE_W * 32) k_pool_enum(PoolArgs a)
 
 static size_t pool_bytes(const RowsDev &R, int nb) { return align256((size_t)R.rows * nb * PMAX * 4); }
 
+// blocks of the enumeration launch: PE_BPS per SM, fewer when there are fewer items
+static int64_t pool_enum_blocks(const RowsDev &R, int nb)
+{
+    int sms = 0;
+    if (device_sms(&sms) != FW_OK) sms = 152;  // no device: the size query still answers
+    const int64_t items = R.rows * nb;
+    return std::max<int64_t>(1, std::min<int64_t>((items + PE_W - 1) / PE_W, (int64_t)sms * PE_BPS));
+}
+
+// per warp of the enumeration launch: the candidate buffer and the fp64 Gram matrix
+static size_t warp_ws_bytes(const RowsDev &R, int nb)
+{
+    return align256((size_t)pool_enum_blocks(R, nb) * PE_W * (GCAP + PMAX * PMAX) * 8);
+}
+
 size_t pool_best_subset_workspace(const RowsDev &R, int nb)
 {
-    return pool_bytes(R, nb) + align256((size_t)R.rows * nb * 4);
+    return pool_bytes(R, nb) + align256((size_t)R.rows * nb * 4) + warp_ws_bytes(R, nb);
 }
 
 fw_status pool_best_subset(const RowsDev &R, const int32_t *k, int nb, const int32_t *E, const fw_gap_out &topk,
@@ -608,6 +645,11 @@ fw_status pool_best_subset(const RowsDev &R, const int32_t *k, int nb, const int
     a.Z = topk.row_sum;
     a.pool = (int32_t *)ws;
     a.pool_n = (int32_t *)((char *)ws + pool_bytes(R, nb));
+    {
+        char *w = (char *)ws + pool_bytes(R, nb) + align256((size_t)R.rows * nb * 4);
+        a.gcand = (uint64_t *)w;
+        a.g64 = (double *)(w + (size_t)pool_enum_blocks(R, nb) * PE_W * GCAP * 8);
+    }
     a.best_gap = best_gap;
     a.best_idx = best_idx;
     a.k_max = k_max;
@@ -623,9 +665,7 @@ fw_status pool_best_subset(const RowsDev &R, const int32_t *k, int nb, const int
         FW_LAUNCH((k_pool_build<DPL, VT>), (unsigned)std::min<int64_t>(R.rows, (int64_t)sms * 4), PB_T, sb, st, a);
         const size_t se = (size_t)PE_W * sizeof(EnumSm);
         FW_CUDA_CHECK(cudaFuncSetAttribute(k_pool_enum<DPL, VT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)se));
-        const int64_t items = R.rows * nb;
-        const int64_t blocks = (items + PE_W - 1) / PE_W;
-        FW_LAUNCH((k_pool_enum<DPL, VT>), (unsigned)std::min<int64_t>(blocks, (int64_t)sms * 16), PE_W * 32, se, st, a);
+        FW_LAUNCH((k_pool_enum<DPL, VT>), (unsigned)pool_enum_blocks(R, nb), PE_W * 32, se, st, a);
     });
     return FW_OK;
 }
