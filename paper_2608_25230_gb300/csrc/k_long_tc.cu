@@ -950,7 +950,7 @@ __global__ void __launch_bounds__(pvm_nt<D>(), 1) k_long_pv_tma(const __grid_con
 // by a column of ones.  Warp 0 copies (V boxes by TMA, logits by cp.async),
 // warp 1 issues the MMAs, warps 2..5 build P^T (K-major, 128-byte swizzle)
 // and flush the TMEM chunk accumulators, each warp its 32 TMEM lanes (dims).
-constexpr int TN_BS = 4;                 // copy slots (V + logits)
+constexpr int TN_BS = 3;                 // copy slots (V + logits): small CTAs, three or four per SM
 constexpr int TN_PW = 4;                 // producer / flush warps
 constexpr int TN_NT = (TN_PW + 2) * 32;  // threads
 template <int NB, int RT> __host__ __device__ constexpr int tn_cols() { return ((NB + 1) * RT + 15) / 16 * 16; }
@@ -960,7 +960,7 @@ template <int NB, int RT> __host__ __device__ constexpr uint32_t tn_tcols()
 }
 
 template <int D, int NB, int RT>
-__global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__ CUtensorMap tmV, const TcArgs a)
+__global__ void __launch_bounds__(TN_NT, 3) k_long_pv_tn(const __grid_constant__ CUtensorMap tmV, const TcArgs a)
 {
     constexpr int NBB = NB + 1;                 // bands
     constexpr int NP = NBB * RT;                // (band, row) pairs
@@ -969,7 +969,11 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
     constexpr int TPR = NPROD / RT;             // producer threads per row (32 or 16)
     constexpr int KPTH = KS / TPR;              // keys per producer thread and stage (2 or 4)
     constexpr int NVBOX = D / 64;               // 64-dim blocks of V
-    constexpr int V_SLOT = 2 * KS * 128;        // two 64-row blocks of the M = 128 operand
+    // a V slot holds the d = 128 dims as two 64-row blocks of the M = 128
+    // operand; for d = 64 it holds one, and every slot's second block is one
+    // shared zero block behind the slots (each slot's descriptor points its
+    // leading byte offset there)
+    constexpr int V_SLOT = NVBOX * KS * 128;
     constexpr int P_TERM = N * 128;             // one split term of P^T: N rows x 64 keys
     constexpr int P_SLOT = NSPLIT * P_TERM;
     constexpr uint32_t TCOLS = tn_tcols<NB, RT>();
@@ -978,8 +982,8 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
     static_assert(NP * (D + 1) * 4 <= TN_BS * V_SLOT, "epilogue staging fits the V slots");
     extern __shared__ uint8_t smraw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~(uintptr_t)1023);
-    uint8_t *sV = sm;                                     // [TN_BS][2][64 keys x 128 B]
-    uint8_t *sP = sV + TN_BS * V_SLOT;                    // [ASLOTS][NSPLIT][N x 128 B]
+    uint8_t *sV = sm;                                     // [TN_BS][NVBOX][64 keys x 128 B] (+ zero block)
+    uint8_t *sP = sV + TN_BS * V_SLOT + (NVBOX == 1 ? KS * 128 : 0);  // [ASLOTS][NSPLIT][N x 128 B]
     float *sL = reinterpret_cast<float *>(sP + ASLOTS * P_SLOT);  // [TN_BS][RT][64]
     float *sG = sL + TN_BS * RT * KS;                     // [TN_BS][64] the vote's G
     float *acc = reinterpret_cast<float *>(sV);           // epilogue: [NP][D + 1]
@@ -1062,12 +1066,10 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
         for (int x = 0; x < NACC; ++x) tc::mbar_init(&accfree[x], TN_PW);
         tc::mbar_init_fence();
     }
-    // d = 64: the second 64-row block of every V slot is zero (M = 128 rows)
+    // d = 64: the second 64-row block of every slot is the shared zero block (M = 128 rows)
     if (NVBOX == 1)
-        for (int e = tid; e < TN_BS * KS * 8; e += TN_NT) {
-            const int slot = e / (KS * 8), q = e % (KS * 8);
-            reinterpret_cast<uint4 *>(sV + slot * V_SLOT + KS * 128)[q] = make_uint4(0u, 0u, 0u, 0u);
-        }
+        for (int e = tid; e < KS * 8; e += TN_NT)
+            reinterpret_cast<uint4 *>(sV + TN_BS * V_SLOT)[e] = make_uint4(0u, 0u, 0u, 0u);
     // rows of P^T past the NP pairs stay zero in every slot and term
     for (int e = tid; e < ASLOTS * NSPLIT * N * 8; e += TN_NT) {
         const int m = (e / 8) % N;
@@ -1166,7 +1168,10 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
                 tc::fence_after_sync();
                 const uint32_t dacc = taddr + (uint32_t)((ch % NACC) * N);
                 const bool fresh = it % CH == 0;
-                const uint64_t abs_ = ad0 + (uint64_t)((bs * V_SLOT) >> 4);
+                // V^T of the slot; d = 64: the second block is the zero block
+                const uint64_t abs_ = NVBOX == 2
+                                          ? ad0 + (uint64_t)((bs * V_SLOT) >> 4)
+                                          : tc::sdesc_sw128(tc::smem_u32(sV) + bs * V_SLOT, (TN_BS - bs) * V_SLOT, 1024);
                 const uint64_t bas = bd0 + (uint64_t)((as * P_SLOT) >> 4);
 #pragma unroll
                 for (int ks = 0; ks < KS / 16; ++ks) {
@@ -1439,10 +1444,10 @@ __global__ void __launch_bounds__(TN_NT, 2) k_long_pv_tn(const __grid_constant__
     }
 }
 
-template <int NB, int RT> size_t pv_tn_smem()
+template <int D, int NB, int RT> size_t pv_tn_smem()
 {
-    return 1024 + (size_t)TN_BS * 2 * KS * 128 + (size_t)ASLOTS * NSPLIT * tn_cols<NB, RT>() * 128 +
-           (size_t)TN_BS * RT * KS * 4 + (size_t)TN_BS * KS * 4;
+    return 1024 + (size_t)TN_BS * (D / 64) * KS * 128 + (D == 64 ? KS * 128 : 0) +
+           (size_t)ASLOTS * NSPLIT * tn_cols<NB, RT>() * 128 + (size_t)TN_BS * RT * KS * 4 + (size_t)TN_BS * KS * 4;
 }
 
 template <int D> size_t pv_tma_smem()
@@ -1482,7 +1487,7 @@ fw_status launch_pv_tma(TcArgs a, const CUtensorMap &mv, cudaStream_t s)
             return FW_OK;
         };
 #define FW_PV_TN(DD, NN, RR) \
-    if (R.d == DD && nb == NN && rt == RR) return launch_tn(k_long_pv_tn<DD, NN, RR>, pv_tn_smem<NN, RR>());
+    if (R.d == DD && nb == NN && rt == RR) return launch_tn(k_long_pv_tn<DD, NN, RR>, pv_tn_smem<DD, NN, RR>());
 #define FW_PV_TN_D(DD) \
     FW_PV_TN(DD, 1, 4) FW_PV_TN(DD, 2, 4) FW_PV_TN(DD, 3, 4) FW_PV_TN(DD, 4, 4) \
     FW_PV_TN(DD, 1, 8) FW_PV_TN(DD, 2, 8) FW_PV_TN(DD, 3, 8) FW_PV_TN(DD, 4, 8)
