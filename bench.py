@@ -88,6 +88,27 @@ def fp32_peak_tflops(device, sm_mhz):
     return sms * 128 * 2 * sm_mhz * 1e6 / 1e12, sms
 
 
+def fp32_fma_measured(fw, device, iters=1 << 15, reps=3):
+    """The fp32 FMA throughput of the library's probe kernel (16 independent
+    chains per thread, 8 CTAs of 256 threads per SM), TFLOP/s: a check of the
+    nominal peak above."""
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    blocks = sms * 8
+    out = torch.empty(blocks * 256, dtype=torch.float32, device=device)
+    for _ in range(2):
+        fw.fp32_fma_probe(blocks, iters, out)
+    torch.cuda.synchronize()
+    best = float("inf")
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fw.fp32_fma_probe(blocks, iters, out)
+        e1.record()
+        e1.synchronize()
+        best = min(best, e0.elapsed_time(e1))
+    return 2.0 * blocks * 256 * 16 * iters / (best * 1e-3) / 1e12
+
+
 class ClockSampler:
     """nvidia-smi sampling of SM clock and throttle reasons during a region."""
 
@@ -772,6 +793,7 @@ def main():
     enum_launch_ms = sum(t for t, _ in enum_ev) / len(enum_ev)
     sm_mhz = clocks.get("sm_mhz") or peaks["sm_max"]
     fma_peak, sms = fp32_peak_tflops(device, sm_mhz)
+    fma_probe = fp32_fma_measured(fw, device)
     gram = wl.gram_flops()
     work = gram + stats["inner_ops"]
     alu_ach = work / (enum_ms * 1e-3) / 1e12
@@ -815,7 +837,10 @@ def main():
                                              "inner-enumeration operations; per step "
                                              f"{gram:.3e} + {stats['inner_ops']:.3e}",
                                   peak_basis=f"{sms} SMs x 128 fp32 lanes x 2 x {sm_mhz:.0f} MHz (median SM clock "
-                                             f"under load)"),
+                                             f"under load)",
+                                  peak_check=dict(fma_probe_tflops=fma_probe, of_nominal=fma_probe / fma_peak,
+                                                  kernel="fw_fp32_fma_probe: 16 independent FMA chains per "
+                                                         "thread, 8 CTAs of 256 threads per SM")),
                 e2e=dict(value=e2e_value, unit="rows/s",
                          h2d_bytes_per_step=e2e.h2d, d2h_bytes_per_step=e2e.d2h,
                          step_ms=[round(t, 2) for t in e2e_times],

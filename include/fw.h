@@ -414,6 +414,14 @@ fw_status fw_contour_alloc_noalloc(const float *scores, int32_t cells, int32_t T
  * a host buffer on the stack, so the call allocates nothing. */
 fw_status fw_sync_status(const int32_t *row_status, int64_t rows, int64_t *first_row, void *stream);
 
+/* Measurement aid, not part of the path: `blocks` CTAs of 256 threads each
+ * run `iters` iterations of 16 independent fp32 FMA chains (so 256 * 16 *
+ * iters FMAs per CTA, 2 flops each) and write one float per thread to
+ * out [blocks * 256] (device) so the work is kept.  Timed by the caller, it
+ * measures the fp32 FMA throughput that the exact search's ALU roofline is
+ * stated against.  FW_ERR_INVALID_ARG for blocks < 1 or iters < 1. */
+fw_status fw_fp32_fma_probe(int32_t blocks, int32_t iters, float *out, void *stream);
+
 /* Human-readable name of a status. */
 const char *fw_status_string(fw_status s);
 

@@ -258,6 +258,12 @@ fw_status fw_sync_status(const int32_t *row_status, int64_t rows, int64_t *first
     return FW_OK;
 }
 
+fw_status fw_fp32_fma_probe(int32_t blocks, int32_t iters, float *out, void *stream)
+{
+    if (blocks < 1 || iters < 1 || !out) return FW_ERR_INVALID_ARG;
+    return fp32_fma_probe(blocks, iters, out, (cudaStream_t)stream);
+}
+
 fw_status fw_best_subset_read_stats(const fw_rows *rows, const void *workspace, fw_best_subset_stats *stats,
                                     void *stream)
 {

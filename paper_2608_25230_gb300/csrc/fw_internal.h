@@ -108,6 +108,9 @@ fw_status selector_audit(const RowsDev &R, const int32_t *s, int nb, const fw_ga
 // swizzle.  False if the driver's encoder is unavailable or refuses the map.
 bool make_tma_2d_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 
+// The fp32 FMA throughput probe (a measurement aid).
+fw_status fp32_fma_probe(int blocks, int iters, float *out, cudaStream_t s);
+
 // Number of SMs of the current device (queried once per device).
 fw_status device_sms(int *sms);
 

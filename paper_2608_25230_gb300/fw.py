@@ -59,6 +59,8 @@ _lib.fw_swap_refine_workspace.restype = C.c_size_t
 _lib.fw_best_subset.argtypes = [C.POINTER(FwRows), vp, vp, vp, vp, C.c_int32, vp, vp, vp, C.c_size_t, vp]
 _lib.fw_best_subset_workspace.argtypes = [C.POINTER(FwRows)]
 _lib.fw_best_subset_workspace.restype = C.c_size_t
+_lib.fw_fp32_fma_probe.argtypes = [C.c_int32, C.c_int32, vp, vp]
+_lib.fw_fp32_fma_probe.restype = C.c_int
 _lib.fw_best_subset_read_stats.argtypes = [C.POINTER(FwRows), vp, C.POINTER(FwBestSubsetStats), vp]
 _lib.fw_best_subset_read_stats.restype = C.c_int
 _lib.fw_contour_alloc.argtypes = [vp, C.c_int32, C.c_int32, C.c_int32, C.c_int64, C.c_int32, vp, vp, vp, vp, vp,
@@ -439,3 +441,9 @@ def selector_audit(rows: Rows, s, topk: dict, *, bits=False, stream=None):
 def raw():
     """The loaded ctypes library (for callers that marshal their own arguments)."""
     return _lib
+
+
+def fp32_fma_probe(blocks: int, iters: int, out: torch.Tensor, stream=None):
+    """fw_fp32_fma_probe (a measurement aid): blocks x 256 threads x 16 chains x
+    iters fp32 FMAs; out: float32 [blocks * 256] on the device."""
+    _check(_lib.fw_fp32_fma_probe(int(blocks), int(iters), _ptr(out), _stream(stream)), "fw_fp32_fma_probe")

@@ -201,12 +201,15 @@ def test_vote_group_of_one_is_own_top_k_set(fw):
 
 def test_vote_long_rows_full_scale_sampled(fw):
     """8 KV heads x 512 query rows x 32,768 keys, budgets 2,048 / 4,096 / 8,192:
-    every group's set checked, six rows' scores."""
+    every group's set checked, the scores of 48 rows (six per head: the first,
+    the last and four drawn at random)."""
     b = workloads.long_rows(seed=0, backend="torch", device="cuda")
     s = group_budgets(b)
     _, _, v = run_vote(fw, b, s)
     H = oracle.HostRows(b)
-    pick = np.sort(np.random.default_rng(0).choice(H.num_rows, 6, replace=False))
+    rng = np.random.default_rng(0)
+    pick = np.sort(np.concatenate([[g * H.R, g * H.R + H.R - 1] for g in range(len(H.n))] +
+                                  [g * H.R + 1 + rng.choice(H.R - 2, 4, replace=False) for g in range(len(H.n))]))
     check_vote(H, s, v, rows_idx=pick)
     gap, dr = np_(v["gap"]), np_(v["dropped"])
     assert np.all(np.isfinite(gap))
