@@ -12,7 +12,7 @@
 //                  Each mass is the fast exponential times 1/Z of its row (a few
 //                  ulp): an accurate exp and a divide per (row, key) would make
 //                  this pass and the scoring pass instruction-bound.
-//   k_vote_select  per group and budget, the order key T of the s-th largest G
+//   k_vote_select  per group and budget (a block each), the order key T of the s-th largest G
 //                  (three-pass radix select over G staged in shared memory) and
 //                  the index L of the last tied key taken; the set is
 //                  {j : key(G_j) > T} + {j : key(G_j) == T, j <= L}.
@@ -113,7 +113,10 @@ __global__ void __launch_bounds__(VS_T) k_vote_select(VoteArgs a)
     __shared__ uint32_t s_digit;
     __shared__ int s_rem, s_L;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-    for (int64_t g = blockIdx.x; g < a.R.num_groups; g += gridDim.x) {
+    // a block per (group, budget): the budgets of a group select side by side
+    for (int64_t item = blockIdx.x; item < a.R.num_groups * a.nb; item += gridDim.x) {
+        const int64_t g = item / a.nb;
+        const int b = (int)(item - g * a.nb);
         const int n = a.R.n[g];
         const float *Gg = a.mass + g * (int64_t)a.R.max_n;
         const float *G = Gg;
@@ -123,7 +126,7 @@ __global__ void __launch_bounds__(VS_T) k_vote_select(VoteArgs a)
             __syncthreads();
             G = sG;
         }
-        for (int b = 0; b < a.nb; ++b) {
+        {
             const int64_t gb = g * a.nb + b;
             const int s = a.s[gb];
             uint32_t T = 0;
@@ -476,7 +479,7 @@ fw_status group_vote(const RowsDev &R, const int32_t *s, int nb, const fw_gap_ou
 
     const size_t sel_smem = a.staged ? (size_t)R.max_n * 4 : 0;
     FW_CUDA_CHECK(cudaFuncSetAttribute(k_vote_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sel_smem));
-    FW_LAUNCH(k_vote_select, (unsigned)std::min<int64_t>(R.num_groups, 1 << 20), VS_T, sel_smem, st, a);
+    FW_LAUNCH(k_vote_select, (unsigned)std::min<int64_t>(R.num_groups * nb, 1 << 20), VS_T, sel_smem, st, a);
 
     // bf16 values: the scoring as band-masked P.V products on the tensor cores
     // (the rows of a group share V and the set); otherwise one warp per row
