@@ -384,9 +384,11 @@ fw_status fw_ragged_append(void *K_store, void *V_store, const int64_t *base, co
  * cudaMalloc would synchronise the device -- and cannot provide the
  * workspace fw_contour_alloc asks for.  This variant takes the same
  * arguments minus the workspace and uses a scratch area compiled into the
- * library instead: 87,552 bytes (20 bytes per cell of the maximum plus
- * 5,632 bytes of histograms and alignment), held by every GPU that loads
- * the library until the process exits.
+ * library instead: 333,568 bytes (80 bytes per cell of the maximum: four
+ * per-cell words, a 48-byte cell record and a 16-byte slice record, no call
+ * using more than max(cells, 2048) slices; plus 5,888 bytes of histograms,
+ * radix state and alignment), held by every GPU that loads the library
+ * until the process exits.
  *   - cells must be <= FW_CONTOUR_NOALLOC_MAX_CELLS, otherwise the call
  *     returns FW_ERR_WORKSPACE and launches nothing; the other argument
  *     rules and all outputs are exactly those of fw_contour_alloc.

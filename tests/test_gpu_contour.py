@@ -51,6 +51,26 @@ def test_contour_ties(fw):
     check(fw, np.ones((6, 500), np.float32), 32, 6 * 100, 100)  # every score equal
 
 
+# Cells long enough to be split over several blocks (slices of >= 4,096
+# positions, up to 8 per cell): ragged last slices, T not a multiple of 4 (the
+# scalar path), a floor spanning slices, ties at tau across slice boundaries,
+# every score equal, and K = 0 (the floors fill the budget).
+@pytest.mark.parametrize("cells,T,floor,frac", [(3, 10000, 32, 1 / 8), (2, 33333, 32, 1 / 8),
+                                                 (5, 9999, 6000, 0.7), (2, 65536, 32, 1 / 16)])
+def test_contour_sliced(fw, cells, T, floor, frac):
+    cb = workloads.contour_cache(seed=cells + T, cells=cells, T=T, with_kv=False, floor=floor, budget_frac=frac)
+    budget = max(cells * min(floor, T), int(round(cells * T * frac)))
+    check(fw, cb.scores, floor, budget, budget // cells)
+
+
+def test_contour_sliced_ties(fw):
+    rng = np.random.default_rng(5)
+    s = (np.round(rng.lognormal(0, 1, size=(4, 9000)) * 4) / 4).astype(np.float32)
+    check(fw, s, 32, 4 * 1100, 1100)
+    check(fw, np.ones((3, 9000), np.float32), 32, 3 * 2000, 2000)
+    check(fw, s, 32, 4 * 32, 1100)  # K = 0
+
+
 def test_compaction_small(fw):
     rng = np.random.default_rng(2)
     cells, T, d = 6, 700, 128

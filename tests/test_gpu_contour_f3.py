@@ -48,6 +48,23 @@ def test_capped_small(fw, cells, T, floor, frac, cap):
     check_capped(fw, cb.scores, floor, budget, budget // cells, max(cap, min(floor, T)))
 
 
+# Cells split over several blocks: the cap's threshold found across slices,
+# a cap at the floor (no non-floor entry kept), a cap above every count.
+@pytest.mark.parametrize("cells,T,floor,frac,cap", [(3, 10000, 32, 0.3, 900), (4, 9001, 16, 0.2, 16),
+                                                    (3, 9000, 0, 0.1, 0), (2, 8000, 8, 0.5, 100000)])
+def test_capped_sliced(fw, cells, T, floor, frac, cap):
+    cb = workloads.contour_cache(seed=cells + T + 1, cells=cells, T=T, with_kv=False, floor=floor, budget_frac=frac)
+    budget = max(cells * min(floor, T), int(round(cells * T * frac)))
+    check_capped(fw, cb.scores, floor, budget, budget // cells, max(cap, min(floor, T)))
+
+
+def test_capped_sliced_ties(fw):
+    rng = np.random.default_rng(6)
+    s = (np.round(rng.lognormal(0, 1, size=(4, 9000)) * 4) / 4).astype(np.float32)
+    check_capped(fw, s, 32, 4 * 1100, 1100, 900)
+    check_capped(fw, np.ones((3, 9000), np.float32), 32, 3 * 2000, 2000, 1500)
+
+
 def test_capped_ties(fw):
     rng = np.random.default_rng(4)
     s = np.round(rng.lognormal(0, 1, size=(12, 2000)) * 4) / 4  # equal scores at both thresholds

@@ -54,7 +54,7 @@ def call_noalloc(fw, scores, floor, budget, s, out=None):
 
 def test_noalloc_matches_the_workspace_entry_point_on_consecutive_calls(fw):
     cases = []
-    for seed, (cells, T, frac) in enumerate([(64, 3000, 1 / 8), (200, 1500, 1 / 4)]):
+    for seed, (cells, T, frac) in enumerate([(64, 3000, 1 / 8), (200, 1500, 1 / 4), (24, 20000, 1 / 8)]):
         cb = workloads.contour_cache(seed=seed + 40, cells=cells, T=T, with_kv=False, budget_frac=frac)
         sc = torch.as_tensor(cb.scores).cuda()
         if seed == 1:
