@@ -507,10 +507,15 @@ def section_contour(fw, device, K, W, flush, peaks, cells=256):
     Ko = torch.empty(cb.total_budget, cb.d, dtype=torch.int16, device=device)
     Vo = torch.empty_like(Ko)
     ev = Events()
+    # outputs and workspace allocated once, as a serving loop would hold them
+    ca = fw.contour_alloc(cb.scores, floor=cb.floor, total_budget=cb.total_budget, uniform_s=cb.uniform_s)
+    cc = fw.contour_alloc_capped(cb.scores, floor=cb.floor, total_budget=cb.total_budget, uniform_s=cb.uniform_s,
+                                 cap=cb.uniform_s)
 
     def step():
         e0 = ev.start()
-        a = fw.contour_alloc(cb.scores, floor=cb.floor, total_budget=cb.total_budget, uniform_s=cb.uniform_s)
+        a = fw.contour_alloc(cb.scores, floor=cb.floor, total_budget=cb.total_budget, uniform_s=cb.uniform_s,
+                             out=ca, workspace=ca["_ws"])
         ev.stop(e0, "alloc")
         e1 = ev.start()
         fw.ragged_compact(Kc, Vc, a["offsets"], a["kept_pos"], cb.total_budget, out=(Ko, Vo))
@@ -524,7 +529,7 @@ def section_contour(fw, device, K, W, flush, peaks, cells=256):
 
     def capped_step():
         holder["c"] = fw.contour_alloc_capped(cb.scores, floor=cb.floor, total_budget=cb.total_budget,
-                                              uniform_s=cb.uniform_s, cap=cb.uniform_s)
+                                              uniform_s=cb.uniform_s, cap=cb.uniform_s, out=cc, workspace=cc["_ws"])
 
     tc_, _ = time_steps(capped_step, K, W, flush, lambda: None)
     ms_capped = tc_ / K

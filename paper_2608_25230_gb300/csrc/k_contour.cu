@@ -733,6 +733,7 @@ __global__ void __launch_bounds__(256) k_compact(const uint4 *K, const uint4 *V,
                                                  uint4 *Vo, int chunks, const int64_t *dst_base,
                                                  const int32_t *capacity, int32_t *status)
 {
+    grid_wait();  // launched chained: the offsets and positions of the kernel before are complete from here on
     const int c = blockIdx.x / chunks;
     const int chunk = blockIdx.x - c * chunks;
     const int64_t cnt = offsets[c + 1] - offsets[c];
@@ -925,10 +926,9 @@ fw_status ragged_compact(const void *K, const void *V, int cells, int T, int row
     const int chunks = (T + RPB - 1) / RPB;
     const int64_t grid = (int64_t)cells * chunks;
     if (grid >= ((int64_t)1 << 31)) return FW_ERR_UNSUPPORTED;
-    FW_LAUNCH(k_compact, (unsigned)grid, 256, 0, s, (const uint4 *)K, (const uint4 *)V, T, vec, offsets, kept_pos,
-              (uint4 *)K_out, (uint4 *)V_out, chunks, (const int64_t *)nullptr, (const int32_t *)nullptr,
-              (int32_t *)nullptr);
-    return FW_OK;
+    return launch_chained(k_compact, (unsigned)grid, 256u, 1u, s, (const uint4 *)K, (const uint4 *)V, T, vec, offsets,
+                          kept_pos, (uint4 *)K_out, (uint4 *)V_out, chunks, (const int64_t *)nullptr,
+                          (const int32_t *)nullptr, (int32_t *)nullptr);
 }
 
 fw_status ragged_compact_to(const void *K, const void *V, int cells, int T, int row_bytes, const int64_t *offsets,
@@ -939,9 +939,8 @@ fw_status ragged_compact_to(const void *K, const void *V, int cells, int T, int 
     const int chunks = (T + RPB - 1) / RPB;
     const int64_t grid = (int64_t)cells * chunks;
     if (grid >= ((int64_t)1 << 31)) return FW_ERR_UNSUPPORTED;
-    FW_LAUNCH(k_compact, (unsigned)grid, 256, 0, s, (const uint4 *)K, (const uint4 *)V, T, vec, offsets, kept_pos,
-              (uint4 *)K_store, (uint4 *)V_store, chunks, base, capacity, status);
-    return FW_OK;
+    return launch_chained(k_compact, (unsigned)grid, 256u, 1u, s, (const uint4 *)K, (const uint4 *)V, T, vec, offsets,
+                          kept_pos, (uint4 *)K_store, (uint4 *)V_store, chunks, base, capacity, status);
 }
 
 fw_status ragged_append(void *K_store, void *V_store, const int64_t *base, const int32_t *capacity, int32_t *counts,

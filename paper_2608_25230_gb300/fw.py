@@ -324,16 +324,34 @@ def sync_status(row_status: torch.Tensor, stream=None):
     return int(st), int(first.value)
 
 
-def contour_alloc(scores: torch.Tensor, *, floor: int, total_budget: int, uniform_s: int, stream=None):
+def _contour_outputs(cells, total_budget, dev, out):
+    if out is not None:  # caller-owned buffers of the same shapes, reused across calls
+        return out
+    return dict(counts=torch.empty(cells, dtype=torch.int32, device=dev),
+                offsets=torch.empty(cells + 1, dtype=torch.int64, device=dev),
+                kept_pos=torch.empty(int(total_budget), dtype=torch.int32, device=dev),
+                tau=torch.empty(1, dtype=torch.float32, device=dev),
+                dropped_uniform=torch.empty(cells, dtype=torch.float32, device=dev),
+                dropped_alloc=torch.empty(cells, dtype=torch.float32, device=dev))
+
+
+def _contour_ws(nbytes, dev, workspace):
+    if workspace is None:
+        return _ws(nbytes, dev)
+    if workspace.numel() * workspace.element_size() < nbytes:
+        raise ValueError(f"workspace holds {workspace.numel() * workspace.element_size()} bytes, {nbytes} needed")
+    return workspace
+
+
+def contour_alloc(scores: torch.Tensor, *, floor: int, total_budget: int, uniform_s: int, stream=None, out=None,
+                  workspace=None):
+    """fw_contour_alloc.  out (a dict as returned) and workspace (a uint8
+    tensor of fw_contour_alloc_workspace bytes) may be passed to reuse
+    buffers across calls."""
     dev = scores.device
     cells, T = scores.shape
-    out = dict(counts=torch.empty(cells, dtype=torch.int32, device=dev),
-               offsets=torch.empty(cells + 1, dtype=torch.int64, device=dev),
-               kept_pos=torch.empty(int(total_budget), dtype=torch.int32, device=dev),
-               tau=torch.empty(1, dtype=torch.float32, device=dev),
-               dropped_uniform=torch.empty(cells, dtype=torch.float32, device=dev),
-               dropped_alloc=torch.empty(cells, dtype=torch.float32, device=dev))
-    ws = _ws(_lib.fw_contour_alloc_workspace(cells, T), dev)
+    out = _contour_outputs(cells, total_budget, dev, out)
+    ws = _contour_ws(_lib.fw_contour_alloc_workspace(cells, T), dev, workspace)
     st = _lib.fw_contour_alloc(_ptr(scores), cells, T, int(floor), int(total_budget), int(uniform_s),
                                _ptr(out["counts"]), _ptr(out["offsets"]), _ptr(out["kept_pos"]), _ptr(out["tau"]),
                                _ptr(out["dropped_uniform"]), _ptr(out["dropped_alloc"]), _ptr(ws), ws.numel(),
@@ -344,18 +362,14 @@ def contour_alloc(scores: torch.Tensor, *, floor: int, total_budget: int, unifor
 
 
 def contour_alloc_capped(scores: torch.Tensor, *, floor: int, total_budget: int, uniform_s: int, cap: int,
-                         stream=None):
+                         stream=None, out=None, workspace=None):
     """fw_contour_alloc_capped: the allocation truncated to `cap` entries per
-    cell.  kept_pos holds total_budget entries; offsets[-1] of them are valid."""
+    cell.  kept_pos holds total_budget entries; offsets[-1] of them are valid.
+    out and workspace as for contour_alloc (the capped workspace size)."""
     dev = scores.device
     cells, T = scores.shape
-    out = dict(counts=torch.empty(cells, dtype=torch.int32, device=dev),
-               offsets=torch.empty(cells + 1, dtype=torch.int64, device=dev),
-               kept_pos=torch.empty(int(total_budget), dtype=torch.int32, device=dev),
-               tau=torch.empty(1, dtype=torch.float32, device=dev),
-               dropped_uniform=torch.empty(cells, dtype=torch.float32, device=dev),
-               dropped_alloc=torch.empty(cells, dtype=torch.float32, device=dev))
-    ws = _ws(_lib.fw_contour_alloc_capped_workspace(cells, T), dev)
+    out = _contour_outputs(cells, total_budget, dev, out)
+    ws = _contour_ws(_lib.fw_contour_alloc_capped_workspace(cells, T), dev, workspace)
     st = _lib.fw_contour_alloc_capped(_ptr(scores), cells, T, int(floor), int(total_budget), int(uniform_s), int(cap),
                                       _ptr(out["counts"]), _ptr(out["offsets"]), _ptr(out["kept_pos"]),
                                       _ptr(out["tau"]), _ptr(out["dropped_uniform"]), _ptr(out["dropped_alloc"]),
